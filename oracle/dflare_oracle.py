@@ -270,6 +270,7 @@ class DraftOracle:
         self.batch = batch
         self.store = round_bf16 if storage == "bf16" else exact
         self.rope_block = rope_block
+        self._cache = {}
         self.alpha = fusion_weights(weights["fuse_logits"], softmax=softmax_fusion)
         D = shape.n_draft_layers
         empty = np.zeros((0, shape.n_kv_heads, shape.head_dim))
@@ -277,8 +278,12 @@ class DraftOracle:
         self.ctx_v = [[empty] * D for _ in range(batch)]
 
     def _dec(self, name, idx=None):
-        a = self.w[name] if idx is None else self.w[name][idx]
-        return decode(a, self.s.dtype)
+        """float64 copy of an input weight (decoded once, then kept)."""
+        key = (name, idx)
+        if key not in self._cache:
+            a = self.w[name] if idx is None else self.w[name][idx]
+            self._cache[key] = decode(a, self.s.dtype)
+        return self._cache[key]
 
     def layer(self, i: int) -> dict:
         return {k: self._dec(k, i) for k in

@@ -1,0 +1,162 @@
+"""GB300 (sm_103a) implementation of DFlare's per-step draft path (arxiv 2606.02091).
+
+The path runs in hand-written CUDA kernels inside ``libdflare.so`` (C ABI in include/dflare.h).
+This package holds the CUDA sources (``csrc/``), the in-tree build (``build.py``) and a thin
+binding (``_lib.py`` for the raw calls, ``DFlare`` below for torch-tensor arguments). PyTorch is
+used only to own device memory and to name the CUDA stream.
+"""
+from __future__ import annotations
+
+import ctypes
+
+from . import _lib
+from ._lib import (  # noqa: F401
+    DFlareError, DFLARE_BF16, DFLARE_F32, FLAG_NO_BLOCK_ROPE, FLAG_RAW_FUSION, FLAG_SIMT_GEMM,
+    DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT, EXPORTS, WEIGHT_FIELDS, load,
+)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need_cuda(name, t, dtype=None):
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+
+
+class DFlare:
+    """One library context: the draft weights, per-layer context KV caches and work buffers.
+
+    Arguments mirror ``dflare_config`` (include/dflare.h). Device buffers passed to the calls
+    are torch CUDA tensors; calls are enqueued on the current torch stream unless one is given.
+    """
+
+    def __init__(self, *, d, n_draft_layers, n_target_layers, n_q_heads, n_kv_heads, head_dim,
+                 ffn, vocab, block, max_batch, max_ctx, max_fuse_rows, mask_token_id=None,
+                 rms_eps=1e-6, rope_theta=1e6, dtype="bf16", flags=0):
+        self._L = load()
+        self.cfg = _lib.Config(d, n_draft_layers, n_target_layers, n_q_heads, n_kv_heads, head_dim,
+                               ffn, vocab, block, max_batch, max_ctx, max_fuse_rows,
+                               vocab - 1 if mask_token_id is None else mask_token_id, rms_eps,
+                               rope_theta, DFLARE_BF16 if dtype == "bf16" else DFLARE_F32, flags)
+        self.dtype = dtype
+        self._ctx = ctypes.c_void_p()
+        _lib.check(self._L.dflare_create(ctypes.byref(self.cfg), ctypes.byref(self._ctx)))
+        self._weights = None
+        self.batch = max_batch
+
+    @classmethod
+    def from_shape(cls, shape, *, max_batch, max_ctx, max_fuse_rows, flags=0):
+        """Build from an object with the fields of ``synth.Shape``."""
+        return cls(d=shape.d, n_draft_layers=shape.n_draft_layers,
+                   n_target_layers=shape.n_target_layers, n_q_heads=shape.n_q_heads,
+                   n_kv_heads=shape.n_kv_heads, head_dim=shape.head_dim, ffn=shape.ffn,
+                   vocab=shape.vocab, block=shape.block, max_batch=max_batch, max_ctx=max_ctx,
+                   max_fuse_rows=max_fuse_rows, mask_token_id=shape.vocab - 1,
+                   rms_eps=shape.rms_eps, rope_theta=shape.rope_theta, dtype=shape.dtype,
+                   flags=flags)
+
+    def close(self):
+        if self._ctx:
+            self._L.dflare_destroy(self._ctx)
+            self._ctx = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, status):
+        return _lib.check(status, self._ctx)
+
+    @property
+    def raw(self):
+        """The dflare_ctx* handle (for direct C-ABI calls)."""
+        return self._ctx
+
+    def set_weights(self, weights: dict, stream=None):
+        """weights: name -> CUDA tensor in the layout of ``dflare_weights`` (kept alive here)."""
+        w = _lib.Weights()
+        for name in WEIGHT_FIELDS:
+            t = weights[name]
+            _need_cuda(name, t)
+            setattr(w, name, t.data_ptr())
+        self._weights = dict(weights)
+        self._check(self._L.dflare_set_weights(self._ctx, ctypes.byref(w), _stream(stream)))
+
+    def reset(self, batch: int, stream=None):
+        self._check(self._L.dflare_reset(self._ctx, batch, _stream(stream)))
+        self.batch = batch
+
+    def fuse_context(self, hidden, n_new, fused_out=None, stream=None):
+        """hidden [T][batch][n_max][d]; n_new int32 [batch] (device)."""
+        import torch
+        _need_cuda("hidden", hidden)
+        _need_cuda("n_new", n_new, torch.int32)
+        _need_cuda("fused_out", fused_out)
+        n_max = hidden.shape[2]
+        self._check(self._L.dflare_fuse_context(self._ctx, _ptr(hidden), _ptr(n_new), n_max,
+                                                _ptr(fused_out), _stream(stream)))
+
+    def draft_block(self, last_token, draft_tokens, logits_out=None, hidden_out=None, stream=None):
+        import torch
+        _need_cuda("last_token", last_token, torch.int32)
+        _need_cuda("draft_tokens", draft_tokens, torch.int32)
+        _need_cuda("logits_out", logits_out, torch.float32)
+        _need_cuda("hidden_out", hidden_out, torch.float32)
+        self._check(self._L.dflare_draft_block(self._ctx, _ptr(last_token), _ptr(draft_tokens),
+                                               _ptr(logits_out), _ptr(hidden_out), _stream(stream)))
+
+    def verify_accept(self, draft_tokens, target_argmax, accept_len, next_token, stream=None):
+        import torch
+        for n, t in (("draft_tokens", draft_tokens), ("target_argmax", target_argmax),
+                     ("accept_len", accept_len), ("next_token", next_token)):
+            _need_cuda(n, t, torch.int32)
+        self._check(self._L.dflare_verify_accept(self._ctx, _ptr(draft_tokens), _ptr(target_argmax),
+                                                 _ptr(accept_len), _ptr(next_token),
+                                                 _stream(stream)))
+
+    def read_kv(self, layer, seq, pos0, n, stream=None):
+        import torch
+        dt = torch.bfloat16 if self.dtype == "bf16" else torch.float32
+        k = torch.empty((n, self.cfg.n_kv_heads, self.cfg.head_dim), dtype=dt, device="cuda")
+        v = torch.empty_like(k)
+        self._check(self._L.dflare_read_kv(self._ctx, layer, seq, pos0, n, _ptr(k), _ptr(v),
+                                           _stream(stream)))
+        return k, v
+
+    def ctx_lens(self, stream=None):
+        arr = (ctypes.c_int32 * self.batch)()
+        self._check(self._L.dflare_ctx_lens(self._ctx, arr, _stream(stream)))
+        return list(arr)
+
+    def device_error(self, stream=None) -> int:
+        bits = ctypes.c_uint32(0)
+        st = self._L.dflare_device_error(self._ctx, ctypes.byref(bits), _stream(stream))
+        if st not in (_lib.DFLARE_OK, _lib.DFLARE_EDEVICE):
+            self._check(st)
+        return bits.value
+
+
+def synthetic_target(draft_tokens, u, r, last, step, threshold, batch, block, target_out,
+                     stream=None):
+    """Stand-in for the target's verification argmax (see dflare_synthetic_target)."""
+    L = load()
+    n_steps = u.shape[0]
+    _lib.check(L.dflare_synthetic_target(_ptr(draft_tokens), _ptr(u), _ptr(r), _ptr(last), n_steps,
+                                         _ptr(step), ctypes.c_uint32(threshold), batch, block,
+                                         _ptr(target_out), _stream(stream)))

@@ -1,0 +1,420 @@
+// Bidirectional block attention over [context ; block] (Sec. 3.2; keys/values per Eq. 4), as a
+// split-KV ("flash-decoding") pass plus a log-sum-exp combine.
+//
+// For one sequence and one KV head, the queries are the B block rows of the H_q/H_kv query
+// heads that share the head: B*G rows (64 for Qwen3 shapes, 128 for GPT-OSS) against L + B keys
+// (context keys from the cache, then the block's own K^d / V^d). Nothing is masked: every query
+// sees every key. The keys of one (sequence, head) are cut into `splits` contiguous ranges so
+// that batch x H_kv x splits CTAs cover the GPU even for a single sequence; each CTA writes an
+// unnormalised partial output with its running max and sum, and a second launch merges them
+// (no CTA ever waits for another).
+//
+// bf16 path: 64 query rows per CTA (4 warps x 16 rows), K/V tiles of 64 keys double-buffered
+// with cp.async, S = Q K^T and O += P V on mma.sync m16n8k16 with P kept in registers.
+// fp32 path: a CUDA-core version of the same split, exact fp32 products.
+#include <math.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace dfl {
+namespace {
+
+constexpr int kQT = 64;    // query rows per CTA
+constexpr int kKT = 64;    // keys per tile
+
+struct AttnArgs {
+    const void* q;        // [batch*B][d_q]
+    const void* kd;       // [batch*B][d_kv]
+    const void* vd;
+    const void* kc;       // this layer's cache [max_batch][H_kv][max_ctx][hd]
+    const void* vc;
+    const int32_t* ctx_len;
+    float* part_o;        // [batch][H_kv][q_tiles][splits][64][hd]
+    float* part_ml;       // [batch][H_kv][q_tiles][splits][64][2]
+    int B, G, hkv, d_q, d_kv, max_ctx, splits, q_tiles;
+    float scale_log2;     // log2(e) / sqrt(hd)
+};
+
+__device__ __forceinline__ void key_range(const AttnArgs& a, int b, int s, int& j0, int& j1, int& L) {
+    L = a.ctx_len[b];
+    const int total = L + a.B;
+    int per = (total + a.splits - 1) / a.splits;
+    per = (per + kKT - 1) / kKT * kKT;
+    j0 = s * per;
+    j1 = min(total, j0 + per);
+}
+
+__device__ __forceinline__ size_t part_index(const AttnArgs& a, int b, int g, int qt, int s) {
+    return (((size_t)b * a.hkv + g) * a.q_tiles + qt) * a.splits + s;
+}
+
+// ------------------------------------------------------------------ bf16, tensor cores
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
+    constexpr int LD = HD + 8;                 // padded smem row (elements)
+    extern __shared__ __align__(16) uint8_t smem[];
+    bf16* Qs = reinterpret_cast<bf16*>(smem);
+    bf16* Ks = Qs + kQT * LD;                  // [2][kKT][LD]
+    bf16* Vs = Ks + 2 * kKT * LD;              // [2][kKT][LD]
+    const int s = blockIdx.x, g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int R = a.B * a.G;
+    int j_begin, j_end, L;
+    key_range(a, b, s, j_begin, j_end, L);
+    const size_t pidx = part_index(a, b, g, qt, s);
+    float* po = a.part_o + pidx * kQT * HD;
+    float* pml = a.part_ml + pidx * kQT * 2;
+    if (j_begin >= j_end) {
+        for (int i = tid; i < kQT; i += blockDim.x) {
+            pml[2 * i] = -INFINITY;
+            pml[2 * i + 1] = 0.f;
+        }
+        return;
+    }
+    const bf16* q = static_cast<const bf16*>(a.q);
+    const bf16* kd = static_cast<const bf16*>(a.kd);
+    const bf16* vd = static_cast<const bf16*>(a.vd);
+    const bf16* kc = static_cast<const bf16*>(a.kc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
+    const bf16* vc = static_cast<const bf16*>(a.vc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
+    const uint32_t sQ = (uint32_t)__cvta_generic_to_shared(Qs);
+    const uint32_t sK = (uint32_t)__cvta_generic_to_shared(Ks);
+    const uint32_t sV = (uint32_t)__cvta_generic_to_shared(Vs);
+    constexpr int PIECES = HD / 8;             // 16-byte pieces per row
+
+    // query rows of this tile: row r -> block position r / G, head g*G + r % G
+    for (int idx = tid; idx < kQT * PIECES; idx += blockDim.x) {
+        const int r = idx / PIECES, pc = idx % PIECES;
+        const int rr = qt * kQT + r;
+        const bool ok = rr < R;
+        const int kpos = ok ? rr / a.G : 0, hh = ok ? rr % a.G : 0;
+        const bf16* src = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + pc * 8;
+        cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
+    }
+    auto load_tile = [&](int j0, int buf) {
+        for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
+            const int r = idx / PIECES, pc = idx % PIECES;
+            const int j = j0 + r;
+            const bool ok = j < j_end;
+            const bf16 *ksrc, *vsrc;
+            if (j < L) {
+                ksrc = kc + (size_t)j * HD + pc * 8;
+                vsrc = vc + (size_t)j * HD + pc * 8;
+            } else {
+                const int k = ok ? j - L : 0;
+                ksrc = kd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
+                vsrc = vd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
+            }
+            const uint32_t off = (uint32_t)((buf * kKT + r) * LD + pc * 8) * 2;
+            cp_async16(sK + off, ok ? (const void*)ksrc : (const void*)kc, ok);
+            cp_async16(sV + off, ok ? (const void*)vsrc : (const void*)vc, ok);
+        }
+    };
+    load_tile(j_begin, 0);
+    cp_commit();
+
+    float o[HD / 8][4];
+#pragma unroll
+    for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+    uint32_t qa[HD / 16][4];
+    const int n_tiles = (j_end - j_begin + kKT - 1) / kKT;
+    for (int t = 0; t < n_tiles; ++t) {
+        const int buf = t & 1;
+        if (t + 1 < n_tiles) load_tile(j_begin + (t + 1) * kKT, buf ^ 1);
+        cp_commit();
+        cp_wait<1>();
+        __syncthreads();
+        if (t == 0) {
+#pragma unroll
+            for (int kk = 0; kk < HD / 16; ++kk) {
+                const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
+                ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2],
+                        qa[kk][3]);
+            }
+        }
+        // S = Q K^T for 16 rows x 64 keys
+        float sc[8][4];
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+            sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+#pragma unroll
+            for (int kk = 0; kk < HD / 16; kk += 2) {
+                const int row = nt * 8 + (lane & 7);
+                const int col = kk * 16 + (lane >> 3) * 8;
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4(sK + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
+                mma16816(sc[nt], qa[kk], b0, b1);
+                mma16816(sc[nt], qa[kk + 1], b2, b3);
+            }
+        }
+        // mask keys past the range, scale into the log2 domain, online softmax
+        const int jt = j_begin + t * kKT;
+        float mx0 = m0, mx1 = m1;
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int j = jt + nt * 8 + (lane & 3) * 2 + e;
+                const bool ok = j < j_end;
+                sc[nt][e] = ok ? sc[nt][e] * a.scale_log2 : -INFINITY;
+                sc[nt][2 + e] = ok ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
+                mx0 = fmaxf(mx0, sc[nt][e]);
+                mx1 = fmaxf(mx1, sc[nt][2 + e]);
+            }
+        }
+#pragma unroll
+        for (int off = 1; off <= 2; off <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+        }
+        const float c0 = exp2f(m0 - mx0), c1 = exp2f(m1 - mx1);
+        m0 = mx0;
+        m1 = mx1;
+        l0 *= c0;
+        l1 *= c1;
+#pragma unroll
+        for (int i = 0; i < HD / 8; ++i) {
+            o[i][0] *= c0; o[i][1] *= c0; o[i][2] *= c1; o[i][3] *= c1;
+        }
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+            sc[nt][0] = exp2f(sc[nt][0] - m0);
+            sc[nt][1] = exp2f(sc[nt][1] - m0);
+            sc[nt][2] = exp2f(sc[nt][2] - m1);
+            sc[nt][3] = exp2f(sc[nt][3] - m1);
+            l0 += sc[nt][0] + sc[nt][1];
+            l1 += sc[nt][2] + sc[nt][3];
+        }
+        // O += P V (P from registers as the A operand; V tiles transposed by ldmatrix)
+#pragma unroll
+        for (int kk = 0; kk < kKT / 16; ++kk) {
+            uint32_t pa[4];
+            pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+            pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+            pa[2] = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+            pa[3] = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+            for (int nt = 0; nt < HD / 8; nt += 2) {
+                const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int col = (nt + (lane >> 4)) * 8;
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(sV + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
+                mma16816(o[nt], pa, b0, b1);
+                mma16816(o[nt + 1], pa, b2, b3);
+            }
+        }
+        __syncthreads();
+    }
+    cp_wait<0>();
+#pragma unroll
+    for (int off = 1; off <= 2; off <<= 1) {
+        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+    }
+    const int r0 = warp * 16 + (lane >> 2), r1 = r0 + 8;
+#pragma unroll
+    for (int nt = 0; nt < HD / 8; ++nt) {
+        const int col = nt * 8 + (lane & 3) * 2;
+        *reinterpret_cast<float2*>(po + (size_t)r0 * HD + col) = make_float2(o[nt][0], o[nt][1]);
+        *reinterpret_cast<float2*>(po + (size_t)r1 * HD + col) = make_float2(o[nt][2], o[nt][3]);
+    }
+    if ((lane & 3) == 0) {
+        pml[2 * r0] = m0;
+        pml[2 * r0 + 1] = l0;
+        pml[2 * r1] = m1;
+        pml[2 * r1 + 1] = l1;
+    }
+}
+
+// ------------------------------------------------------------------ CUDA-core path
+
+template <class T, int HD>
+__global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
+    constexpr int PER = HD / 32;
+    const int s = blockIdx.x, g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int R = a.B * a.G;
+    int j_begin, j_end, L;
+    key_range(a, b, s, j_begin, j_end, L);
+    const size_t pidx = part_index(a, b, g, qt, s);
+    float* po = a.part_o + pidx * kQT * HD;
+    float* pml = a.part_ml + pidx * kQT * 2;
+    const T* q = static_cast<const T*>(a.q);
+    const T* kd = static_cast<const T*>(a.kd);
+    const T* vd = static_cast<const T*>(a.vd);
+    const T* kc = static_cast<const T*>(a.kc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
+    const T* vc = static_cast<const T*>(a.vc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
+    for (int r = warp; r < kQT; r += 4) {
+        const int rr = qt * kQT + r;
+        float m = -INFINITY, l = 0.f, acc[PER], qv[PER];
+#pragma unroll
+        for (int e = 0; e < PER; ++e) acc[e] = 0.f;
+        if (rr < R && j_begin < j_end) {
+            const int kpos = rr / a.G, hh = rr % a.G;
+            const T* qrow = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD;
+#pragma unroll
+            for (int e = 0; e < PER; ++e) qv[e] = to_f(qrow[lane + 32 * e]);
+            for (int j = j_begin; j < j_end; ++j) {
+                const T *kr, *vr;
+                if (j < L) {
+                    kr = kc + (size_t)j * HD;
+                    vr = vc + (size_t)j * HD;
+                } else {
+                    kr = kd + ((size_t)b * a.B + (j - L)) * a.d_kv + (size_t)g * HD;
+                    vr = vd + ((size_t)b * a.B + (j - L)) * a.d_kv + (size_t)g * HD;
+                }
+                float dot = 0.f;
+#pragma unroll
+                for (int e = 0; e < PER; ++e) dot = fmaf(qv[e], to_f(kr[lane + 32 * e]), dot);
+                const float sc = warp_sum(dot) * a.scale_log2;
+                const float mn = fmaxf(m, sc);
+                const float corr = exp2f(m - mn), p = exp2f(sc - mn);
+                l = l * corr + p;
+#pragma unroll
+                for (int e = 0; e < PER; ++e) acc[e] = fmaf(p, to_f(vr[lane + 32 * e]), acc[e] * corr);
+                m = mn;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < PER; ++e) po[(size_t)r * HD + lane + 32 * e] = acc[e];
+        if (lane == 0) {
+            pml[2 * r] = m;
+            pml[2 * r + 1] = l;
+        }
+    }
+}
+
+// ------------------------------------------------------------------ combine
+
+template <class T, int HD>
+__global__ void attn_combine_kernel(const AttnArgs a, T* __restrict__ out) {
+    const int rr = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int qt = rr / kQT, r = rr % kQT;
+    const int kpos = rr / a.G, hh = rr % a.G;
+    float M = -INFINITY;
+    for (int s = 0; s < a.splits; ++s)
+        M = fmaxf(M, a.part_ml[(part_index(a, b, g, qt, s) * kQT + r) * 2]);
+    float den = 0.f, num[HD / 64 > 0 ? HD / 64 : 1];
+    constexpr int PER = HD / 64;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) num[e] = 0.f;
+    for (int s = 0; s < a.splits; ++s) {
+        const size_t pi = part_index(a, b, g, qt, s) * kQT + r;
+        const float ms = a.part_ml[pi * 2];
+        if (ms == -INFINITY) continue;
+        const float w = exp2f(ms - M);
+        den = fmaf(w, a.part_ml[pi * 2 + 1], den);
+#pragma unroll
+        for (int e = 0; e < PER; ++e) num[e] = fmaf(w, a.part_o[pi * HD + threadIdx.x + 64 * e], num[e]);
+    }
+    T* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) orow[threadIdx.x + 64 * e] = from_f<T>(num[e] / den);
+}
+
+template <int HD>
+size_t mma_smem_bytes() {
+    return (size_t)(kQT + 4 * kKT) * (HD + 8) * sizeof(bf16);
+}
+
+template <class T, int HD>
+cudaError_t run(dflare_ctx* c, const AttnArgs& a, bool mma, cudaStream_t s) {
+    dim3 grid(a.splits, a.hkv * a.q_tiles, c->batch);
+    if (mma) {
+        static bool configured = false;
+        if (!configured) {
+            cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)mma_smem_bytes<HD>());
+            if (e != cudaSuccess) return e;
+            configured = true;
+        }
+        attn_mma_kernel<HD><<<grid, 128, mma_smem_bytes<HD>(), s>>>(a);
+    } else {
+        attn_simt_kernel<T, HD><<<grid, 128, 0, s>>>(a);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    attn_combine_kernel<T, HD><<<dim3(a.B * a.G, a.hkv, c->batch), 64, 0, s>>>(a, static_cast<T*>(c->attn));
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+// Split count: about two CTAs per SM over batch x H_kv x q_tiles, and at least 128 keys per
+// split at the context capacity.
+int attention_splits(const dflare_config& g, int batch, int num_sms) {
+    const int G = g.n_q_heads / g.n_kv_heads;
+    const int q_tiles = (g.block * G + kQT - 1) / kQT;
+    const int base = batch * g.n_kv_heads * q_tiles;
+    int sp = (2 * num_sms + base - 1) / base;
+    sp = std::min(sp, (g.max_ctx + g.block + 127) / 128);
+    return std::max(1, sp);
+}
+
+cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
+    const dflare_config& g = c->cfg;
+    AttnArgs a;
+    a.q = c->q;
+    a.kd = c->kd;
+    a.vd = c->vd;
+    const size_t layer_elems = (size_t)g.max_batch * g.n_kv_heads * g.max_ctx * g.head_dim;
+    a.kc = static_cast<const uint8_t*>(c->kcache) + layer * layer_elems * c->esz;
+    a.vc = static_cast<const uint8_t*>(c->vcache) + layer * layer_elems * c->esz;
+    a.ctx_len = c->ctx_len;
+    a.part_o = c->attn_o;
+    a.part_ml = c->attn_ml;
+    a.B = g.block;
+    a.G = g.n_q_heads / g.n_kv_heads;
+    a.hkv = g.n_kv_heads;
+    a.d_q = g.n_q_heads * g.head_dim;
+    a.d_kv = g.n_kv_heads * g.head_dim;
+    a.max_ctx = g.max_ctx;
+    a.splits = attention_splits(g, c->batch, c->num_sms);
+    a.q_tiles = (a.B * a.G + kQT - 1) / kQT;
+    a.scale_log2 = 1.4426950408889634f / sqrtf((float)g.head_dim);
+    const bool f32 = g.dtype == DFLARE_F32;
+    if (g.head_dim == 64)
+        return f32 ? run<float, 64>(c, a, false, s) : run<bf16, 64>(c, a, true, s);
+    return f32 ? run<float, 128>(c, a, false, s) : run<bf16, 128>(c, a, true, s);
+}
+
+}  // namespace dfl

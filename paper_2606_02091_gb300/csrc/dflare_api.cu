@@ -1,0 +1,547 @@
+// The C ABI of libdflare (include/dflare.h): argument checks, device memory of a context, and the
+// launch sequence of the three calls of the draft path.
+#include <math.h>
+#include <string.h>
+
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+
+using namespace dfl;
+
+namespace dfl {
+int attention_splits(const dflare_config& g, int batch, int num_sms);
+}
+
+namespace {
+
+thread_local std::string g_create_error;
+
+dflare_status fail(dflare_ctx* c, dflare_status st, const std::string& m) {
+    if (c)
+        c->msg = m;
+    else
+        g_create_error = m;
+    return st;
+}
+
+#define CUDA_TRY(expr)                                                                     \
+    do {                                                                                   \
+        cudaError_t e_ = (expr);                                                           \
+        if (e_ != cudaSuccess)                                                             \
+            return fail(c, DFLARE_ECUDA, std::string(#expr) + ": " + cudaGetErrorString(e_)); \
+    } while (0)
+
+bool check_config(const dflare_config* g, std::string* why) {
+    auto bad = [&](const char* m) {
+        *why = std::string("invalid config: ") + m;
+        return false;
+    };
+    if (!g) return bad("null");
+    if (g->d < 64 || g->d % 64 != 0 || g->d > 4096) return bad("d must be a multiple of 64 in [64, 4096]");
+    if (g->n_draft_layers < 1 || g->n_draft_layers > 16) return bad("n_draft_layers must be in [1, 16]");
+    if (g->n_target_layers < 1 || g->n_target_layers > 64) return bad("n_target_layers must be in [1, 64]");
+    if (g->head_dim != 64 && g->head_dim != 128) return bad("head_dim must be 64 or 128");
+    if (g->n_kv_heads < 1 || g->n_q_heads < 1 || g->n_q_heads % g->n_kv_heads != 0)
+        return bad("n_q_heads must be a positive multiple of n_kv_heads");
+    if ((g->n_q_heads * g->head_dim) % 128 != 0 || (g->n_kv_heads * g->head_dim) % 128 != 0)
+        return bad("n_q_heads*head_dim and n_kv_heads*head_dim must be multiples of 128");
+    if (g->ffn < 64 || g->ffn % 64 != 0) return bad("ffn must be a positive multiple of 64");
+    if (g->vocab < 2) return bad("vocab must be >= 2");
+    if (g->mask_token_id < 0 || g->mask_token_id >= g->vocab) return bad("mask_token_id outside [0, vocab)");
+    if (g->block < 1 || g->block > 32) return bad("block must be in [1, 32]");
+    if (g->max_batch < 1 || g->max_batch > 64) return bad("max_batch must be in [1, 64]");
+    if (g->max_ctx < 1 || g->max_ctx > (1 << 22)) return bad("max_ctx must be in [1, 2^22]");
+    if (g->max_fuse_rows < 1 || g->max_fuse_rows > (1 << 20)) return bad("max_fuse_rows must be in [1, 2^20]");
+    if (!(g->rms_eps >= 0.f) || !isfinite(g->rms_eps)) return bad("rms_eps must be finite and >= 0");
+    if (!(g->rope_theta > 0.f) || !isfinite(g->rope_theta)) return bad("rope_theta must be finite and > 0");
+    if (g->dtype != DFLARE_BF16 && g->dtype != DFLARE_F32) return bad("dtype must be DFLARE_BF16 or DFLARE_F32");
+    if (g->flags & ~(DFLARE_FLAG_NO_BLOCK_ROPE | DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_SIMT_GEMM))
+        return bad("unknown flag bits");
+    return true;
+}
+
+template <class P>
+cudaError_t dalloc(P** p, size_t bytes, std::vector<void*>& owned) {
+    void* q = nullptr;
+    cudaError_t e = cudaMalloc(&q, bytes < 256 ? 256 : bytes);
+    if (e == cudaSuccess) {
+        owned.push_back(q);
+        *p = static_cast<P*>(q);
+    }
+    return e;
+}
+
+// Device allocations of each context, freed by dflare_destroy.
+std::mutex g_own_mu;
+std::map<const dflare_ctx*, std::vector<void*>> g_owned;
+
+void free_all(dflare_ctx* c) {
+    std::vector<void*> v;
+    {
+        std::lock_guard<std::mutex> lk(g_own_mu);
+        auto it = g_owned.find(c);
+        if (it != g_owned.end()) {
+            v.swap(it->second);
+            g_owned.erase(it);
+        }
+    }
+    for (void* p : v) cudaFree(p);
+}
+
+bool use_tc(const dflare_ctx* c) {
+    return c->cfg.dtype == DFLARE_BF16 && !(c->cfg.flags & DFLARE_FLAG_SIMT_GEMM);
+}
+
+dflare_status gemm(dflare_ctx* c, const GemmDesc& g, cudaStream_t s) {
+    cudaError_t e;
+    std::string why;
+    if (use_tc(c))
+        e = launch_gemm_tc(c, g, s, &why);
+    else
+        e = launch_gemm_simt(c, g, s);
+    if (e != cudaSuccess)
+        return fail(c, DFLARE_ECUDA, "GEMM launch: " + (why.empty() ? std::string(cudaGetErrorString(e)) : why));
+    return DFLARE_OK;
+}
+
+EpiParams epi_base(const dflare_ctx* c) {
+    EpiParams ep;
+    memset(&ep, 0, sizeof(ep));
+    const dflare_config& g = c->cfg;
+    ep.d_q = g.n_q_heads * g.head_dim;
+    ep.d_kv = g.n_kv_heads * g.head_dim;
+    ep.head_dim = g.head_dim;
+    ep.block = g.block;
+    ep.max_ctx = g.max_ctx;
+    ep.max_batch = g.max_batch;
+    ep.rope_cos = c->rope_cos;
+    ep.rope_sin = c->rope_sin;
+    return ep;
+}
+
+// Calls the user's trace hook around one launch (see dflare_set_trace).
+struct Trace {
+    dflare_ctx* c;
+    const char* name;
+    cudaStream_t s;
+    Trace(dflare_ctx* c_, const char* n, cudaStream_t s_) : c(c_), name(n), s(s_) {
+        if (c->trace_fn) c->trace_fn(c->trace_user, name, 0, s);
+    }
+    ~Trace() {
+        if (c->trace_fn) c->trace_fn(c->trace_user, name, 1, s);
+    }
+};
+
+dflare_status traced_gemm(dflare_ctx* c, const char* name, const GemmDesc& g, cudaStream_t s) {
+    Trace t(c, name, s);
+    return gemm(c, g, s);
+}
+
+const uint8_t* at(const void* base, size_t elems, size_t esz) {
+    return static_cast<const uint8_t*>(base) + elems * esz;
+}
+
+}  // namespace
+
+extern "C" {
+
+dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
+    dflare_ctx* c = nullptr;
+    std::string why;
+    if (!out) return fail(nullptr, DFLARE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (!check_config(cfg, &why)) return fail(nullptr, DFLARE_EINVAL, why);
+    c = new dflare_ctx();
+    c->cfg = *cfg;
+    c->esz = cfg->dtype == DFLARE_BF16 ? 2 : 4;
+    std::vector<void*> owned;
+    auto bail = [&](dflare_status st, const std::string& m) {
+        for (void* p : owned) cudaFree(p);
+        delete c;
+        return fail(nullptr, st, m);
+    };
+    cudaError_t e = cudaGetDevice(&c->device);
+    if (e != cudaSuccess) return bail(DFLARE_ECUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+    e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess) return bail(DFLARE_ECUDA, std::string("cudaDeviceGetAttribute: ") + cudaGetErrorString(e));
+    const dflare_config& g = c->cfg;
+    const size_t esz = c->esz;
+    const size_t d = g.d, D = g.n_draft_layers, B = g.block, V = g.vocab, F = g.ffn;
+    const size_t d_q = (size_t)g.n_q_heads * g.head_dim, d_kv = (size_t)g.n_kv_heads * g.head_dim;
+    const size_t rows = (size_t)g.max_batch * B, mrows = (size_t)g.max_batch * (B > 1 ? B - 1 : 1);
+    const size_t kv = D * g.max_batch * d_kv * (size_t)g.max_ctx;
+    // split-KV partial buffers sized for the largest batch x splits product
+    const int G = g.n_q_heads / g.n_kv_heads;
+    const int q_tiles = (g.block * G + 63) / 64;
+    size_t part_rows = 0;
+    for (int b = 1; b <= g.max_batch; ++b) {
+        const size_t r = (size_t)b * g.n_kv_heads * q_tiles * attention_splits(g, b, c->num_sms) * 64;
+        if (r > part_rows) part_rows = r;
+    }
+    c->ws_floats = (size_t)8 << 20;
+    c->tile_cnt_n = 8192;
+#define ALLOC(ptr, bytes)                                                                    \
+    do {                                                                                     \
+        e = dalloc(&(ptr), (bytes), owned);                                                  \
+        if (e != cudaSuccess)                                                                \
+            return bail(DFLARE_ENOMEM, std::string("cudaMalloc(" #ptr ", ") +               \
+                                           std::to_string((size_t)(bytes)) + "): " +           \
+                                           cudaGetErrorString(e));                           \
+    } while (0)
+    ALLOC(c->kcache, kv * esz);
+    ALLOC(c->vcache, kv * esz);
+    ALLOC(c->ctx_len, g.max_batch * sizeof(int32_t));
+    ALLOC(c->app_base, g.max_batch * sizeof(int32_t));
+    ALLOC(c->app_cnt, g.max_batch * sizeof(int32_t));
+    ALLOC(c->alpha, D * g.n_target_layers * sizeof(float));
+    ALLOC(c->fused, D * (size_t)g.max_fuse_rows * d * esz);
+    ALLOC(c->x, rows * d * sizeof(float));
+    ALLOC(c->xn, rows * d * esz);
+    ALLOC(c->q, rows * d_q * esz);
+    ALLOC(c->kd, rows * d_kv * esz);
+    ALLOC(c->vd, rows * d_kv * esz);
+    ALLOC(c->attn, rows * d_q * esz);
+    ALLOC(c->act, rows * F * esz);
+    ALLOC(c->xh, mrows * d * esz);
+    ALLOC(c->logits, mrows * V * sizeof(float));
+    ALLOC(c->attn_o, part_rows * g.head_dim * sizeof(float));
+    ALLOC(c->attn_ml, part_rows * 2 * sizeof(float));
+    ALLOC(c->ws, c->ws_floats * sizeof(float));
+    ALLOC(c->tile_cnt, (size_t)c->tile_cnt_n * sizeof(uint32_t));
+    ALLOC(c->amax_slot, mrows * sizeof(unsigned long long));
+    ALLOC(c->amax_cnt, sizeof(uint32_t));
+    const size_t half = g.head_dim / 2, npos = (size_t)g.max_ctx + B;
+    ALLOC(c->rope_cos, npos * half * sizeof(float));
+    ALLOC(c->rope_sin, npos * half * sizeof(float));
+    ALLOC(c->err, sizeof(uint32_t));
+#undef ALLOC
+    // zero what must start at zero (counters, lengths, error word, stale-row buffers)
+    struct Z { void* p; size_t n; } zs[] = {
+        {c->ctx_len, g.max_batch * sizeof(int32_t)}, {c->app_base, g.max_batch * sizeof(int32_t)},
+        {c->app_cnt, g.max_batch * sizeof(int32_t)}, {c->tile_cnt, (size_t)c->tile_cnt_n * 4},
+        {c->amax_slot, mrows * 8}, {c->amax_cnt, 4}, {c->err, 4},
+        {c->fused, D * (size_t)g.max_fuse_rows * d * esz}, {c->x, rows * d * 4}};
+    for (auto& z : zs) {
+        e = cudaMemset(z.p, 0, z.n);
+        if (e != cudaSuccess) return bail(DFLARE_ECUDA, std::string("cudaMemset: ") + cudaGetErrorString(e));
+    }
+    // rotary table: cos/sin of pos * theta^(-2j/hd), evaluated in double, stored as float
+    {
+        std::vector<float> cs(npos * half), sn(npos * half);
+        for (size_t j = 0; j < half; ++j) {
+            const double inv = pow((double)g.rope_theta, -2.0 * (double)j / (double)g.head_dim);
+            for (size_t p = 0; p < npos; ++p) {
+                const double ang = (double)p * inv;
+                cs[p * half + j] = (float)cos(ang);
+                sn[p * half + j] = (float)sin(ang);
+            }
+        }
+        e = cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice);
+        if (e == cudaSuccess) e = cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return bail(DFLARE_ECUDA, std::string("rotary table upload: ") + cudaGetErrorString(e));
+    }
+    {
+        std::lock_guard<std::mutex> lk(g_own_mu);
+        g_owned[c] = owned;
+    }
+    c->batch = g.max_batch;
+    *out = c;
+    return DFLARE_OK;
+}
+
+dflare_status dflare_destroy(dflare_ctx* c) {
+    if (!c) return DFLARE_OK;
+    cudaDeviceSynchronize();
+    free_all(c);
+    delete c;
+    return DFLARE_OK;
+}
+
+dflare_status dflare_set_weights(dflare_ctx* c, const dflare_weights* w, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!w) return fail(c, DFLARE_EINVAL, "weights is NULL");
+    const void* ptrs[] = {w->fuse_logits, w->fuse_norm, w->w_kv_ctx, w->attn_norm, w->w_qkv,
+                          w->w_o, w->mlp_norm, w->w_gate, w->w_up, w->w_down, w->final_norm,
+                          w->embed, w->lm_head};
+    const char* names[] = {"fuse_logits", "fuse_norm", "w_kv_ctx", "attn_norm", "w_qkv", "w_o",
+                           "mlp_norm", "w_gate", "w_up", "w_down", "final_norm", "embed", "lm_head"};
+    for (int i = 0; i < 13; ++i) {
+        if (!ptrs[i]) return fail(c, DFLARE_EINVAL, std::string("weight ") + names[i] + " is NULL");
+        if (reinterpret_cast<uintptr_t>(ptrs[i]) % 16 != 0)
+            return fail(c, DFLARE_EINVAL, std::string("weight ") + names[i] + " is not 16-byte aligned");
+    }
+    c->w = *w;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    CUDA_TRY(launch_fusion_alpha(c, s));
+    c->weights_set = true;
+    return DFLARE_OK;
+}
+
+dflare_status dflare_reset(dflare_ctx* c, int batch, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (batch < 1 || batch > c->cfg.max_batch)
+        return fail(c, DFLARE_ECAPACITY, "batch outside [1, max_batch]");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    c->batch = batch;
+    CUDA_TRY(cudaMemsetAsync(c->ctx_len, 0, c->cfg.max_batch * sizeof(int32_t), s));
+    return DFLARE_OK;
+}
+
+dflare_status dflare_fuse_context(dflare_ctx* c, const void* hidden, const int32_t* n_new,
+                                  int n_max, void* fused_out, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!c->weights_set) return fail(c, DFLARE_ESTATE, "dflare_set_weights has not been called");
+    if (!hidden || !n_new) return fail(c, DFLARE_EINVAL, "target_hidden or n_new is NULL");
+    if (n_max < 1) return fail(c, DFLARE_EINVAL, "n_max must be >= 1");
+    if ((long long)c->batch * n_max > c->cfg.max_fuse_rows)
+        return fail(c, DFLARE_ECAPACITY, "batch * n_max exceeds max_fuse_rows");
+    if (n_max > c->cfg.max_ctx) return fail(c, DFLARE_ECAPACITY, "n_max exceeds max_ctx");
+    if (reinterpret_cast<uintptr_t>(hidden) % 16 || reinterpret_cast<uintptr_t>(fused_out) % 16)
+        return fail(c, DFLARE_EINVAL, "target_hidden and fused_out must be 16-byte aligned");
+    const dflare_config& g = c->cfg;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    {
+        Trace t(c, "fuse_begin", s);
+        CUDA_TRY(launch_fuse_begin(c, n_new, n_max, s));
+    }
+    {
+        Trace t(c, "fuse_layers", s);
+        CUDA_TRY(launch_fuse_layers(c, hidden, n_max, fused_out, s));
+    }
+    GemmDesc gd{};
+    gd.a = c->w.w_kv_ctx;
+    gd.b = c->fused;
+    gd.groups = g.n_draft_layers;
+    gd.n = 2 * g.n_kv_heads * g.head_dim;
+    gd.k = g.d;
+    gd.m_tok = c->batch * n_max;
+    gd.b_group_rows = g.max_fuse_rows;
+    gd.ep = epi_base(c);
+    gd.ep.kind = EPI_KV_APPEND;
+    gd.ep.m_tok = gd.m_tok;
+    gd.ep.n = gd.n;
+    gd.ep.kcache = c->kcache;
+    gd.ep.vcache = c->vcache;
+    gd.ep.app_base = c->app_base;
+    gd.ep.app_cnt = c->app_cnt;
+    gd.ep.n_max = n_max;
+    return traced_gemm(c, "gemm_kv_ctx", gd, s);
+}
+
+dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32_t* draft_tokens,
+                                 float* logits_out, float* hidden_out, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!c->weights_set) return fail(c, DFLARE_ESTATE, "dflare_set_weights has not been called");
+    if (!last_token || !draft_tokens) return fail(c, DFLARE_EINVAL, "last_token or draft_tokens is NULL");
+    const dflare_config& g = c->cfg;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t esz = c->esz, d = g.d, B = g.block, F = g.ffn;
+    const size_t d_q = (size_t)g.n_q_heads * g.head_dim, d_kv = (size_t)g.n_kv_heads * g.head_dim;
+    const int rows = c->batch * g.block;
+    const size_t hid_stride = (size_t)c->batch * B * d;
+    {
+        Trace t(c, "embed", s);
+        CUDA_TRY(launch_embed(c, last_token, s));
+    }
+    if (hidden_out)
+        CUDA_TRY(cudaMemcpyAsync(hidden_out, c->x, hid_stride * 4, cudaMemcpyDeviceToDevice, s));
+    for (int i = 0; i < g.n_draft_layers; ++i) {
+        if (i > 0) {
+            Trace t(c, "rmsnorm", s);
+            CUDA_TRY(launch_rmsnorm(c, at(c->w.attn_norm, i * d, esz), rows, false, c->xn, s));
+        }
+        // Q = X~ W_Q, K^d = X~ W_K^d, V^d = X~ W_V^d with the rotary embedding (Eq. 4)
+        GemmDesc q{};
+        q.a = at(c->w.w_qkv, i * (d_q + 2 * d_kv) * d, esz);
+        q.b = c->xn;
+        q.groups = 1;
+        q.n = (int)(d_q + 2 * d_kv);
+        q.k = g.d;
+        q.m_tok = rows;
+        q.b_group_rows = rows;
+        q.ep = epi_base(c);
+        q.ep.kind = EPI_QKV;
+        q.ep.m_tok = rows;
+        q.ep.n = q.n;
+        q.ep.q = c->q;
+        q.ep.kd = c->kd;
+        q.ep.vd = c->vd;
+        q.ep.ctx_len = c->ctx_len;
+        q.ep.rope = (g.flags & DFLARE_FLAG_NO_BLOCK_ROPE) ? 0 : 1;
+        dflare_status st = traced_gemm(c, "gemm_qkv", q, s);
+        if (st != DFLARE_OK) return st;
+        // bidirectional attention over [context ; block] (Sec. 3.2)
+        {
+            Trace t(c, "attention", s);
+            CUDA_TRY(launch_attention(c, i, s));
+        }
+        // X += O W_O
+        GemmDesc o{};
+        o.a = at(c->w.w_o, i * d * d_q, esz);
+        o.b = c->attn;
+        o.groups = 1;
+        o.n = g.d;
+        o.k = (int)d_q;
+        o.m_tok = rows;
+        o.b_group_rows = rows;
+        o.ep = epi_base(c);
+        o.ep.kind = EPI_RESID;
+        o.ep.m_tok = rows;
+        o.ep.n = g.d;
+        o.ep.resid = c->x;
+        o.ep.ld_resid = g.d;
+        if ((st = traced_gemm(c, "gemm_o", o, s)) != DFLARE_OK) return st;
+        // SwiGLU MLP: X += W_down (silu(X~ W_gate) * (X~ W_up))
+        {
+            Trace t(c, "rmsnorm", s);
+            CUDA_TRY(launch_rmsnorm(c, at(c->w.mlp_norm, i * d, esz), rows, false, c->xn, s));
+        }
+        GemmDesc gu{};
+        gu.a = at(c->w.w_gate, i * F * d, esz);
+        gu.a2 = at(c->w.w_up, i * F * d, esz);
+        gu.b = c->xn;
+        gu.groups = 1;
+        gu.n = g.ffn;
+        gu.k = g.d;
+        gu.m_tok = rows;
+        gu.b_group_rows = rows;
+        gu.ep = epi_base(c);
+        gu.ep.kind = EPI_SWIGLU;
+        gu.ep.m_tok = rows;
+        gu.ep.n = g.ffn;
+        gu.ep.out = c->act;
+        gu.ep.ldo = g.ffn;
+        if ((st = traced_gemm(c, "gemm_gate_up", gu, s)) != DFLARE_OK) return st;
+        GemmDesc dn{};
+        dn.a = at(c->w.w_down, i * d * F, esz);
+        dn.b = c->act;
+        dn.groups = 1;
+        dn.n = g.d;
+        dn.k = g.ffn;
+        dn.m_tok = rows;
+        dn.b_group_rows = rows;
+        dn.ep = epi_base(c);
+        dn.ep.kind = EPI_RESID;
+        dn.ep.m_tok = rows;
+        dn.ep.n = g.d;
+        dn.ep.resid = c->x;
+        dn.ep.ld_resid = g.d;
+        if ((st = traced_gemm(c, "gemm_down", dn, s)) != DFLARE_OK) return st;
+        if (hidden_out)
+            CUDA_TRY(cudaMemcpyAsync(hidden_out + (size_t)(i + 1) * hid_stride, c->x, hid_stride * 4,
+                                     cudaMemcpyDeviceToDevice, s));
+    }
+    if (g.block < 2) return DFLARE_OK;
+    // final RMSNorm of the mask rows, LM head, greedy argmax (Sec. 3.2)
+    const int mrows = c->batch * (g.block - 1);
+    {
+        Trace t(c, "rmsnorm", s);
+        CUDA_TRY(launch_rmsnorm(c, c->w.final_norm, mrows, true, c->xh, s));
+    }
+    GemmDesc h{};
+    h.a = c->w.lm_head;
+    h.b = c->xh;
+    h.groups = 1;
+    h.n = g.vocab;
+    h.k = g.d;
+    h.m_tok = mrows;
+    h.b_group_rows = mrows;
+    h.ep = epi_base(c);
+    h.ep.kind = EPI_F32;
+    h.ep.m_tok = mrows;
+    h.ep.n = g.vocab;
+    h.ep.out = c->logits;
+    h.ep.ldo = g.vocab;
+    dflare_status st = traced_gemm(c, "gemm_lm_head", h, s);
+    if (st != DFLARE_OK) return st;
+    {
+        Trace t(c, "argmax", s);
+        CUDA_TRY(launch_argmax(c, mrows, draft_tokens, s));
+    }
+    if (logits_out)
+        CUDA_TRY(cudaMemcpyAsync(logits_out, c->logits, (size_t)mrows * g.vocab * 4,
+                                 cudaMemcpyDeviceToDevice, s));
+    return DFLARE_OK;
+}
+
+dflare_status dflare_verify_accept(dflare_ctx* c, const int32_t* draft, const int32_t* target,
+                                   int32_t* accept_len, int32_t* next_token, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!target || !accept_len || !next_token || (!draft && c->cfg.block > 1))
+        return fail(c, DFLARE_EINVAL, "a verification buffer is NULL");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    Trace t(c, "verify", s);
+    CUDA_TRY(launch_verify(c, draft, target, accept_len, next_token, s));
+    return DFLARE_OK;
+}
+
+dflare_status dflare_read_kv(dflare_ctx* c, int layer, int seq, int pos0, int n, void* k_out,
+                             void* v_out, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    const dflare_config& g = c->cfg;
+    if (layer < 0 || layer >= g.n_draft_layers || seq < 0 || seq >= g.max_batch || pos0 < 0 || n < 0 ||
+        (long long)pos0 + n > g.max_ctx)
+        return fail(c, DFLARE_EINVAL, "layer, seq or position range out of bounds");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t hd = g.head_dim, esz = c->esz;
+    for (int h = 0; h < g.n_kv_heads; ++h) {
+        const size_t row0 = (((size_t)layer * g.max_batch + seq) * g.n_kv_heads + h) * g.max_ctx + pos0;
+        if (k_out)
+            CUDA_TRY(cudaMemcpy2DAsync(static_cast<uint8_t*>(k_out) + h * hd * esz, g.n_kv_heads * hd * esz,
+                                       static_cast<uint8_t*>(c->kcache) + row0 * hd * esz, hd * esz,
+                                       hd * esz, n, cudaMemcpyDeviceToDevice, s));
+        if (v_out)
+            CUDA_TRY(cudaMemcpy2DAsync(static_cast<uint8_t*>(v_out) + h * hd * esz, g.n_kv_heads * hd * esz,
+                                       static_cast<uint8_t*>(c->vcache) + row0 * hd * esz, hd * esz,
+                                       hd * esz, n, cudaMemcpyDeviceToDevice, s));
+    }
+    return DFLARE_OK;
+}
+
+dflare_status dflare_ctx_lens(dflare_ctx* c, int32_t* host, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!host) return fail(c, DFLARE_EINVAL, "ctx_len_host is NULL");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    CUDA_TRY(cudaMemcpy(host, c->ctx_len, c->batch * sizeof(int32_t), cudaMemcpyDeviceToHost));
+    return DFLARE_OK;
+}
+
+dflare_status dflare_device_error(dflare_ctx* c, uint32_t* bits, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!bits) return fail(c, DFLARE_EINVAL, "bits_host is NULL");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    CUDA_TRY(cudaMemcpy(bits, c->err, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+    CUDA_TRY(cudaMemset(c->err, 0, sizeof(uint32_t)));
+    return *bits ? DFLARE_EDEVICE : DFLARE_OK;
+}
+
+dflare_status dflare_set_trace(dflare_ctx* c, dflare_trace_fn fn, void* user) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    c->trace_fn = fn;
+    c->trace_user = user;
+    return DFLARE_OK;
+}
+
+const char* dflare_last_error(const dflare_ctx* c) {
+    return c ? c->msg.c_str() : g_create_error.c_str();
+}
+
+dflare_status dflare_synthetic_target(const int32_t* draft, const uint32_t* u, const int32_t* r,
+                                      const int32_t* last, int n_steps, int32_t* step,
+                                      uint32_t threshold, int batch, int block, int32_t* target,
+                                      void* stream) {
+    dflare_ctx* c = nullptr;
+    if (!u || !r || !last || !step || !target || (!draft && block > 1))
+        return fail(nullptr, DFLARE_EINVAL, "a synthetic-target buffer is NULL");
+    if (n_steps < 1 || batch < 1 || block < 1 || block > 32)
+        return fail(nullptr, DFLARE_EINVAL, "n_steps, batch or block out of range");
+    CUDA_TRY(launch_synthetic_target(draft, u, r, last, n_steps, step, threshold, batch, block,
+                                     target, static_cast<cudaStream_t>(stream)));
+    return DFLARE_OK;
+}
+
+}  // extern "C"

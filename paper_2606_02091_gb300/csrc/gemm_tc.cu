@@ -1,0 +1,481 @@
+// Weight-streaming projection GEMM on the sm_103a tensor cores (tcgen05 + TMEM + TMA).
+//
+// Every projection of the draft path (context K/V of Eq. 4, Q/K^d/V^d, attention output, SwiGLU
+// gate/up and down, LM head) multiplies a few activation rows (batch * B tokens, at most a few
+// hundred) by a large weight matrix, so each weight byte is used only m_tok times: the kernel is
+// bound by HBM bandwidth while m_tok is below ~280. The layout is therefore "swap AB": the
+// 128-row UMMA M dimension runs over weight rows (output features) and the small token count is
+// the UMMA N dimension (16..256), so one instruction covers a 128 x bn x 16 piece.
+//
+// Work unit = (group, 128-feature tile, token tile, K split). A persistent grid of one CTA per SM
+// walks the units. Per CTA (192 threads):
+//   warp 4    TMA producer: 128x64 bf16 weight tile (+ the up tile for SwiGLU) and a bn x 64
+//             activation tile per stage, 128-byte swizzled, into a ring of up to 8 stages.
+//   warp 5    allocates TMEM, issues tcgen05.mma (one thread), commits stages back to the
+//             producer and finished accumulators to the epilogue; two accumulator buffers let
+//             the next unit's MMAs overlap the current unit's epilogue.
+//   warps 0-3 epilogue: tcgen05.ld of the accumulator (thread t = TMEM lane t = feature t),
+//             split-K reduction through a global workspace (the last CTA of a tile sums the
+//             partials in split order, so results are deterministic), then the fused epilogue.
+// Every wait on an mbarrier is bounded (2 s); on a timeout the CTA sets DFLARE_DEVERR_TIMEOUT,
+// stops issuing work, drains what it issued and frees its TMEM.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "epilogue.cuh"
+
+namespace dfl {
+namespace {
+
+constexpr int kThreads = 192;
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kChunk = 16;
+constexpr int kMaxStages = 8;
+constexpr uint64_t kTimeoutNs = 2000000000ull;
+constexpr int kSmemLimit = 227 * 1024;
+
+struct TcArgs {
+    int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks;
+    int bn, n_a, stages, n_bufs, tmem_cols;
+    uint32_t idesc;
+    uint32_t stage_bytes, tx_bytes;
+    float* ws;
+    uint32_t* tile_cnt;
+    uint32_t* err;
+    EpiParams ep;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: false when the CTA aborted or this wait timed out.
+__device__ __noinline__ bool bar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                      uint32_t* err) {
+    for (int i = 0; i < 128; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        for (int i = 0; i < 128; ++i)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (globaltimer_ns() - t0 > kTimeoutNs) {
+            *abort_flag = 1;
+            atomicOr(err, DFLARE_DEVERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            int z, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Shared-memory matrix descriptor: K-major operand, rows of 128 bytes, 128-byte swizzle,
+// 8-row core-matrix groups 1024 bytes apart (SBO), descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+struct Unit {
+    int group, n_tile, tok_tile, split, tile_id, kb0, kb1;
+};
+__device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
+    Unit x;
+    x.split = u % a.splits;
+    x.tile_id = u / a.splits;
+    int t = x.tile_id;
+    x.tok_tile = t % a.tok_tiles;
+    t /= a.tok_tiles;
+    x.n_tile = t % a.n_tiles;
+    x.group = t / a.n_tiles;
+    x.kb0 = x.split * a.kb_per_split;
+    x.kb1 = min(a.k_blocks, x.kb0 + a.kb_per_split);
+    return x;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+               const __grid_constant__ CUtensorMap tmB, const TcArgs args) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+    uint8_t* smem = smem_raw + pad;
+    const uint32_t sbase = raw + pad;
+    const int S = args.stages;
+    float* epi = reinterpret_cast<float*>(smem + (size_t)S * args.stage_bytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + 2 * kChunk * 128);
+    uint32_t* misc = reinterpret_cast<uint32_t*>(bars + 2 * S + 5);
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * S + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * S + 2 + b); };
+    const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
+    const uint32_t a_bytes = kBM * kBK * 2;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(tfull_bar(b), 1);
+            mbar_init(tempty_bar(b), 128);
+        }
+        mbar_init(drain_bar, 1);
+        misc[1] = 0;
+        misc[2] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 5) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(&misc[0])),
+                     "r"(args.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = misc[0];
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(&misc[1]);
+
+    if (warp == 4) {
+        if (lane == 0) {
+            // ---------------- TMA producer
+            int stage = 0;
+            uint32_t phase = 0, issued = 0, issued_phase = 0;
+            bool ok = true;
+            for (int u = blockIdx.x; u < args.n_units && ok; u += gridDim.x) {
+                const Unit x = decode_unit(args, u);
+                for (int kb = x.kb0; kb < x.kb1; ++kb) {
+                    if (!bar_wait(empty_bar(stage), phase ^ 1u, abort_flag, args.err)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t st = sbase + (uint32_t)stage * args.stage_bytes;
+                    mbar_expect_tx(full_bar(stage), args.tx_bytes);
+                    tma_load_3d(st, &tmA, kb * kBK, x.n_tile * kBM, x.group, full_bar(stage));
+                    uint32_t b_off = a_bytes;
+                    if (args.n_a == 2) {
+                        tma_load_3d(st + a_bytes, &tmA2, kb * kBK, x.n_tile * kBM, x.group,
+                                    full_bar(stage));
+                        b_off += a_bytes;
+                    }
+                    tma_load_3d(st + b_off, &tmB, kb * kBK, x.tok_tile * args.bn, x.group,
+                                full_bar(stage));
+                    issued |= 1u << stage;
+                    issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+                    if (++stage == S) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            // make sure no copy is still landing in shared memory when the CTA exits
+            for (int s = 0; s < S; ++s)
+                if (issued & (1u << s)) {
+                    volatile int never = 0;
+                    bar_wait(full_bar(s), (issued_phase >> s) & 1u, ok ? &never : abort_flag,
+                             args.err);
+                }
+        }
+    } else if (warp == 5) {
+        if (lane == 0) {
+            // ---------------- MMA issuer
+            int stage = 0, acc = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            const int acc_cols = args.n_a * args.bn;
+            bool ok = true;
+            for (int u = blockIdx.x; u < args.n_units && ok; u += gridDim.x) {
+                const Unit x = decode_unit(args, u);
+                if (!bar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, args.err)) break;
+                tc_fence_after();
+                const uint32_t d0 = tmem + (uint32_t)(acc * acc_cols);
+                for (int kb = x.kb0; kb < x.kb1; ++kb) {
+                    if (!bar_wait(full_bar(stage), phase, abort_flag, args.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t st = sbase + (uint32_t)stage * args.stage_bytes;
+                    const uint64_t da = smem_desc(st);
+                    const uint64_t da2 = smem_desc(st + a_bytes);
+                    const uint64_t db = smem_desc(st + a_bytes * args.n_a);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        const uint32_t accum = (kb > x.kb0 || k > 0) ? 1u : 0u;
+                        umma_bf16(d0, da + 2 * k, db + 2 * k, args.idesc, accum);
+                        if (args.n_a == 2)
+                            umma_bf16(d0 + args.bn, da2 + 2 * k, db + 2 * k, args.idesc, accum);
+                    }
+                    umma_commit(empty_bar(stage));
+                    if (++stage == S) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                umma_commit(tfull_bar(acc));
+                if (args.n_bufs == 2) {
+                    acc ^= 1;
+                    if (acc == 0) acc_phase ^= 1u;
+                } else {
+                    acc_phase ^= 1u;
+                }
+            }
+            // all issued MMAs complete before TMEM is released
+            umma_commit(drain_bar);
+            volatile int never = 0;
+            bar_wait(drain_bar, 0, &never, args.err);
+        }
+    } else {
+        // ---------------- epilogue warps 0-3 (thread t <-> TMEM lane t <-> feature t of a tile)
+        const int t = threadIdx.x;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        const int acc_cols = args.n_a * args.bn;
+        const int bn = args.bn, na = args.n_a;
+        for (int u = blockIdx.x; u < args.n_units; u += gridDim.x) {
+            const Unit x = decode_unit(args, u);
+            if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, args.err)) break;
+            tc_fence_after();
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
+            bool final_tile = true;
+            if (args.splits > 1) {
+                float* dst = args.ws + (size_t)(x.tile_id * args.splits + x.split) * na * bn * 128;
+                for (int a = 0; a < na; ++a)
+                    for (int c0 = 0; c0 < bn; c0 += kChunk) {
+                        float v[kChunk];
+                        tmem_ld16(taddr + (uint32_t)(a * bn + c0), v);
+#pragma unroll
+                        for (int c = 0; c < kChunk; ++c) dst[(size_t)(a * bn + c0 + c) * 128 + t] = v[c];
+                    }
+                tc_fence_before();
+                mbar_arrive(tempty_bar(acc));
+                __threadfence();
+                epi_bar();
+                if (t == 0) {
+                    const uint32_t prev = atomicAdd(&args.tile_cnt[x.tile_id], 1u);
+                    misc[2] = (prev == (uint32_t)(args.splits - 1)) ? 1u : 0u;
+                    if (prev == (uint32_t)(args.splits - 1)) args.tile_cnt[x.tile_id] = 0;
+                }
+                epi_bar();
+                final_tile = misc[2] != 0;
+                __threadfence();
+            }
+            if (final_tile) {
+                for (int c0 = 0; c0 < bn; c0 += kChunk) {
+                    for (int a = 0; a < na; ++a) {
+                        float v[kChunk];
+                        if (args.splits == 1) {
+                            tmem_ld16(taddr + (uint32_t)(a * bn + c0), v);
+                        } else {
+#pragma unroll
+                            for (int c = 0; c < kChunk; ++c) v[c] = 0.f;
+                            for (int s = 0; s < args.splits; ++s) {
+                                const float* src =
+                                    args.ws + (size_t)(x.tile_id * args.splits + s) * na * bn * 128;
+#pragma unroll
+                                for (int c = 0; c < kChunk; ++c)
+                                    v[c] += __ldcg(src + (size_t)(a * bn + c0 + c) * 128 + t);
+                            }
+                        }
+#pragma unroll
+                        for (int c = 0; c < kChunk; ++c) epi[(a * kChunk + c) * 128 + t] = v[c];
+                    }
+                    epi_bar();
+                    apply_epilogue<bf16>(args.ep, epi, kChunk, x.group, x.n_tile,
+                                         x.tok_tile * bn + c0, t);
+                    epi_bar();
+                }
+            }
+            if (args.splits == 1) {
+                tc_fence_before();
+                mbar_arrive(tempty_bar(acc));
+            }
+            if (args.n_bufs == 2) {
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1u;
+            } else {
+                acc_phase ^= 1u;
+            }
+        }
+    }
+    __syncthreads();
+    if (warp == 5) {
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(args.tmem_cols)
+                     : "memory");
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// bf16 tensor [groups][rows][k] (row stride k, group stride group_rows rows) -> 3-D tensor map
+// with a box of 64 (k) x box_rows x 1, 128-byte swizzle, zero fill outside the tensor.
+bool make_map(CUtensorMap* m, const void* base, int k, int rows, int groups, long long group_rows,
+              int box_rows) {
+    auto enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)k, (cuuint64_t)rows, (cuuint64_t)groups};
+    cuuint64_t strides[2] = {(cuuint64_t)k * 2, (cuuint64_t)group_rows * k * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kBK, (cuuint32_t)box_rows, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+               es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why) {
+    if (g.m_tok <= 0 || g.n <= 0) return cudaSuccess;
+    TcArgs a{};
+    a.n_a = g.a2 ? 2 : 1;
+    a.bn = g.m_tok <= 256 ? ((g.m_tok + 15) / 16) * 16 : 256;
+    a.tok_tiles = (g.m_tok + a.bn - 1) / a.bn;
+    a.n_tiles = (g.n + kBM - 1) / kBM;
+    a.k_blocks = (g.k + kBK - 1) / kBK;
+    const int tiles = g.groups * a.n_tiles * a.tok_tiles;
+    const int sms = c->num_sms;
+    // split-K choice: minimise waves * k-blocks per unit (+1 for the reduction), within the
+    // workspace and counter capacity
+    int best = 1;
+    long long best_cost = (long long)((tiles + sms - 1) / sms) * a.k_blocks;
+    for (int sp = 2; sp <= 16 && sp <= a.k_blocks / 2; ++sp) {
+        const int kbp = (a.k_blocks + sp - 1) / sp;
+        const int spn = (a.k_blocks + kbp - 1) / kbp;
+        const size_t need = (size_t)tiles * spn * a.n_a * a.bn * 128;
+        if (need > c->ws_floats || tiles > c->tile_cnt_n) break;
+        const long long cost = (long long)((tiles * spn + sms - 1) / sms) * kbp + 1;
+        if (cost < best_cost) {
+            best_cost = cost;
+            best = spn;
+        }
+    }
+    a.kb_per_split = (a.k_blocks + best - 1) / best;
+    a.splits = (a.k_blocks + a.kb_per_split - 1) / a.kb_per_split;
+    a.n_units = tiles * a.splits;
+    const uint32_t a_bytes = kBM * kBK * 2;
+    a.stage_bytes = a_bytes * a.n_a + (uint32_t)a.bn * kBK * 2;
+    a.tx_bytes = a.stage_bytes;
+    const int epi_bytes = 2 * kChunk * 128 * 4;
+    const int fixed = 1024 + epi_bytes + 8 * (2 * kMaxStages + 5) + 16;
+    a.stages = std::min(kMaxStages, (kSmemLimit - fixed) / (int)a.stage_bytes);
+    if (a.stages < 2) {
+        if (why) *why = "tcgen05 GEMM: tile does not fit in shared memory";
+        return cudaErrorInvalidValue;
+    }
+    const int smem = 1024 + a.stages * (int)a.stage_bytes + epi_bytes + 8 * (2 * a.stages + 5) + 16;
+    a.n_bufs = (2 * a.n_a * a.bn <= 512) ? 2 : 1;
+    int cols = 32;
+    while (cols < a.n_bufs * a.n_a * a.bn) cols <<= 1;
+    a.tmem_cols = cols;
+    // kind::f16 instruction descriptor: fp32 accumulate, bf16 A and B, both K-major,
+    // N = bn (bits 17-22, N >> 3), M = 128 (bits 24-28, M >> 4)
+    a.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(a.bn >> 3) << 17) |
+              ((uint32_t)(kBM >> 4) << 24);
+    a.ws = c->ws;
+    a.tile_cnt = c->tile_cnt;
+    a.err = c->err;
+    a.ep = g.ep;
+
+    CUtensorMap ma, ma2, mb;
+    if (!make_map(&ma, g.a, g.k, g.n, g.groups, g.n, kBM) ||
+        !make_map(&ma2, g.a2 ? g.a2 : g.a, g.k, g.n, g.groups, g.n, kBM) ||
+        !make_map(&mb, g.b, g.k, g.m_tok, g.groups, g.b_group_rows, a.bn)) {
+        if (why) *why = "cuTensorMapEncodeTiled failed (alignment or driver entry point)";
+        return cudaErrorInvalidValue;
+    }
+    static int configured = 0;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmemLimit);
+        if (e != cudaSuccess) return e;
+        configured = 1;
+    }
+    const int grid = std::min(a.n_units, sms);
+    gemm_tc_kernel<<<grid, kThreads, smem, s>>>(ma, ma2, mb, a);
+    return cudaGetLastError();
+}
+
+}  // namespace dfl

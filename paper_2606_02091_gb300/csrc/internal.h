@@ -1,0 +1,128 @@
+// Host-side internals of libdflare: the context object and the kernel launchers.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "dflare.h"
+
+namespace dfl {
+
+// Epilogue kinds of the projection GEMMs (applied to a 128-feature x token tile in fp32).
+enum EpiKind : int {
+    EPI_STORE = 0,      // out[tok][n] = acc                      (storage type)
+    EPI_F32 = 1,        // out[tok][n] = acc                      (fp32: logits)
+    EPI_RESID = 2,      // resid[tok][n] += acc                   (fp32 residual stream)
+    EPI_QKV = 3,        // Q / K^d / V^d with rotary embedding on Q and K^d at the block positions
+    EPI_KV_APPEND = 4,  // context K^t (rotated) / V^t appended to the layer's cache
+    EPI_SWIGLU = 5      // out[tok][n] = silu(gate) * up          (two accumulators)
+};
+
+struct EpiParams {
+    int kind;
+    int m_tok;             // valid token rows per group
+    int n;                 // valid output features per group
+    void* out;             // EPI_STORE / EPI_F32 / EPI_SWIGLU
+    int ldo;
+    float* resid;          // EPI_RESID
+    int ld_resid;
+    void* q;               // EPI_QKV outputs: [tok][d_q], [tok][d_kv], [tok][d_kv]
+    void* kd;
+    void* vd;
+    int d_q, d_kv;
+    const int32_t* ctx_len;  // EPI_QKV: block row k of sequence b sits at ctx_len[b] + k
+    int block;
+    void* kcache;          // EPI_KV_APPEND: [D][max_batch][H_kv][max_ctx][hd]
+    void* vcache;
+    const int32_t* app_base;  // first new position of each sequence
+    const int32_t* app_cnt;   // rows appended per sequence
+    int n_max;             // token row tok = b * n_max + r
+    int max_ctx;
+    int max_batch;
+    int head_dim;
+    const float* rope_cos;   // [positions][hd/2]
+    const float* rope_sin;
+    int rope;              // apply the rotary embedding (EPI_QKV)
+};
+
+// One projection GEMM: out = epilogue(B x A^T) per group, where A holds `groups` stacked weight
+// matrices [N][K] (row-major, out x in) and B holds the activations, m_tok valid rows per group
+// with `b_group_rows` rows between groups.
+struct GemmDesc {
+    const void* a;
+    const void* a2;        // second weight matrix for EPI_SWIGLU (up), else nullptr
+    const void* b;
+    int groups;
+    int n, k, m_tok;
+    long long b_group_rows;
+    EpiParams ep;
+};
+
+}  // namespace dfl
+
+struct dflare_ctx {
+    dflare_config cfg;
+    int device = 0;
+    int num_sms = 0;
+    int batch = 0;
+    bool weights_set = false;
+    dflare_weights w{};
+    size_t esz = 2;            // bytes per storage element
+
+    void* kcache = nullptr;    // [D][max_batch][H_kv][max_ctx][hd]
+    void* vcache = nullptr;
+    int32_t* ctx_len = nullptr;    // [max_batch]
+    int32_t* app_base = nullptr;   // [max_batch]
+    int32_t* app_cnt = nullptr;    // [max_batch]
+    float* alpha = nullptr;        // [D][T]
+    void* fused = nullptr;         // [D][max_fuse_rows][d]
+    float* x = nullptr;            // [max_batch*B][d] residual stream
+    void* xn = nullptr;            // [max_batch*B][d] normalised activations
+    void* q = nullptr;             // [max_batch*B][d_q]
+    void* kd = nullptr;            // [max_batch*B][d_kv]
+    void* vd = nullptr;
+    void* attn = nullptr;          // [max_batch*B][d_q]
+    void* act = nullptr;           // [max_batch*B][F]
+    void* xh = nullptr;            // [max_batch*(B-1)][d]
+    float* logits = nullptr;       // [max_batch*(B-1)][V]
+    float* attn_o = nullptr;       // split-KV partial outputs
+    float* attn_ml = nullptr;      // split-KV partial (max, sum)
+    int attn_splits = 1;
+    float* ws = nullptr;           // split-K workspace
+    size_t ws_floats = 0;
+    uint32_t* tile_cnt = nullptr;  // split-K arrival counters
+    int tile_cnt_n = 0;
+    unsigned long long* amax_slot = nullptr;  // packed (value, index) per logits row
+    uint32_t* amax_cnt = nullptr;
+    float* rope_cos = nullptr;     // [max_ctx + B][hd/2]
+    float* rope_sin = nullptr;
+    uint32_t* err = nullptr;       // device error word
+    dflare_trace_fn trace_fn = nullptr;
+    void* trace_user = nullptr;
+    std::string msg;
+};
+
+namespace dfl {
+
+// launchers (each returns the first CUDA error it meets)
+cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why);
+cudaError_t launch_gemm_simt(dflare_ctx* c, const GemmDesc& g, cudaStream_t s);
+cudaError_t launch_fusion_alpha(dflare_ctx* c, cudaStream_t s);
+cudaError_t launch_fuse_begin(dflare_ctx* c, const int32_t* n_new, int n_max, cudaStream_t s);
+cudaError_t launch_fuse_layers(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,
+                               cudaStream_t s);
+cudaError_t launch_embed(dflare_ctx* c, const int32_t* last_token, cudaStream_t s);
+cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gather_mask_rows,
+                           void* out, cudaStream_t s);
+cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s);
+cudaError_t launch_argmax(dflare_ctx* c, int rows, int32_t* tokens, cudaStream_t s);
+cudaError_t launch_verify(dflare_ctx* c, const int32_t* draft, const int32_t* target,
+                          int32_t* accept_len, int32_t* next_token, cudaStream_t s);
+cudaError_t launch_synthetic_target(const int32_t* draft, const uint32_t* u, const int32_t* r,
+                                    const int32_t* last, int n_steps, int32_t* step,
+                                    uint32_t threshold, int batch, int block, int32_t* target,
+                                    cudaStream_t s);
+
+}  // namespace dfl

@@ -1,0 +1,120 @@
+"""Shared test helpers: run a workload through the GPU library and through the oracle.
+
+The two sides get the same seeded input bytes from ``synth``; neither sees the other's outputs.
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+
+import oracle as O
+import synth
+
+# workloads small enough for the oracle in seconds, spanning several 128-feature tiles, ragged
+# contexts, a vocabulary that is not a multiple of 4 and both head sizes
+SMALL_HD128 = synth.Workload(
+    "small_bf16_hd128",
+    synth.Shape(d=512, n_draft_layers=3, n_target_layers=5, n_q_heads=8, n_kv_heads=2,
+                head_dim=128, ffn=1472, vocab=3001, block=16),
+    (100, 37, 250), 0.85, seed=11)
+SMALL_HD64 = synth.Workload(
+    "small_bf16_hd64",
+    synth.Shape(d=384, n_draft_layers=2, n_target_layers=4, n_q_heads=8, n_kv_heads=2,
+                head_dim=64, ffn=640, vocab=2048, block=8),
+    (65, 300), 0.75, seed=12)
+TINY = synth.preset("tiny_f32")
+
+
+def rel_err(x, y):
+    """max |x - y| / max(|y|, 1e-3 * rms(y)), elementwise denominator."""
+    x = np.asarray(x, np.float64)
+    y = np.asarray(y, np.float64)
+    rms = np.sqrt(np.mean(y * y)) if y.size else 0.0
+    den = np.maximum(np.abs(y), 1e-3 * rms)
+    den = np.where(den == 0, 1.0, den)
+    return float(np.max(np.abs(x - y) / den)) if y.size else 0.0
+
+
+def tolerance(w: synth.Workload) -> float:
+    return 2e-2 if w.shape.dtype == "bf16" else 1e-5
+
+
+def to_device(a: np.ndarray):
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if a.dtype == np.uint16:
+        t = t.view(torch.bfloat16)
+    return t.cuda()
+
+
+def storage_name(w: synth.Workload) -> str:
+    return "bf16" if w.shape.dtype == "bf16" else "exact"
+
+
+def fill_hidden(w: synth.Workload, lens, pos0=None):
+    """[T][batch][n_max][d] target states for positions pos0[b] .. pos0[b] + lens[b] - 1."""
+    s = w.shape
+    n_max = max(max(lens), 1)
+    dt = np.uint16 if s.dtype == "bf16" else np.float32
+    H = np.zeros((s.n_target_layers, w.batch, n_max, s.d), dt)
+    for b, n in enumerate(lens):
+        if n:
+            H[:, b, :n] = synth.hidden_states(w, b, 0 if pos0 is None else pos0[b], n)
+    return H
+
+
+class GpuRun:
+    """The library on one workload: weights uploaded, sequences reset."""
+
+    def __init__(self, w: synth.Workload, flags: int = 0, max_ctx: int | None = None,
+                 max_fuse_rows: int | None = None, weights: dict | None = None):
+        import torch
+        from paper_2606_02091_gb300 import DFlare
+        self.w = w
+        self.W = synth.weights(w) if weights is None else weights
+        s = w.shape
+        self.max_ctx = max_ctx or (max(w.ctx_lens) + 8 * s.block + 64)
+        mfr = max_fuse_rows or w.batch * max(max(w.ctx_lens), s.block)
+        self.lib = DFlare.from_shape(s, max_batch=w.batch, max_ctx=self.max_ctx,
+                                     max_fuse_rows=mfr, flags=flags)
+        self.dev = {k: to_device(v) for k, v in self.W.items()}
+        self.lib.set_weights(self.dev)
+        self.lib.reset(w.batch)
+        self.torch = torch
+
+    def fuse(self, lens, pos0=None, want_fused=True):
+        torch = self.torch
+        H = to_device(fill_hidden(self.w, lens, pos0))
+        n_new = torch.tensor(list(lens), dtype=torch.int32, device="cuda")
+        fused = None
+        if want_fused:
+            s = self.w.shape
+            dt = torch.bfloat16 if s.dtype == "bf16" else torch.float32
+            fused = torch.zeros((s.n_draft_layers, self.w.batch, H.shape[2], s.d), dtype=dt,
+                                device="cuda")
+        self.lib.fuse_context(H, n_new, fused)
+        return fused
+
+    def draft(self, last_tokens):
+        torch = self.torch
+        s = self.w.shape
+        bsz = self.w.batch
+        last = torch.tensor(np.asarray(last_tokens, np.int32), device="cuda")
+        toks = torch.zeros((bsz, s.block - 1), dtype=torch.int32, device="cuda")
+        logits = torch.zeros((bsz, s.block - 1, s.vocab), dtype=torch.float32, device="cuda")
+        hidden = torch.zeros((s.n_draft_layers + 1, bsz, s.block, s.d), dtype=torch.float32,
+                             device="cuda")
+        self.lib.draft_block(last, toks, logits, hidden)
+        torch.cuda.synchronize()
+        return toks.cpu().numpy(), logits.cpu().numpy(), hidden.cpu().numpy()
+
+
+def f64(t):
+    """device tensor -> float64 numpy (bf16 widened exactly)."""
+    import torch
+    return t.detach().to(torch.float64).cpu().numpy()
+
+
+def oracle_for(w: synth.Workload, W: dict, **kw):
+    return O.DraftOracle(W, w.shape, w.batch, storage=storage_name(w), **kw)

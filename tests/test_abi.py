@@ -1,0 +1,90 @@
+"""The C-ABI library: it builds, loads without a GPU, exports every entry point include/dflare.h
+declares, and rejects bad arguments on the host before touching a device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "dflare.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_02091_gb300 import build, _lib
+    build.build()
+    return _lib.load()
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dflare_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_three_calls():
+    names = _declared()
+    for n in ("dflare_fuse_context", "dflare_draft_block", "dflare_verify_accept"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    from paper_2606_02091_gb300 import _lib
+    names = _declared()
+    assert sorted(_lib.EXPORTS) == names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def _cfg(**kw):
+    from paper_2606_02091_gb300 import _lib
+    base = dict(d=256, n_draft_layers=4, n_target_layers=8, n_q_heads=4, n_kv_heads=2,
+                head_dim=64, ffn=768, vocab=4096, block=8, max_batch=1, max_ctx=256,
+                max_fuse_rows=256, mask_token_id=4095, rms_eps=1e-6, rope_theta=1e6, dtype=1,
+                flags=0)
+    base.update(kw)
+    return _lib.Config(**base)
+
+
+@pytest.mark.parametrize("field,value", [
+    ("d", 100), ("d", 0), ("d", 8192), ("n_draft_layers", 0), ("n_draft_layers", 17),
+    ("n_target_layers", 0), ("n_target_layers", 65), ("head_dim", 96), ("n_q_heads", 3),
+    ("n_kv_heads", 0), ("ffn", 100), ("vocab", 1), ("mask_token_id", 4096), ("mask_token_id", -1),
+    ("block", 0), ("block", 33), ("max_batch", 0), ("max_batch", 65), ("max_ctx", 0),
+    ("max_fuse_rows", 0), ("rms_eps", -1.0), ("rope_theta", 0.0), ("dtype", 2), ("flags", 0x80),
+])
+def test_create_rejects_bad_config_on_host(lib, field, value):
+    ctx = ctypes.c_void_p()
+    st = lib.dflare_create(ctypes.byref(_cfg(**{field: value})), ctypes.byref(ctx))
+    assert st == 1                                       # DFLARE_EINVAL, no device touched
+    assert not ctx
+    assert lib.dflare_last_error(None).startswith(b"invalid config")
+
+
+def test_create_null_out(lib):
+    assert lib.dflare_create(ctypes.byref(_cfg()), None) == 1
+
+
+def test_null_context_calls_fail(lib):
+    assert lib.dflare_reset(None, 1, None) == 1
+    assert lib.dflare_fuse_context(None, None, None, 1, None, None) == 1
+    assert lib.dflare_draft_block(None, None, None, None, None, None) == 1
+    assert lib.dflare_verify_accept(None, None, None, None, None, None) == 1
+    assert lib.dflare_destroy(None) == 0
+
+
+def test_synthetic_target_argument_checks(lib):
+    assert lib.dflare_synthetic_target(None, None, None, None, 1, None, 0, 1, 8, None, None) == 1
+
+
+def test_valid_config_without_gpu_fails_loudly(lib):
+    """With no GPU the valid config is accepted by the checks and then fails in CUDA: the
+    library never falls back to the CPU."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    ctx = ctypes.c_void_p()
+    st = lib.dflare_create(ctypes.byref(_cfg()), ctypes.byref(ctx))
+    assert st == 3                                       # DFLARE_ECUDA
+    assert not ctx

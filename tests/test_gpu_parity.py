@@ -1,0 +1,196 @@
+"""GPU path vs the CPU oracle, element by element, on the same seeded inputs (Eq. 3, Eq. 4,
+Sec. 3.2). Tolerances: fused context and hidden states within max relative error 2e-2 (bf16
+storage) or 1e-5 (fp32 storage); token ids and acceptance lengths bit-exact, except draft
+positions whose top-2 logit gap (on the oracle's logits) is below 1e-2."""
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+from tests.harness import (SMALL_HD128, SMALL_HD64, TINY, GpuRun, f64, oracle_for, rel_err,
+                           tolerance)
+
+pytestmark = pytest.mark.gpu
+GAP = 1e-2
+WORKLOADS = [TINY, SMALL_HD128, SMALL_HD64]
+
+
+@pytest.fixture(scope="module", params=WORKLOADS, ids=lambda w: w.name)
+def run(request):
+    w = request.param
+    g = GpuRun(w)
+    o = oracle_for(w, g.W)
+    fused = g.fuse(w.ctx_lens)
+    F = [o.fuse_context(b, synth.hidden_states(w, b, 0, n)) for b, n in enumerate(w.ctx_lens)]
+    return w, g, o, fused, F
+
+
+def test_fusion_matches_oracle(run):
+    w, g, o, fused, F = run
+    got = f64(fused)
+    for b, n in enumerate(w.ctx_lens):
+        err = rel_err(got[:, b, :n], F[b])
+        assert err <= tolerance(w), (b, err)
+
+
+def test_context_lengths(run):
+    w, g, o, fused, F = run
+    assert g.lib.ctx_lens() == list(w.ctx_lens)
+    assert g.lib.device_error() == 0
+
+
+def test_context_kv_matches_oracle(run):
+    w, g, o, fused, F = run
+    for b, n in enumerate(w.ctx_lens):
+        for i in range(w.shape.n_draft_layers):
+            k, v = g.lib.read_kv(i, b, 0, n)
+            assert rel_err(f64(k), o.ctx_k[b][i]) <= tolerance(w), (b, i, "K")
+            assert rel_err(f64(v), o.ctx_v[b][i]) <= tolerance(w), (b, i, "V")
+
+
+def _check_draft(w, tok, logits, hidden, o_res):
+    tol = tolerance(w)
+    for b, (ot, ol, oh) in enumerate(o_res):
+        for i in range(oh.shape[0]):
+            err = rel_err(hidden[i, b], oh[i])
+            assert err <= tol, f"seq {b} hidden after layer {i - 1}: rel err {err}"
+        assert rel_err(logits[b], ol) <= tol, f"seq {b} logits"
+        gap = O.top2_gap(ol)
+        keep = gap >= GAP
+        np.testing.assert_array_equal(tok[b][keep], ot[keep])
+        # the GPU's own argmax decision on its own logits is exact
+        np.testing.assert_array_equal(tok[b], O.argmax_lowest(logits[b]))
+
+
+def test_draft_block_matches_oracle(run):
+    w, g, o, fused, F = run
+    x_t = synth.initial_tokens(w)
+    tok, logits, hidden = g.draft(x_t)
+    o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
+    _check_draft(w, tok, logits, hidden, o_res)
+
+
+def test_steps_with_verification(run):
+    """Two more block steps: draft -> synthetic target -> prefix accept -> fuse tau positions."""
+    import torch
+    from paper_2606_02091_gb300 import synthetic_target
+    w, g, o, fused, F = run
+    s = w.shape
+    x_t = synth.initial_tokens(w).astype(np.int64)
+    thr = synth.accept_threshold(w.match_p)
+    lens = list(w.ctx_lens)
+    in_sync = [True] * w.batch
+    step_ctr = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for step in range(2):
+        tok, logits, hidden = g.draft(x_t)
+        o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
+        u, r, last = synth.target_draws(w, step)
+        tgt = torch.zeros((w.batch, s.block), dtype=torch.int32, device="cuda")
+        acc = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
+        nxt = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
+        dt = torch.tensor(tok, device="cuda")
+        step_ctr.fill_(0)
+        synthetic_target(dt, torch.tensor(u.view(np.int32), device="cuda"), torch.tensor(r, device="cuda"),
+                         torch.tensor(last, device="cuda"), step_ctr, thr, w.batch, s.block, tgt)
+        g.lib.verify_accept(dt, tgt, acc, nxt)
+        tgt_h, acc_h, nxt_h = tgt.cpu().numpy(), acc.cpu().numpy(), nxt.cpu().numpy()
+        for b in range(w.batch):
+            # integer work on identical integer inputs: exact
+            gt = O.synthetic_target(tok[b], u[0, b], r[0, b], last[0, b], thr)
+            np.testing.assert_array_equal(tgt_h[b], gt)
+            assert (acc_h[b], nxt_h[b]) == O.verify_accept(tok[b], gt)
+            if not in_sync[b]:
+                continue
+            ot, ol, oh = o_res[b]
+            if not np.array_equal(tok[b], ot):
+                assert np.all(O.top2_gap(ol)[tok[b] != ot] < GAP)
+                in_sync[b] = False      # a near-tie made the two chains diverge
+                continue
+            for i in range(oh.shape[0]):
+                assert rel_err(hidden[i, b], oh[i]) <= tolerance(w)
+        # commit tau positions on both sides and continue from the target's extra token
+        taus = [int(a) for a in acc_h]
+        g.fuse(taus, pos0=lens, want_fused=False)
+        for b in range(w.batch):
+            o.fuse_context(b, synth.hidden_states(w, b, lens[b], taus[b]))
+            lens[b] += taus[b]
+        x_t = nxt_h.astype(np.int64)
+        assert g.lib.ctx_lens() == lens
+    assert g.lib.device_error() == 0
+
+
+def test_rope_off_block_is_mask_permutation_equivariant():
+    """With block RoPE off, all mask rows have the same input, so their hidden states and logits
+    coincide (the bidirectional block has no position-dependent mask)."""
+    from paper_2606_02091_gb300 import FLAG_NO_BLOCK_ROPE
+    w = SMALL_HD64
+    g = GpuRun(w, flags=FLAG_NO_BLOCK_ROPE)
+    g.fuse(w.ctx_lens, want_fused=False)
+    tok, logits, hidden = g.draft(synth.initial_tokens(w))
+    o = oracle_for(w, g.W, rope_block=False)
+    for b, n in enumerate(w.ctx_lens):
+        o.fuse_context(b, synth.hidden_states(w, b, 0, n))
+    for b in range(w.batch):
+        for k in range(2, w.shape.block):
+            np.testing.assert_array_equal(hidden[:, b, k], hidden[:, b, 1])
+            np.testing.assert_array_equal(tok[b, k - 1], tok[b, 0])
+        ot, ol, oh = o.draft_block(b, int(synth.initial_tokens(w)[b]))
+        for i in range(oh.shape[0]):
+            assert rel_err(hidden[i, b], oh[i]) <= tolerance(w)
+
+
+def test_raw_fusion_ablation():
+    """-Softmax (Table 2): alpha = W^fuse as is."""
+    from paper_2606_02091_gb300 import FLAG_RAW_FUSION
+    w = TINY
+    g = GpuRun(w, flags=FLAG_RAW_FUSION)
+    fused = f64(g.fuse(w.ctx_lens))
+    o = oracle_for(w, g.W, softmax_fusion=False)
+    F = o.fuse_context(0, synth.hidden_states(w, 0, 0, w.ctx_lens[0]))
+    assert rel_err(fused[:, 0], F) <= tolerance(w)
+
+
+def test_empty_and_capacity_edges():
+    """n_new = 0 appends nothing; an append past max_ctx is refused by the device and flagged."""
+    import torch
+    from paper_2606_02091_gb300 import DEVERR_CAPACITY
+    w = SMALL_HD64
+    g = GpuRun(w, max_ctx=310)
+    g.fuse([0, 0], want_fused=False)
+    assert g.lib.ctx_lens() == [0, 0]
+    # an empty context still drafts (the block attends only to itself)
+    tok, logits, hidden = g.draft(synth.initial_tokens(w))
+    o = oracle_for(w, g.W)
+    for b in range(w.batch):
+        ot, ol, oh = o.draft_block(b, int(synth.initial_tokens(w)[b]))
+        for i in range(oh.shape[0]):
+            assert rel_err(hidden[i, b], oh[i]) <= tolerance(w)
+    g.fuse([65, 300], want_fused=False)
+    assert g.lib.device_error() == 0
+    g.fuse([5, 11], pos0=[65, 300], want_fused=False)       # 300 + 11 > 310: refused
+    assert g.lib.ctx_lens() == [70, 300]
+    assert g.lib.device_error() & DEVERR_CAPACITY
+    assert g.lib.device_error() == 0                       # the word was cleared
+
+
+def test_bad_token_is_flagged():
+    from paper_2606_02091_gb300 import DEVERR_TOKEN
+    w = SMALL_HD64
+    g = GpuRun(w)
+    g.fuse(w.ctx_lens, want_fused=False)
+    g.draft([w.shape.vocab + 5, -1])
+    assert g.lib.device_error() & DEVERR_TOKEN
+
+
+def test_simt_gemm_agrees_with_tcgen05_gemm():
+    """The two GEMM implementations give the same path within the bf16 tolerance."""
+    from paper_2606_02091_gb300 import FLAG_SIMT_GEMM
+    w = SMALL_HD128
+    a, b = GpuRun(w), GpuRun(w, flags=FLAG_SIMT_GEMM, weights=None)
+    a.fuse(w.ctx_lens, want_fused=False)
+    b.fuse(w.ctx_lens, want_fused=False)
+    x_t = synth.initial_tokens(w)
+    ta, la, ha = a.draft(x_t)
+    tb, lb, hb = b.draft(x_t)
+    assert rel_err(ha, hb) <= tolerance(w)
+    assert rel_err(la, lb) <= tolerance(w)
