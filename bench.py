@@ -206,7 +206,7 @@ class Cudart:
             lib = ctypes.CDLL(cands[0])
         self.lib = lib
         lib.cudaEventCreate.argtypes = [ctypes.POINTER(ctypes.c_void_p)]
-        lib.cudaEventRecord.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+        lib.cudaEventRecordWithFlags.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint]
         lib.cudaEventElapsedTime.argtypes = [ctypes.POINTER(ctypes.c_float), ctypes.c_void_p,
                                              ctypes.c_void_p]
         lib.cudaEventDestroy.argtypes = [ctypes.c_void_p]
@@ -217,7 +217,8 @@ class Cudart:
         return e
 
     def record(self, e, stream):
-        assert self.lib.cudaEventRecord(e, stream) == 0
+        # cudaEventRecordExternal: inside stream capture this becomes an event-record node
+        assert self.lib.cudaEventRecordWithFlags(e, stream, 1) == 0
 
     def elapsed(self, a, b):
         ms = ctypes.c_float()
@@ -344,7 +345,7 @@ def run_ours(args):
         step()
     torch.cuda.synchronize()
     launches_per_step = sum(KERNELS_PER_TRACE.get(k, 1) * v for k, v in counts.items()) / 3 + 1
-    L_.dflare_set_trace(lib.raw, ctypes.cast(None, P._lib.TRACE_FN), None)
+    L_.dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
 
     cs = torch.cuda.Stream()
     cs.wait_stream(torch.cuda.current_stream())
@@ -407,7 +408,7 @@ def run_ours(args):
     with torch.cuda.stream(cs):
         with torch.cuda.graph(g2, stream=cs):
             step()
-    L_.dflare_set_trace(lib.raw, ctypes.cast(None, P._lib.TRACE_FN), None)
+    L_.dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
     torch.cuda.synchronize()
     per = {}
     nb = args.breakdown_steps

@@ -10,8 +10,10 @@
 // (no CTA ever waits for another).
 //
 // bf16 path: 64 query rows per CTA (4 warps x 16 rows), K/V tiles of 64 keys double-buffered
-// with cp.async, S = Q K^T and O += P V on mma.sync m16n8k16 with P kept in registers.
+// with cp.async, S = Q K^T (bf16) and O += P V (fp16 operands) on mma.sync m16n8k16 with P
+// kept in registers.
 // fp32 path: a CUDA-core version of the same split, exact fp32 products.
+#include <cuda_fp16.h>
 #include <math.h>
 
 #include <algorithm>
@@ -82,9 +84,29 @@ __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+// P.V runs on fp16 operands: P in [0, 1] keeps 11 significant bits instead of bf16's 8, and
+// the bf16 values of V convert to fp16 exactly (except magnitudes below 2^-14, which are far
+// below anything that moves an output).
+__device__ __forceinline__ void mma16816_f16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+    __half2 h = __floats2half2_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&h);
+}
+// 8 bf16 values in shared memory -> 8 fp16 values in place
+__device__ __forceinline__ void bf16x8_to_f16x8(void* p) {
+    uint4 u = *reinterpret_cast<uint4*>(p);
+    __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&u);
+    uint4 o;
+    __half2* h = reinterpret_cast<__half2*>(&o);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __float22half2_rn(__bfloat1622float2(b[i]));
+    *reinterpret_cast<uint4*>(p) = o;
 }
 
 template <int HD>
@@ -161,6 +183,11 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
         if (t + 1 < n_tiles) load_tile(j_begin + (t + 1) * kKT, buf ^ 1);
         cp_commit();
         cp_wait<1>();
+        // this thread's copies of tile t have landed: convert its V pieces to fp16
+        for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
+            const int r = idx / PIECES, pc = idx % PIECES;
+            bf16x8_to_f16x8(Vs + (buf * kKT + r) * LD + pc * 8);
+        }
         __syncthreads();
         if (t == 0) {
 #pragma unroll
@@ -227,18 +254,18 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
 #pragma unroll
         for (int kk = 0; kk < kKT / 16; ++kk) {
             uint32_t pa[4];
-            pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
-            pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
-            pa[2] = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            pa[3] = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+            pa[0] = pack_f16(sc[2 * kk][0], sc[2 * kk][1]);
+            pa[1] = pack_f16(sc[2 * kk][2], sc[2 * kk][3]);
+            pa[2] = pack_f16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+            pa[3] = pack_f16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
 #pragma unroll
             for (int nt = 0; nt < HD / 8; nt += 2) {
                 const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 const int col = (nt + (lane >> 4)) * 8;
                 uint32_t b0, b1, b2, b3;
                 ldsm_x4_t(sV + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
-                mma16816(o[nt], pa, b0, b1);
-                mma16816(o[nt + 1], pa, b2, b3);
+                mma16816_f16(o[nt], pa, b0, b1);
+                mma16816_f16(o[nt + 1], pa, b2, b3);
             }
         }
         __syncthreads();
@@ -379,14 +406,16 @@ cudaError_t run(dflare_ctx* c, const AttnArgs& a, bool mma, cudaStream_t s) {
 
 }  // namespace
 
-// Split count: about two CTAs per SM over batch x H_kv x q_tiles, and at least 128 keys per
-// split at the context capacity.
-int attention_splits(const dflare_config& g, int batch, int num_sms) {
+// Split count: enough CTAs for about two per SM over batch x H_kv x q_tiles, but no split
+// shorter than 256 keys at the host's upper bound of the context length (each split writes a
+// 64 x hd fp32 partial, as many bytes as 128 keys of K and V). The device derives the actual
+// ranges from the true lengths, so a stale bound (e.g. a replayed graph) only costs speed.
+int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub) {
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + kQT - 1) / kQT;
     const int base = batch * g.n_kv_heads * q_tiles;
     int sp = (2 * num_sms + base - 1) / base;
-    sp = std::min(sp, (g.max_ctx + g.block + 127) / 128);
+    sp = std::min(sp, (len_ub + g.block + 255) / 256);
     return std::max(1, sp);
 }
 
@@ -408,7 +437,7 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
     a.d_q = g.n_q_heads * g.head_dim;
     a.d_kv = g.n_kv_heads * g.head_dim;
     a.max_ctx = g.max_ctx;
-    a.splits = attention_splits(g, c->batch, c->num_sms);
+    a.splits = attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
     a.q_tiles = (a.B * a.G + kQT - 1) / kQT;
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)g.head_dim);
     const bool f32 = g.dtype == DFLARE_F32;

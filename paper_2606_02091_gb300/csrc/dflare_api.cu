@@ -3,6 +3,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <map>
 #include <mutex>
 #include <string>
@@ -13,7 +14,7 @@
 using namespace dfl;
 
 namespace dfl {
-int attention_splits(const dflare_config& g, int batch, int num_sms);
+int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub);
 }
 
 namespace {
@@ -179,7 +180,7 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     const int q_tiles = (g.block * G + 63) / 64;
     size_t part_rows = 0;
     for (int b = 1; b <= g.max_batch; ++b) {
-        const size_t r = (size_t)b * g.n_kv_heads * q_tiles * attention_splits(g, b, c->num_sms) * 64;
+        const size_t r = (size_t)b * g.n_kv_heads * q_tiles * attention_splits(g, b, c->num_sms, g.max_ctx) * 64;
         if (r > part_rows) part_rows = r;
     }
     c->ws_floats = (size_t)8 << 20;
@@ -287,6 +288,7 @@ dflare_status dflare_reset(dflare_ctx* c, int batch, void* stream) {
         return fail(c, DFLARE_ECAPACITY, "batch outside [1, max_batch]");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     c->batch = batch;
+    c->ctx_ub = 0;
     CUDA_TRY(cudaMemsetAsync(c->ctx_len, 0, c->cfg.max_batch * sizeof(int32_t), s));
     return DFLARE_OK;
 }
@@ -329,6 +331,7 @@ dflare_status dflare_fuse_context(dflare_ctx* c, const void* hidden, const int32
     gd.ep.app_base = c->app_base;
     gd.ep.app_cnt = c->app_cnt;
     gd.ep.n_max = n_max;
+    c->ctx_ub = std::min(c->cfg.max_ctx, c->ctx_ub + n_max);
     return traced_gemm(c, "gemm_kv_ctx", gd, s);
 }
 

@@ -67,6 +67,7 @@ struct dflare_ctx {
     int device = 0;
     int num_sms = 0;
     int batch = 0;
+    int ctx_ub = 0;            // host-side upper bound of every sequence's context length
     bool weights_set = false;
     dflare_weights w{};
     size_t esz = 2;            // bytes per storage element

@@ -27,13 +27,20 @@ TINY = synth.preset("tiny_f32")
 
 
 def rel_err(x, y):
-    """max |x - y| / max(|y|, 1e-3 * rms(y)), elementwise denominator."""
+    """Max relative error: max_i |x_i - y_i| / max(|y_i|, rms(y)).
+
+    Elements at least as large as the tensor's RMS are compared relative to themselves; smaller
+    ones relative to the RMS, so that an element that is near zero because of cancellation does
+    not turn rounding noise of the order of its neighbours into a huge ratio.
+    """
     x = np.asarray(x, np.float64)
     y = np.asarray(y, np.float64)
-    rms = np.sqrt(np.mean(y * y)) if y.size else 0.0
-    den = np.maximum(np.abs(y), 1e-3 * rms)
+    if not y.size:
+        return 0.0
+    rms = float(np.sqrt(np.mean(y * y)))
+    den = np.maximum(np.abs(y), rms)
     den = np.where(den == 0, 1.0, den)
-    return float(np.max(np.abs(x - y) / den)) if y.size else 0.0
+    return float(np.max(np.abs(x - y) / den))
 
 
 def tolerance(w: synth.Workload) -> float:
