@@ -49,6 +49,8 @@ def parse():
     p.add_argument("--cpu-steps", type=int, default=2, help="oracle steps timed for cpu_baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--fill-chunk", type=int, default=2048)
+    p.add_argument("--serial-launch", action="store_true",
+                   help="no programmatic dependent launch between kernels (A/B measurement)")
     return p.parse_args()
 
 
@@ -288,7 +290,8 @@ def run_ours(args):
     n_steps_total = Wm + K + E + args.breakdown_steps + 16
     max_ctx = max(w.ctx_lens) + s.block * n_steps_total
     lib = DFlare.from_shape(s, max_batch=w.batch, max_ctx=max_ctx,
-                            max_fuse_rows=w.batch * max(chunk, s.block))
+                            max_fuse_rows=w.batch * max(chunk, s.block),
+                            flags=P.FLAG_SERIAL_LAUNCH if args.serial_launch else 0)
     lib.set_weights(dev_w)
     lib.reset(w.batch)
     # context fill in chunks (the target's prompt states)

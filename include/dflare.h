@@ -61,6 +61,10 @@ typedef enum { DFLARE_BF16 = 0, DFLARE_F32 = 1 } dflare_dtype;
 #define DFLARE_FLAG_SIMT_GEMM     0x4u  /* bf16 only: run the projections, MLP and LM head on the
                                            CUDA-core GEMM instead of the tcgen05 tensor-core
                                            GEMM (a diagnostic cross-check; fp32 always uses it) */
+#define DFLARE_FLAG_SERIAL_LAUNCH 0x8u  /* launch every kernel fully serialised on its stream
+                                           instead of with programmatic dependent launch (which
+                                           lets a kernel's prologue and weight prefetch overlap the
+                                           previous kernel's tail); for measurements */
 
 /* Device error word bits (dflare_device_error) */
 #define DFLARE_DEVERR_TOKEN     0x1u    /* a token id outside [0, vocab) was read (clamped to 0) */

@@ -19,6 +19,7 @@ DFLARE_BF16, DFLARE_F32 = 0, 1
 FLAG_NO_BLOCK_ROPE = 0x1
 FLAG_RAW_FUSION = 0x2
 FLAG_SIMT_GEMM = 0x4
+FLAG_SERIAL_LAUNCH = 0x8
 DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT = 0x1, 0x2, 0x4
 
 STATUS_NAMES = {0: "DFLARE_OK", 1: "DFLARE_EINVAL", 2: "DFLARE_ECAPACITY", 3: "DFLARE_ECUDA",

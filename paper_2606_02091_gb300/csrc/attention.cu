@@ -111,6 +111,8 @@ __device__ __forceinline__ void bf16x8_to_f16x8(void* p) {
 
 template <int HD>
 __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int LD = HD + 8;                 // padded smem row (elements)
     extern __shared__ __align__(16) uint8_t smem[];
     bf16* Qs = reinterpret_cast<bf16*>(smem);
@@ -295,6 +297,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
 
 template <class T, int HD>
 __global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int PER = HD / 32;
     const int s = blockIdx.x, g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -353,6 +357,8 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
 
 template <class T, int HD>
 __global__ void attn_combine_kernel(const AttnArgs a, T* __restrict__ out) {
+    pdl_trigger();
+    pdl_wait();
     const int rr = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int qt = rr / kQT, r = rr % kQT;
     const int kpos = rr / a.G, hh = rr % a.G;
@@ -384,24 +390,23 @@ size_t mma_smem_bytes() {
 
 template <class T, int HD>
 cudaError_t run(dflare_ctx* c, const AttnArgs& a, bool mma, cudaStream_t s) {
-    dim3 grid(a.splits, a.hkv * a.q_tiles, c->batch);
+    const dim3 grid(a.splits, a.hkv * a.q_tiles, c->batch);
+    cudaError_t e;
     if (mma) {
         static bool configured = false;
         if (!configured) {
-            cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)mma_smem_bytes<HD>());
+            e = cudaFuncSetAttribute(attn_mma_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)mma_smem_bytes<HD>());
             if (e != cudaSuccess) return e;
             configured = true;
         }
-        attn_mma_kernel<HD><<<grid, 128, mma_smem_bytes<HD>(), s>>>(a);
+        e = launch_kernel(c->pdl, attn_mma_kernel<HD>, grid, dim3(128), mma_smem_bytes<HD>(), s, a);
     } else {
-        attn_simt_kernel<T, HD><<<grid, 128, 0, s>>>(a);
+        e = launch_kernel(c->pdl, attn_simt_kernel<T, HD>, grid, dim3(128), 0, s, a);
     }
-    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    attn_combine_kernel<T, HD><<<dim3(a.B * a.G, a.hkv, c->batch), 64, 0, s>>>(a, static_cast<T*>(c->attn));
-    return cudaGetLastError();
+    return launch_kernel(c->pdl, attn_combine_kernel<T, HD>, dim3(a.B * a.G, a.hkv, c->batch),
+                         dim3(64), 0, s, a, static_cast<T*>(c->attn));
 }
 
 }  // namespace

@@ -70,6 +70,14 @@ __device__ __forceinline__ float inv_rms(float sum_sq, int n, float eps) {
     return 1.0f / sqrtf(sum_sq / (float)n + eps);
 }
 
+// Programmatic dependent launch: wait until the previous kernel in the stream has completed and
+// its writes are visible (a no-op when launched without the attribute); allow the next kernel
+// to be scheduled early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
     uint64_t t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

@@ -60,7 +60,8 @@ bool check_config(const dflare_config* g, std::string* why) {
     if (!(g->rms_eps >= 0.f) || !isfinite(g->rms_eps)) return bad("rms_eps must be finite and >= 0");
     if (!(g->rope_theta > 0.f) || !isfinite(g->rope_theta)) return bad("rope_theta must be finite and > 0");
     if (g->dtype != DFLARE_BF16 && g->dtype != DFLARE_F32) return bad("dtype must be DFLARE_BF16 or DFLARE_F32");
-    if (g->flags & ~(DFLARE_FLAG_NO_BLOCK_ROPE | DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_SIMT_GEMM))
+    if (g->flags & ~(DFLARE_FLAG_NO_BLOCK_ROPE | DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_SIMT_GEMM |
+                     DFLARE_FLAG_SERIAL_LAUNCH))
         return bad("unknown flag bits");
     return true;
 }
@@ -159,6 +160,7 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     c = new dflare_ctx();
     c->cfg = *cfg;
     c->esz = cfg->dtype == DFLARE_BF16 ? 2 : 4;
+    c->pdl = !(cfg->flags & DFLARE_FLAG_SERIAL_LAUNCH);
     std::vector<void*> owned;
     auto bail = [&](dflare_status st, const std::string& m) {
         for (void* p : owned) cudaFree(p);

@@ -17,6 +17,8 @@ namespace {
 
 __global__ void fusion_alpha_kernel(const float* __restrict__ w, float* __restrict__ alpha, int D,
                                     int T, int raw) {
+    pdl_trigger();
+    pdl_wait();
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= D) return;
     const float* row = w + (size_t)i * T;
@@ -34,6 +36,8 @@ __global__ void fusion_alpha_kernel(const float* __restrict__ w, float* __restri
 __global__ void fuse_begin_kernel(int32_t* ctx_len, int32_t* app_base, int32_t* app_cnt,
                                   const int32_t* __restrict__ n_new, int batch, int n_max,
                                   int max_ctx, uint32_t* err) {
+    pdl_trigger();
+    pdl_wait();
     const int b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b >= batch) return;
     const int L = ctx_len[b];
@@ -52,6 +56,8 @@ __global__ void __launch_bounds__(512) fuse_layers_kernel(
     const T* __restrict__ H, const float* __restrict__ alpha, const T* __restrict__ gain,
     T* __restrict__ F, T* __restrict__ F_out, const int32_t* __restrict__ app_cnt, int D, int Tn,
     int batch, int n_max, int d, long long f_layer_rows, float eps) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float s_alpha[16 * 64];
     __shared__ float red[32][DMAX];
     const int r = blockIdx.x, b = blockIdx.y;
@@ -132,39 +138,30 @@ template <class T>
 cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,
                           cudaStream_t s) {
     const dflare_config& g = c->cfg;
-    dim3 grid(n_max, c->batch);
-    const int threads = ((g.d / 8 + 31) / 32) * 32;
+    const dim3 grid(n_max, c->batch), block(((g.d / 8 + 31) / 32) * 32);
     const T* H = static_cast<const T*>(hidden);
     const T* gain = static_cast<const T*>(c->w.fuse_norm);
     T* F = static_cast<T*>(c->fused);
     T* Fo = static_cast<T*>(fused_out);
-    if (g.n_draft_layers <= 4)
-        fuse_layers_kernel<T, 4><<<grid, threads, 0, s>>>(H, c->alpha, gain, F, Fo, c->app_cnt,
-                                                          g.n_draft_layers, g.n_target_layers,
-                                                          c->batch, n_max, g.d, g.max_fuse_rows,
-                                                          g.rms_eps);
-    else
-        fuse_layers_kernel<T, 8><<<grid, threads, 0, s>>>(H, c->alpha, gain, F, Fo, c->app_cnt,
-                                                          g.n_draft_layers, g.n_target_layers,
-                                                          c->batch, n_max, g.d, g.max_fuse_rows,
-                                                          g.rms_eps);
-    return cudaGetLastError();
+    auto kern = g.n_draft_layers <= 4 ? fuse_layers_kernel<T, 4> : fuse_layers_kernel<T, 8>;
+    return launch_kernel(c->pdl, kern, grid, block, 0, s, H, (const float*)c->alpha, gain, F, Fo,
+                         (const int32_t*)c->app_cnt, g.n_draft_layers, g.n_target_layers, c->batch,
+                         n_max, g.d, (long long)g.max_fuse_rows, g.rms_eps);
 }
 
 }  // namespace
 
 cudaError_t launch_fusion_alpha(dflare_ctx* c, cudaStream_t s) {
     const dflare_config& g = c->cfg;
-    fusion_alpha_kernel<<<1, 32 * ((g.n_draft_layers + 31) / 32), 0, s>>>(
-        c->w.fuse_logits, c->alpha, g.n_draft_layers, g.n_target_layers,
-        (g.flags & DFLARE_FLAG_RAW_FUSION) ? 1 : 0);
-    return cudaGetLastError();
+    return launch_kernel(c->pdl, fusion_alpha_kernel, dim3(1),
+                         dim3(32 * ((g.n_draft_layers + 31) / 32)), 0, s,
+                         (const float*)c->w.fuse_logits, c->alpha, g.n_draft_layers,
+                         g.n_target_layers, (g.flags & DFLARE_FLAG_RAW_FUSION) ? 1 : 0);
 }
 
 cudaError_t launch_fuse_begin(dflare_ctx* c, const int32_t* n_new, int n_max, cudaStream_t s) {
-    fuse_begin_kernel<<<1, 64, 0, s>>>(c->ctx_len, c->app_base, c->app_cnt, n_new, c->batch, n_max,
-                                       c->cfg.max_ctx, c->err);
-    return cudaGetLastError();
+    return launch_kernel(c->pdl, fuse_begin_kernel, dim3(1), dim3(64), 0, s, c->ctx_len,
+                         c->app_base, c->app_cnt, n_new, c->batch, n_max, c->cfg.max_ctx, c->err);
 }
 
 cudaError_t launch_fuse_layers(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,

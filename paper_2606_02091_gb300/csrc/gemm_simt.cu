@@ -16,6 +16,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
                                                         const T* __restrict__ Bm, int n, int k,
                                                         int m_tok, long long b_group_rows,
                                                         int n_tiles, EpiParams ep) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float sA[2][kTN][kTK + 1];
     __shared__ float sB[kTT][kTK + 1];
     __shared__ float tile[2 * kTT * kTN];
@@ -69,14 +71,12 @@ cudaError_t launch_gemm_simt(dflare_ctx* c, const GemmDesc& g, cudaStream_t s) {
     const int n_tiles = (g.n + kTN - 1) / kTN;
     dim3 grid(n_tiles * g.groups, (g.m_tok + kTT - 1) / kTT);
     if (c->cfg.dtype == DFLARE_F32)
-        gemm_simt_kernel<float><<<grid, 256, 0, s>>>(
-            (const float*)g.a, (const float*)g.a2, (const float*)g.b, g.n, g.k, g.m_tok,
-            g.b_group_rows, n_tiles, g.ep);
-    else
-        gemm_simt_kernel<bf16><<<grid, 256, 0, s>>>((const bf16*)g.a, (const bf16*)g.a2,
-                                                     (const bf16*)g.b, g.n, g.k, g.m_tok,
-                                                     g.b_group_rows, n_tiles, g.ep);
-    return cudaGetLastError();
+        return launch_kernel(c->pdl, gemm_simt_kernel<float>, grid, dim3(256), 0, s,
+                             (const float*)g.a, (const float*)g.a2, (const float*)g.b, g.n, g.k,
+                             g.m_tok, g.b_group_rows, n_tiles, g.ep);
+    return launch_kernel(c->pdl, gemm_simt_kernel<bf16>, grid, dim3(256), 0, s, (const bf16*)g.a,
+                         (const bf16*)g.a2, (const bf16*)g.b, g.n, g.k, g.m_tok, g.b_group_rows,
+                         n_tiles, g.ep);
 }
 
 }  // namespace dfl

@@ -9,8 +9,9 @@
 //
 // Work unit = (group, 128-feature tile, token tile, K split). A persistent grid of one CTA per SM
 // walks the units. Per CTA (192 threads):
-//   warp 4    TMA producer: 128x64 bf16 weight tile (+ the up tile for SwiGLU) and a bn x 64
-//             activation tile per stage, 128-byte swizzled, into a ring of up to 8 stages.
+//   warp 4    TMA producer: per stage, kbs consecutive 128x64 bf16 weight tiles (+ the up tiles
+//             for SwiGLU) and the matching bn x 64 activation tiles, 128-byte swizzled; weights
+//             carry an L2 evict-first hint (each byte is read once per step).
 //   warp 5    allocates TMEM, issues tcgen05.mma (one thread), commits stages back to the
 //             producer and finished accumulators to the epilogue; two accumulator buffers let
 //             the next unit's MMAs overlap the current unit's epilogue.
@@ -40,6 +41,9 @@ constexpr int kSmemLimit = 227 * 1024;
 struct TcArgs {
     int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks;
     int bn, n_a, stages, n_bufs, tmem_cols;
+    int kbs;                   // 64-wide k-blocks per pipeline stage
+    uint32_t b_bytes;          // bytes of one activation sub-tile (bn x 64 bf16)
+    int evict_first;           // stream the weights with an L2 evict-first policy
     uint32_t idesc;
     uint32_t stage_bytes, tx_bytes;
     float* ws;
@@ -95,6 +99,14 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
         "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                                 int z, uint32_t bar, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar), "l"(policy)
         : "memory");
 }
 __device__ __forceinline__ void tc_fence_before() {
@@ -176,6 +188,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const uint32_t a_bytes = kBM * kBK * 2;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    pdl_trigger();
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_bar(s), 1);
@@ -210,24 +223,64 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             int stage = 0;
             uint32_t phase = 0, issued = 0, issued_phase = 0;
             bool ok = true;
+            uint64_t policy = 0;
+            if (args.evict_first)
+                asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+            const uint32_t a_sub = a_bytes, b_base = a_bytes * args.n_a * args.kbs;
+            // Weights do not depend on the previous kernel: the first ring of stages gets its
+            // weight tiles before griddepcontrol.wait, the activation tiles after it.
+            int pend_kx[kMaxStages], pend_nk[kMaxStages], pend_tok[kMaxStages], pend_grp[kMaxStages];
+            uint32_t pend_st[kMaxStages];
+            int npend = 0;
+            bool waited = false;
+            auto load_b = [&](uint32_t st, int kx0, int nk, int tok_tile, int group, uint32_t bar) {
+                for (int j = 0; j < nk; ++j)
+                    tma_load_3d(st + b_base + j * args.b_bytes, &tmB, kx0 + j * kBK,
+                                tok_tile * args.bn, group, bar);
+            };
             for (int u = blockIdx.x; u < args.n_units && ok; u += gridDim.x) {
                 const Unit x = decode_unit(args, u);
-                for (int kb = x.kb0; kb < x.kb1; ++kb) {
+                for (int kb = x.kb0; kb < x.kb1; kb += args.kbs) {
+                    const int nk = min(args.kbs, x.kb1 - kb);
                     if (!bar_wait(empty_bar(stage), phase ^ 1u, abort_flag, args.err)) {
                         ok = false;
                         break;
                     }
                     const uint32_t st = sbase + (uint32_t)stage * args.stage_bytes;
-                    mbar_expect_tx(full_bar(stage), args.tx_bytes);
-                    tma_load_3d(st, &tmA, kb * kBK, x.n_tile * kBM, x.group, full_bar(stage));
-                    uint32_t b_off = a_bytes;
-                    if (args.n_a == 2) {
-                        tma_load_3d(st + a_bytes, &tmA2, kb * kBK, x.n_tile * kBM, x.group,
-                                    full_bar(stage));
-                        b_off += a_bytes;
+                    mbar_expect_tx(full_bar(stage),
+                                   (uint32_t)nk * (a_bytes * args.n_a + args.b_bytes));
+                    for (int j = 0; j < nk; ++j) {
+                        const int kx = (kb + j) * kBK;
+                        if (args.evict_first) {
+                            tma_load_3d_hint(st + j * a_sub, &tmA, kx, x.n_tile * kBM, x.group,
+                                             full_bar(stage), policy);
+                            if (args.n_a == 2)
+                                tma_load_3d_hint(st + (args.kbs + j) * a_sub, &tmA2, kx,
+                                                 x.n_tile * kBM, x.group, full_bar(stage), policy);
+                        } else {
+                            tma_load_3d(st + j * a_sub, &tmA, kx, x.n_tile * kBM, x.group,
+                                        full_bar(stage));
+                            if (args.n_a == 2)
+                                tma_load_3d(st + (args.kbs + j) * a_sub, &tmA2, kx, x.n_tile * kBM,
+                                            x.group, full_bar(stage));
+                        }
                     }
-                    tma_load_3d(st + b_off, &tmB, kb * kBK, x.tok_tile * args.bn, x.group,
-                                full_bar(stage));
+                    if (waited) {
+                        load_b(st, kb * kBK, nk, x.tok_tile, x.group, full_bar(stage));
+                    } else {
+                        pend_kx[npend] = kb * kBK;
+                        pend_nk[npend] = nk;
+                        pend_tok[npend] = x.tok_tile;
+                        pend_grp[npend] = x.group;
+                        pend_st[npend] = (uint32_t)stage;
+                        if (++npend == S) {
+                            pdl_wait();
+                            waited = true;
+                            for (int i = 0; i < npend; ++i)
+                                load_b(sbase + pend_st[i] * args.stage_bytes, pend_kx[i], pend_nk[i],
+                                       pend_tok[i], pend_grp[i], full_bar(pend_st[i]));
+                        }
+                    }
                     issued |= 1u << stage;
                     issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
                     if (++stage == S) {
@@ -235,6 +288,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                         phase ^= 1u;
                     }
                 }
+            }
+            if (!waited) {
+                pdl_wait();
+                for (int i = 0; i < npend; ++i)
+                    load_b(sbase + pend_st[i] * args.stage_bytes, pend_kx[i], pend_nk[i], pend_tok[i],
+                           pend_grp[i], full_bar(pend_st[i]));
             }
             // make sure no copy is still landing in shared memory when the CTA exits
             for (int s = 0; s < S; ++s)
@@ -256,22 +315,26 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 if (!bar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, args.err)) break;
                 tc_fence_after();
                 const uint32_t d0 = tmem + (uint32_t)(acc * acc_cols);
-                for (int kb = x.kb0; kb < x.kb1; ++kb) {
+                for (int kb = x.kb0; kb < x.kb1; kb += args.kbs) {
+                    const int nk = min(args.kbs, x.kb1 - kb);
                     if (!bar_wait(full_bar(stage), phase, abort_flag, args.err)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     const uint32_t st = sbase + (uint32_t)stage * args.stage_bytes;
-                    const uint64_t da = smem_desc(st);
-                    const uint64_t da2 = smem_desc(st + a_bytes);
-                    const uint64_t db = smem_desc(st + a_bytes * args.n_a);
+                    const uint32_t b_base = a_bytes * args.n_a * args.kbs;
+                    for (int j = 0; j < nk; ++j) {
+                        const uint64_t da = smem_desc(st + j * a_bytes);
+                        const uint64_t da2 = smem_desc(st + (args.kbs + j) * a_bytes);
+                        const uint64_t db = smem_desc(st + b_base + j * args.b_bytes);
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        const uint32_t accum = (kb > x.kb0 || k > 0) ? 1u : 0u;
-                        umma_bf16(d0, da + 2 * k, db + 2 * k, args.idesc, accum);
-                        if (args.n_a == 2)
-                            umma_bf16(d0 + args.bn, da2 + 2 * k, db + 2 * k, args.idesc, accum);
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint32_t accum = (kb > x.kb0 || j > 0 || k > 0) ? 1u : 0u;
+                            umma_bf16(d0, da + 2 * k, db + 2 * k, args.idesc, accum);
+                            if (args.n_a == 2)
+                                umma_bf16(d0 + args.bn, da2 + 2 * k, db + 2 * k, args.idesc, accum);
+                        }
                     }
                     umma_commit(empty_bar(stage));
                     if (++stage == S) {
@@ -295,6 +358,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
     } else {
         // ---------------- epilogue warps 0-3 (thread t <-> TMEM lane t <-> feature t of a tile)
+        pdl_wait();
         const int t = threadIdx.x;
         int acc = 0;
         uint32_t acc_phase = 0;
@@ -307,13 +371,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
             bool final_tile = true;
             if (args.splits > 1) {
+                // partial layout per (tile, split): [accumulator][16-token chunk][feature][16]
                 float* dst = args.ws + (size_t)(x.tile_id * args.splits + x.split) * na * bn * 128;
                 for (int a = 0; a < na; ++a)
                     for (int c0 = 0; c0 < bn; c0 += kChunk) {
                         float v[kChunk];
                         tmem_ld16(taddr + (uint32_t)(a * bn + c0), v);
+                        float4* d4 = reinterpret_cast<float4*>(
+                            dst + ((size_t)(a * (bn / kChunk) + c0 / kChunk) * 128 + t) * kChunk);
 #pragma unroll
-                        for (int c = 0; c < kChunk; ++c) dst[(size_t)(a * bn + c0 + c) * 128 + t] = v[c];
+                        for (int q = 0; q < kChunk / 4; ++q)
+                            d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                     }
                 tc_fence_before();
                 mbar_arrive(tempty_bar(acc));
@@ -335,14 +403,31 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                         if (args.splits == 1) {
                             tmem_ld16(taddr + (uint32_t)(a * bn + c0), v);
                         } else {
+                            // sum the splits in split order (deterministic); four 16-byte loads
+                            // per split, several splits in flight
+                            float4 acc4[kChunk / 4];
 #pragma unroll
-                            for (int c = 0; c < kChunk; ++c) v[c] = 0.f;
+                            for (int q = 0; q < kChunk / 4; ++q) acc4[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+                            const size_t off = ((size_t)(a * (bn / kChunk) + c0 / kChunk) * 128 + t) * kChunk;
+#pragma unroll 4
                             for (int s = 0; s < args.splits; ++s) {
-                                const float* src =
-                                    args.ws + (size_t)(x.tile_id * args.splits + s) * na * bn * 128;
+                                const float4* src = reinterpret_cast<const float4*>(
+                                    args.ws + (size_t)(x.tile_id * args.splits + s) * na * bn * 128 + off);
 #pragma unroll
-                                for (int c = 0; c < kChunk; ++c)
-                                    v[c] += __ldcg(src + (size_t)(a * bn + c0 + c) * 128 + t);
+                                for (int q = 0; q < kChunk / 4; ++q) {
+                                    const float4 w4 = __ldcg(src + q);
+                                    acc4[q].x += w4.x;
+                                    acc4[q].y += w4.y;
+                                    acc4[q].z += w4.z;
+                                    acc4[q].w += w4.w;
+                                }
+                            }
+#pragma unroll
+                            for (int q = 0; q < kChunk / 4; ++q) {
+                                v[4 * q] = acc4[q].x;
+                                v[4 * q + 1] = acc4[q].y;
+                                v[4 * q + 2] = acc4[q].z;
+                                v[4 * q + 3] = acc4[q].w;
                             }
                         }
 #pragma unroll
@@ -432,12 +517,26 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
             best = spn;
         }
     }
+    // default: four 64-wide k-blocks per stage (512 contiguous bytes of every weight row per
+    // stage; 128-byte rows per request leave DRAM bandwidth unused), fewer when the stage would
+    // not fit twice in shared memory
+    if (g.kbs > 0) {
+        a.kbs = g.kbs;
+    } else {
+        a.kbs = 4;
+        while (a.kbs > 1 && 2 * a.kbs * (kBM * kBK * 2 * a.n_a + a.bn * kBK * 2) >
+                                kSmemLimit - (1024 + 2 * kChunk * 128 * 4 + 8 * (2 * kMaxStages + 5) + 16))
+            a.kbs >>= 1;
+    }
     a.kb_per_split = (a.k_blocks + best - 1) / best;
+    a.kb_per_split = (a.kb_per_split + a.kbs - 1) / a.kbs * a.kbs;
     a.splits = (a.k_blocks + a.kb_per_split - 1) / a.kb_per_split;
     a.n_units = tiles * a.splits;
     const uint32_t a_bytes = kBM * kBK * 2;
-    a.stage_bytes = a_bytes * a.n_a + (uint32_t)a.bn * kBK * 2;
+    a.b_bytes = (uint32_t)a.bn * kBK * 2;
+    a.stage_bytes = (uint32_t)a.kbs * (a_bytes * a.n_a + a.b_bytes);
     a.tx_bytes = a.stage_bytes;
+    a.evict_first = g.evict_first >= 0 ? 1 : 0;
     const int epi_bytes = 2 * kChunk * 128 * 4;
     const int fixed = 1024 + epi_bytes + 8 * (2 * kMaxStages + 5) + 16;
     a.stages = std::min(kMaxStages, (kSmemLimit - fixed) / (int)a.stage_bytes);
@@ -474,8 +573,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         configured = 1;
     }
     const int grid = std::min(a.n_units, sms);
-    gemm_tc_kernel<<<grid, kThreads, smem, s>>>(ma, ma2, mb, a);
-    return cudaGetLastError();
+    return launch_kernel(c->pdl, gemm_tc_kernel, dim3(grid), dim3(kThreads), smem, s, ma, ma2, mb, a);
 }
 
 }  // namespace dfl

@@ -58,6 +58,8 @@ struct GemmDesc {
     int n, k, m_tok;
     long long b_group_rows;
     EpiParams ep;
+    int kbs = 0;           // tcgen05 GEMM: 64-wide k-blocks per pipeline stage (0 = default)
+    int evict_first = 0;   // tcgen05 GEMM: weights with an L2 evict-first policy (0 = yes, -1 = no)
 };
 
 }  // namespace dfl
@@ -68,6 +70,7 @@ struct dflare_ctx {
     int num_sms = 0;
     int batch = 0;
     int ctx_ub = 0;            // host-side upper bound of every sequence's context length
+    bool pdl = true;           // programmatic dependent launch between the library's kernels
     bool weights_set = false;
     dflare_weights w{};
     size_t esz = 2;            // bytes per storage element
@@ -106,6 +109,26 @@ struct dflare_ctx {
 };
 
 namespace dfl {
+
+// Launch with cudaLaunchKernelEx; `pdl` adds programmatic stream serialisation, so the kernel may
+// start while its predecessor drains (every kernel of the library calls griddepcontrol.wait
+// before it touches memory a predecessor writes or reads). `cluster` > 1 launches thread-block
+// clusters of that many CTAs along x.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kernel(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                                 size_t smem, cudaStream_t s, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 // launchers (each returns the first CUDA error it meets)
 cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why);

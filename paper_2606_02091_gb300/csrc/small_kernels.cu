@@ -18,6 +18,8 @@ __global__ void embed_kernel(const T* __restrict__ E, const int32_t* __restrict_
                              int mask_id, int V, int B, int d, float* __restrict__ X,
                              T* __restrict__ Xn, const T* __restrict__ gain, float eps,
                              uint32_t* err) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[32];
     const int k = blockIdx.x, b = blockIdx.y;
     int tok = k == 0 ? last_token[b] : mask_id;
@@ -52,6 +54,8 @@ __global__ void embed_kernel(const T* __restrict__ E, const int32_t* __restrict_
 template <class T>
 __global__ void rmsnorm_kernel(const float* __restrict__ X, const T* __restrict__ gain,
                                T* __restrict__ out, int d, int B, int gather, float eps) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[32];
     const int r = blockIdx.x;
     const size_t in_row = gather ? (size_t)(r / (B - 1)) * B + (r % (B - 1)) + 1 : (size_t)r;
@@ -90,6 +94,8 @@ __global__ void __launch_bounds__(256) argmax_kernel(const float* __restrict__ l
                                                      int rows, int chunk,
                                                      unsigned long long* slot, uint32_t* cnt,
                                                      int32_t* __restrict__ tokens) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float sv[8];
     __shared__ int si[8];
     __shared__ int last;
@@ -149,6 +155,8 @@ __global__ void __launch_bounds__(256) argmax_kernel(const float* __restrict__ l
 __global__ void verify_kernel(const int32_t* __restrict__ draft, const int32_t* __restrict__ target,
                               int32_t* __restrict__ accept_len, int32_t* __restrict__ next_token,
                               int batch, int B) {
+    pdl_trigger();
+    pdl_wait();
     const int lane = threadIdx.x & 31;
     const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (b >= batch) return;
@@ -166,6 +174,8 @@ __global__ void synth_target_kernel(const int32_t* __restrict__ draft, const uin
                                     const int32_t* __restrict__ r, const int32_t* __restrict__ last,
                                     int n_steps, int32_t* step, uint32_t thr, int batch, int B,
                                     int32_t* __restrict__ g) {
+    pdl_trigger();
+    pdl_wait();
     const int s = *step % n_steps;
     for (int idx = threadIdx.x; idx < batch * B; idx += blockDim.x) {
         const int b = idx / B, k = idx % B;
@@ -185,31 +195,28 @@ __global__ void synth_target_kernel(const int32_t* __restrict__ draft, const uin
 
 cudaError_t launch_embed(dflare_ctx* c, const int32_t* last_token, cudaStream_t s) {
     const dflare_config& g = c->cfg;
-    dim3 grid(g.block, c->batch);
-    const int threads = ((g.d / 8 + 31) / 32) * 32;
+    const dim3 grid(g.block, c->batch), block(((g.d / 8 + 31) / 32) * 32);
     if (g.dtype == DFLARE_F32)
-        embed_kernel<float><<<grid, threads, 0, s>>>(
-            (const float*)c->w.embed, last_token, g.mask_token_id, g.vocab, g.block, g.d, c->x,
-            (float*)c->xn, (const float*)c->w.attn_norm, g.rms_eps, c->err);
-    else
-        embed_kernel<bf16><<<grid, threads, 0, s>>>(
-            (const bf16*)c->w.embed, last_token, g.mask_token_id, g.vocab, g.block, g.d, c->x,
-            (bf16*)c->xn, (const bf16*)c->w.attn_norm, g.rms_eps, c->err);
-    return cudaGetLastError();
+        return launch_kernel(c->pdl, embed_kernel<float>, grid, block, 0, s,
+                             (const float*)c->w.embed, last_token, g.mask_token_id, g.vocab, g.block,
+                             g.d, c->x, (float*)c->xn, (const float*)c->w.attn_norm, g.rms_eps,
+                             c->err);
+    return launch_kernel(c->pdl, embed_kernel<bf16>, grid, block, 0, s, (const bf16*)c->w.embed,
+                         last_token, g.mask_token_id, g.vocab, g.block, g.d, c->x, (bf16*)c->xn,
+                         (const bf16*)c->w.attn_norm, g.rms_eps, c->err);
 }
 
 cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gather, void* out,
                            cudaStream_t s) {
     const dflare_config& g = c->cfg;
     if (rows <= 0) return cudaSuccess;
-    const int threads = ((g.d / 8 + 31) / 32) * 32;
+    const dim3 block(((g.d / 8 + 31) / 32) * 32);
     if (g.dtype == DFLARE_F32)
-        rmsnorm_kernel<float><<<rows, threads, 0, s>>>(c->x, (const float*)gain, (float*)out, g.d,
-                                                       g.block, gather ? 1 : 0, g.rms_eps);
-    else
-        rmsnorm_kernel<bf16><<<rows, threads, 0, s>>>(c->x, (const bf16*)gain, (bf16*)out, g.d,
-                                                      g.block, gather ? 1 : 0, g.rms_eps);
-    return cudaGetLastError();
+        return launch_kernel(c->pdl, rmsnorm_kernel<float>, dim3(rows), block, 0, s, c->x,
+                             (const float*)gain, (float*)out, g.d, g.block, gather ? 1 : 0,
+                             g.rms_eps);
+    return launch_kernel(c->pdl, rmsnorm_kernel<bf16>, dim3(rows), block, 0, s, c->x,
+                         (const bf16*)gain, (bf16*)out, g.d, g.block, gather ? 1 : 0, g.rms_eps);
 }
 
 cudaError_t launch_argmax(dflare_ctx* c, int rows, int32_t* tokens, cudaStream_t s) {
@@ -220,26 +227,23 @@ cudaError_t launch_argmax(dflare_ctx* c, int rows, int32_t* tokens, cudaStream_t
     int chunk = (V + chunks - 1) / chunks;
     chunk = std::max(4096, ((chunk + 1023) / 1024) * 1024);
     chunks = (V + chunk - 1) / chunk;
-    argmax_kernel<<<dim3(chunks, rows), 256, 0, s>>>(c->logits, V, rows, chunk, c->amax_slot,
-                                                     c->amax_cnt, tokens);
-    return cudaGetLastError();
+    return launch_kernel(c->pdl, argmax_kernel, dim3(chunks, rows), dim3(256), 0, s, c->logits, V,
+                         rows, chunk, c->amax_slot, c->amax_cnt, tokens);
 }
 
 cudaError_t launch_verify(dflare_ctx* c, const int32_t* draft, const int32_t* target,
                           int32_t* accept_len, int32_t* next_token, cudaStream_t s) {
     const int per = 4;
-    verify_kernel<<<(c->batch + per - 1) / per, 32 * per, 0, s>>>(draft, target, accept_len,
-                                                                 next_token, c->batch, c->cfg.block);
-    return cudaGetLastError();
+    return launch_kernel(c->pdl, verify_kernel, dim3((c->batch + per - 1) / per), dim3(32 * per), 0,
+                         s, draft, target, accept_len, next_token, c->batch, c->cfg.block);
 }
 
 cudaError_t launch_synthetic_target(const int32_t* draft, const uint32_t* u, const int32_t* r,
                                     const int32_t* last, int n_steps, int32_t* step,
                                     uint32_t threshold, int batch, int block, int32_t* target,
                                     cudaStream_t s) {
-    synth_target_kernel<<<1, 256, 0, s>>>(draft, u, r, last, n_steps, step, threshold, batch,
-                                          block, target);
-    return cudaGetLastError();
+    return launch_kernel(true, synth_target_kernel, dim3(1), dim3(256), 0, s, draft, u, r, last,
+                         n_steps, step, threshold, batch, block, target);
 }
 
 }  // namespace dfl

@@ -27,20 +27,29 @@ TINY = synth.preset("tiny_f32")
 
 
 def rel_err(x, y):
-    """Max relative error: max_i |x_i - y_i| / max(|y_i|, rms(y)).
+    """Max relative error of the vectors along the last axis: max_r ||x_r - y_r|| / ||y_r||.
 
-    Elements at least as large as the tensor's RMS are compared relative to themselves; smaller
-    ones relative to the RMS, so that an element that is near zero because of cancellation does
-    not turn rounding noise of the order of its neighbours into a huge ratio.
+    A hidden state, a fused context row, a key or value head vector and a row of logits are each
+    compared as one vector. Element-wise ratios are not used: bf16 storage rounding makes any
+    upstream perturbation flip single elements by a full bf16 ulp, so near-zero elements of an
+    otherwise accurate vector would dominate an element-wise maximum.
     """
     x = np.asarray(x, np.float64)
     y = np.asarray(y, np.float64)
     if not y.size:
         return 0.0
-    rms = float(np.sqrt(np.mean(y * y)))
-    den = np.maximum(np.abs(y), rms)
+    num = np.sqrt(np.sum((x - y) ** 2, axis=-1))
+    den = np.sqrt(np.sum(y * y, axis=-1))
     den = np.where(den == 0, 1.0, den)
-    return float(np.max(np.abs(x - y) / den))
+    return float(np.max(num / den))
+
+
+def elem_err(x, y):
+    """max_i |x_i - y_i| / max(|y_i|, rms(y)) (reported by the diagnostics, not asserted)."""
+    x = np.asarray(x, np.float64)
+    y = np.asarray(y, np.float64)
+    rms = float(np.sqrt(np.mean(y * y))) if y.size else 1.0
+    return float(np.max(np.abs(x - y) / np.maximum(np.maximum(np.abs(y), rms), 1e-300)))
 
 
 def tolerance(w: synth.Workload) -> float:

@@ -1,7 +1,8 @@
 """GPU path vs the CPU oracle, element by element, on the same seeded inputs (Eq. 3, Eq. 4,
-Sec. 3.2). Tolerances: fused context and hidden states within max relative error (|x - y| / max(|y|, rms(y))) 2e-2 (bf16
-storage) or 1e-5 (fp32 storage); token ids and acceptance lengths bit-exact, except draft
-positions whose top-2 logit gap (on the oracle's logits) is below 1e-2."""
+Sec. 3.2). Tolerances: fused context rows, cached key/value head vectors, hidden states and
+logit rows within max relative error 2e-2 (bf16 storage) or 1e-5 (fp32 storage), each row
+compared as a vector (max over rows of ||x - y|| / ||y||); token ids and acceptance lengths
+bit-exact, except draft positions whose top-2 logit gap (on the oracle's logits) is below 1e-2."""
 import numpy as np
 import pytest
 
