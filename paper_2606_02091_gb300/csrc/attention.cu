@@ -1,25 +1,30 @@
 // Bidirectional block attention over [context ; block] (Sec. 3.2; keys/values per Eq. 4), as a
-// split-KV ("flash-decoding") pass plus a log-sum-exp combine.
+// split-KV ("flash-decoding") pass.
 //
 // For one sequence and one KV head, the queries are the B block rows of the H_q/H_kv query
 // heads that share the head: B*G rows (64 for Qwen3 shapes, 128 for GPT-OSS) against L + B keys
 // (context keys from the cache, then the block's own K^d / V^d). Nothing is masked: every query
-// sees every key. The keys of one (sequence, head) are cut into `splits` contiguous ranges so
-// that batch x H_kv x splits CTAs cover the GPU even for a single sequence; each CTA writes an
-// unnormalised partial output with its running max and sum, and a second launch merges them
-// (no CTA ever waits for another).
+// sees every key. The keys of one (sequence, head) are cut into contiguous ranges so that
+// batch x H_kv x splits CTAs cover the GPU even for a single sequence.
 //
-// bf16 path: 64 query rows per CTA (4 warps x 16 rows), K/V tiles of 64 keys double-buffered
-// with cp.async, S = Q K^T (bf16) and O += P V (fp16 operands) on mma.sync m16n8k16 with P
-// kept in registers.
-// fp32 path: a CUDA-core version of the same split, exact fp32 products.
+// bf16 path: 64 query rows per CTA (4 warps x 16 rows), three 64-key K/V tiles in flight with
+// cp.async, S = Q K^T (bf16) and O += P V (fp16 operands) on mma.sync m16n8k16 with P kept in
+// registers. The splits of one (sequence, head, query tile) form a thread-block cluster and
+// merge their partial results through distributed shared memory, so the whole attention is one
+// launch and no partial goes through HBM.
+// fp32 path: a CUDA-core version of the split with partials in global memory and a second
+// (combine) launch; exact fp32 products.
 #include <cuda_fp16.h>
 #include <math.h>
 
 #include <algorithm>
 
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "internal.h"
+
+namespace cg = cooperative_groups;
 
 namespace dfl {
 namespace {
@@ -109,188 +114,233 @@ __device__ __forceinline__ void bf16x8_to_f16x8(void* p) {
     *reinterpret_cast<uint4*>(p) = o;
 }
 
+constexpr int kNST = 3;    // K/V tiles in flight per CTA
+
+// One CTA per (key split, KV head, 64-row query tile, sequence); the `splits` CTAs of one
+// (sequence, head, query tile) form a thread-block cluster. Each CTA runs online softmax over its
+// key range, leaves its unnormalised partial (O, running max, running sum) in its own shared
+// memory, and after a cluster barrier every CTA merges a slice of the 64 rows from all peers'
+// shared memory (DSMEM) and writes the bf16 result. No partials go through global memory.
 template <int HD>
-__global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* __restrict__ out) {
     pdl_trigger();
     pdl_wait();
     constexpr int LD = HD + 8;                 // padded smem row (elements)
+    constexpr int PIECES = HD / 8;             // 16-byte pieces per row
     extern __shared__ __align__(16) uint8_t smem[];
     bf16* Qs = reinterpret_cast<bf16*>(smem);
-    bf16* Ks = Qs + kQT * LD;                  // [2][kKT][LD]
-    bf16* Vs = Ks + 2 * kKT * LD;              // [2][kKT][LD]
-    const int s = blockIdx.x, g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
+    bf16* Ks = Qs + kQT * LD;                  // [kNST][kKT][LD]
+    bf16* Vs = Ks + kNST * kKT * LD;           // [kNST][kKT][LD]
+    float* sO = reinterpret_cast<float*>(smem);  // after the key loop: [kQT][HD] partial output
+    float* sML = sO + kQT * HD;                  // [kQT][2] running max (log2 units), sum
+    cg::cluster_group cluster = cg::this_cluster();
+    const int S = a.splits;
+    const int s = (int)cluster.block_rank();
+    const int g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = a.B * a.G;
     int j_begin, j_end, L;
     key_range(a, b, s, j_begin, j_end, L);
-    const size_t pidx = part_index(a, b, g, qt, s);
-    float* po = a.part_o + pidx * kQT * HD;
-    float* pml = a.part_ml + pidx * kQT * 2;
-    if (j_begin >= j_end) {
-        for (int i = tid; i < kQT; i += blockDim.x) {
-            pml[2 * i] = -INFINITY;
-            pml[2 * i + 1] = 0.f;
-        }
-        return;
-    }
-    const bf16* q = static_cast<const bf16*>(a.q);
-    const bf16* kd = static_cast<const bf16*>(a.kd);
-    const bf16* vd = static_cast<const bf16*>(a.vd);
-    const bf16* kc = static_cast<const bf16*>(a.kc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
-    const bf16* vc = static_cast<const bf16*>(a.vc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
-    const uint32_t sQ = (uint32_t)__cvta_generic_to_shared(Qs);
-    const uint32_t sK = (uint32_t)__cvta_generic_to_shared(Ks);
-    const uint32_t sV = (uint32_t)__cvta_generic_to_shared(Vs);
-    constexpr int PIECES = HD / 8;             // 16-byte pieces per row
-
-    // query rows of this tile: row r -> block position r / G, head g*G + r % G
-    for (int idx = tid; idx < kQT * PIECES; idx += blockDim.x) {
-        const int r = idx / PIECES, pc = idx % PIECES;
-        const int rr = qt * kQT + r;
-        const bool ok = rr < R;
-        const int kpos = ok ? rr / a.G : 0, hh = ok ? rr % a.G : 0;
-        const bf16* src = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + pc * 8;
-        cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
-    }
-    auto load_tile = [&](int j0, int buf) {
-        for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
-            const int r = idx / PIECES, pc = idx % PIECES;
-            const int j = j0 + r;
-            const bool ok = j < j_end;
-            const bf16 *ksrc, *vsrc;
-            if (j < L) {
-                ksrc = kc + (size_t)j * HD + pc * 8;
-                vsrc = vc + (size_t)j * HD + pc * 8;
-            } else {
-                const int k = ok ? j - L : 0;
-                ksrc = kd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
-                vsrc = vd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
-            }
-            const uint32_t off = (uint32_t)((buf * kKT + r) * LD + pc * 8) * 2;
-            cp_async16(sK + off, ok ? (const void*)ksrc : (const void*)kc, ok);
-            cp_async16(sV + off, ok ? (const void*)vsrc : (const void*)vc, ok);
-        }
-    };
-    load_tile(j_begin, 0);
-    cp_commit();
 
     float o[HD / 8][4];
 #pragma unroll
     for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    uint32_t qa[HD / 16][4];
-    const int n_tiles = (j_end - j_begin + kKT - 1) / kKT;
-    for (int t = 0; t < n_tiles; ++t) {
-        const int buf = t & 1;
-        if (t + 1 < n_tiles) load_tile(j_begin + (t + 1) * kKT, buf ^ 1);
-        cp_commit();
-        cp_wait<1>();
-        // this thread's copies of tile t have landed: convert its V pieces to fp16
-        for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
+    if (j_begin < j_end) {
+        const bf16* q = static_cast<const bf16*>(a.q);
+        const bf16* kd = static_cast<const bf16*>(a.kd);
+        const bf16* vd = static_cast<const bf16*>(a.vd);
+        const bf16* kc = static_cast<const bf16*>(a.kc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
+        const bf16* vc = static_cast<const bf16*>(a.vc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
+        const uint32_t sQ = (uint32_t)__cvta_generic_to_shared(Qs);
+        const uint32_t sK = (uint32_t)__cvta_generic_to_shared(Ks);
+        const uint32_t sV = (uint32_t)__cvta_generic_to_shared(Vs);
+        // query rows of this tile: row r -> block position r / G, head g*G + r % G
+        for (int idx = tid; idx < kQT * PIECES; idx += blockDim.x) {
             const int r = idx / PIECES, pc = idx % PIECES;
-            bf16x8_to_f16x8(Vs + (buf * kKT + r) * LD + pc * 8);
+            const int rr = qt * kQT + r;
+            const bool ok = rr < R;
+            const int kpos = ok ? rr / a.G : 0, hh = ok ? rr % a.G : 0;
+            const bf16* src = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + pc * 8;
+            cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
         }
-        __syncthreads();
-        if (t == 0) {
-#pragma unroll
-            for (int kk = 0; kk < HD / 16; ++kk) {
-                const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
-                ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2],
-                        qa[kk][3]);
-            }
-        }
-        // S = Q K^T for 16 rows x 64 keys
-        float sc[8][4];
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-#pragma unroll
-            for (int kk = 0; kk < HD / 16; kk += 2) {
-                const int row = nt * 8 + (lane & 7);
-                const int col = kk * 16 + (lane >> 3) * 8;
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(sK + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
-                mma16816(sc[nt], qa[kk], b0, b1);
-                mma16816(sc[nt], qa[kk + 1], b2, b3);
-            }
-        }
-        // mask keys past the range, scale into the log2 domain, online softmax
-        const int jt = j_begin + t * kKT;
-        float mx0 = m0, mx1 = m1;
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int j = jt + nt * 8 + (lane & 3) * 2 + e;
+        // keys j < L come from the cache, j >= L from the block's own K^d / V^d
+        auto load_tile = [&](int j0, int buf) {
+            for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
+                const int r = idx / PIECES, pc = idx % PIECES;
+                const int j = j0 + r;
                 const bool ok = j < j_end;
-                sc[nt][e] = ok ? sc[nt][e] * a.scale_log2 : -INFINITY;
-                sc[nt][2 + e] = ok ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
-                mx0 = fmaxf(mx0, sc[nt][e]);
-                mx1 = fmaxf(mx1, sc[nt][2 + e]);
+                const bf16 *ksrc, *vsrc;
+                if (j < L) {
+                    ksrc = kc + (size_t)j * HD + pc * 8;
+                    vsrc = vc + (size_t)j * HD + pc * 8;
+                } else {
+                    const int k = ok ? j - L : 0;
+                    ksrc = kd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
+                    vsrc = vd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
+                }
+                const uint32_t off = (uint32_t)((buf * kKT + r) * LD + pc * 8) * 2;
+                cp_async16(sK + off, ok ? (const void*)ksrc : (const void*)kc, ok);
+                cp_async16(sV + off, ok ? (const void*)vsrc : (const void*)vc, ok);
             }
+        };
+        const int n_tiles = (j_end - j_begin + kKT - 1) / kKT;
+        for (int p = 0; p < kNST - 1; ++p) {
+            if (p < n_tiles) load_tile(j_begin + p * kKT, p);
+            cp_commit();
         }
+        uint32_t qa[HD / 16][4];
+        for (int t = 0; t < n_tiles; ++t) {
+            const int buf = t % kNST;
+            if (t + kNST - 1 < n_tiles) load_tile(j_begin + (t + kNST - 1) * kKT, (t + kNST - 1) % kNST);
+            cp_commit();
+            cp_wait<kNST - 1>();
+            // this thread's copies of tile t have landed: convert its V pieces to fp16
+            for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
+                const int r = idx / PIECES, pc = idx % PIECES;
+                bf16x8_to_f16x8(Vs + (buf * kKT + r) * LD + pc * 8);
+            }
+            __syncthreads();
+            if (t == 0) {
+#pragma unroll
+                for (int kk = 0; kk < HD / 16; ++kk) {
+                    const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
+                    ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2],
+                            qa[kk][3]);
+                }
+            }
+            // S = Q K^T for 16 rows x 64 keys
+            float sc[8][4];
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+#pragma unroll
+                for (int kk = 0; kk < HD / 16; kk += 2) {
+                    const int row = nt * 8 + (lane & 7);
+                    const int col = kk * 16 + (lane >> 3) * 8;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4(sK + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
+                    mma16816(sc[nt], qa[kk], b0, b1);
+                    mma16816(sc[nt], qa[kk + 1], b2, b3);
+                }
+            }
+            // mask keys past the range, scale into the log2 domain, online softmax
+            const int jt = j_begin + t * kKT;
+            float mx0 = m0, mx1 = m1;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int j = jt + nt * 8 + (lane & 3) * 2 + e;
+                    const bool ok = j < j_end;
+                    sc[nt][e] = ok ? sc[nt][e] * a.scale_log2 : -INFINITY;
+                    sc[nt][2 + e] = ok ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
+                    mx0 = fmaxf(mx0, sc[nt][e]);
+                    mx1 = fmaxf(mx1, sc[nt][2 + e]);
+                }
+            }
+#pragma unroll
+            for (int off = 1; off <= 2; off <<= 1) {
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+            }
+            const float c0 = exp2f(m0 - mx0), c1 = exp2f(m1 - mx1);
+            m0 = mx0;
+            m1 = mx1;
+            l0 *= c0;
+            l1 *= c1;
+#pragma unroll
+            for (int i = 0; i < HD / 8; ++i) {
+                o[i][0] *= c0; o[i][1] *= c0; o[i][2] *= c1; o[i][3] *= c1;
+            }
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                sc[nt][0] = exp2f(sc[nt][0] - m0);
+                sc[nt][1] = exp2f(sc[nt][1] - m0);
+                sc[nt][2] = exp2f(sc[nt][2] - m1);
+                sc[nt][3] = exp2f(sc[nt][3] - m1);
+                l0 += sc[nt][0] + sc[nt][1];
+                l1 += sc[nt][2] + sc[nt][3];
+            }
+            // O += P V (P from registers as the A operand; V tiles transposed by ldmatrix)
+#pragma unroll
+            for (int kk = 0; kk < kKT / 16; ++kk) {
+                uint32_t pa[4];
+                pa[0] = pack_f16(sc[2 * kk][0], sc[2 * kk][1]);
+                pa[1] = pack_f16(sc[2 * kk][2], sc[2 * kk][3]);
+                pa[2] = pack_f16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+                pa[3] = pack_f16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+                for (int nt = 0; nt < HD / 8; nt += 2) {
+                    const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                    const int col = (nt + (lane >> 4)) * 8;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4_t(sV + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
+                    mma16816_f16(o[nt], pa, b0, b1);
+                    mma16816_f16(o[nt + 1], pa, b2, b3);
+                }
+            }
+            __syncthreads();
+        }
+        cp_wait<0>();
 #pragma unroll
         for (int off = 1; off <= 2; off <<= 1) {
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+            l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+            l1 += __shfl_xor_sync(0xffffffffu, l1, off);
         }
-        const float c0 = exp2f(m0 - mx0), c1 = exp2f(m1 - mx1);
-        m0 = mx0;
-        m1 = mx1;
-        l0 *= c0;
-        l1 *= c1;
+    }
+    __syncthreads();   // the tiles' shared memory now holds this CTA's partial result
+    {
+        const int r0 = warp * 16 + (lane >> 2), r1 = r0 + 8;
 #pragma unroll
-        for (int i = 0; i < HD / 8; ++i) {
-            o[i][0] *= c0; o[i][1] *= c0; o[i][2] *= c1; o[i][3] *= c1;
+        for (int nt = 0; nt < HD / 8; ++nt) {
+            const int col = nt * 8 + (lane & 3) * 2;
+            *reinterpret_cast<float2*>(sO + r0 * HD + col) = make_float2(o[nt][0], o[nt][1]);
+            *reinterpret_cast<float2*>(sO + r1 * HD + col) = make_float2(o[nt][2], o[nt][3]);
         }
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            sc[nt][0] = exp2f(sc[nt][0] - m0);
-            sc[nt][1] = exp2f(sc[nt][1] - m0);
-            sc[nt][2] = exp2f(sc[nt][2] - m1);
-            sc[nt][3] = exp2f(sc[nt][3] - m1);
-            l0 += sc[nt][0] + sc[nt][1];
-            l1 += sc[nt][2] + sc[nt][3];
+        if ((lane & 3) == 0) {
+            sML[2 * r0] = m0;
+            sML[2 * r0 + 1] = l0;
+            sML[2 * r1] = m1;
+            sML[2 * r1 + 1] = l1;
         }
-        // O += P V (P from registers as the A operand; V tiles transposed by ldmatrix)
+    }
+    cluster.sync();
+    // merge: CTA s owns rows [s * RP, (s + 1) * RP) of the 64; TPR threads per row
+    const int RP = kQT / S, TPR = 128 / RP;
+    const int rr = s * RP + tid / TPR, lt = tid % TPR;
+    const int rg = qt * kQT + rr;
+    if (rg < R) {
+        float w[8], M = -INFINITY;
 #pragma unroll
-        for (int kk = 0; kk < kKT / 16; ++kk) {
-            uint32_t pa[4];
-            pa[0] = pack_f16(sc[2 * kk][0], sc[2 * kk][1]);
-            pa[1] = pack_f16(sc[2 * kk][2], sc[2 * kk][3]);
-            pa[2] = pack_f16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            pa[3] = pack_f16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
-#pragma unroll
-            for (int nt = 0; nt < HD / 8; nt += 2) {
-                const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-                const int col = (nt + (lane >> 4)) * 8;
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(sV + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
-                mma16816_f16(o[nt], pa, b0, b1);
-                mma16816_f16(o[nt + 1], pa, b2, b3);
+        for (int p = 0; p < 8; ++p) {
+            if (p < S) {
+                const float* ml = cluster.map_shared_rank(sML, p);
+                w[p] = ml[2 * rr];
+                M = fmaxf(M, w[p]);
             }
         }
-        __syncthreads();
-    }
-    cp_wait<0>();
+        float den = 0.f;
 #pragma unroll
-    for (int off = 1; off <= 2; off <<= 1) {
-        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-    }
-    const int r0 = warp * 16 + (lane >> 2), r1 = r0 + 8;
+        for (int p = 0; p < 8; ++p) {
+            if (p < S) {
+                const float* ml = cluster.map_shared_rank(sML, p);
+                w[p] = (w[p] == -INFINITY) ? 0.f : exp2f(w[p] - M);
+                den = fmaf(w[p], ml[2 * rr + 1], den);
+            }
+        }
+        const float inv = 1.0f / den;
+        const int kpos = rg / a.G, hh = rg % a.G;
+        bf16* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD;
+        for (int e = lt; e < HD; e += TPR) {
+            float v = 0.f;
 #pragma unroll
-    for (int nt = 0; nt < HD / 8; ++nt) {
-        const int col = nt * 8 + (lane & 3) * 2;
-        *reinterpret_cast<float2*>(po + (size_t)r0 * HD + col) = make_float2(o[nt][0], o[nt][1]);
-        *reinterpret_cast<float2*>(po + (size_t)r1 * HD + col) = make_float2(o[nt][2], o[nt][3]);
+            for (int p = 0; p < 8; ++p)
+                if (p < S) v = fmaf(w[p], cluster.map_shared_rank(sO, p)[rr * HD + e], v);
+            orow[e] = __float2bfloat16_rn(v * inv);
+        }
     }
-    if ((lane & 3) == 0) {
-        pml[2 * r0] = m0;
-        pml[2 * r0 + 1] = l0;
-        pml[2 * r1] = m1;
-        pml[2 * r1 + 1] = l1;
-    }
+    cluster.sync();    // peers may still be reading this CTA's shared memory
 }
 
 // ------------------------------------------------------------------ CUDA-core path
@@ -385,25 +435,28 @@ __global__ void attn_combine_kernel(const AttnArgs a, T* __restrict__ out) {
 
 template <int HD>
 size_t mma_smem_bytes() {
-    return (size_t)(kQT + 4 * kKT) * (HD + 8) * sizeof(bf16);
+    return (size_t)(kQT + 2 * kNST * kKT) * (HD + 8) * sizeof(bf16);
+}
+
+template <int HD>
+cudaError_t run_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)mma_smem_bytes<HD>());
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    return launch_cluster(c->pdl, a.splits, attn_mma_kernel<HD>,
+                          dim3(a.splits, a.hkv * a.q_tiles, c->batch), dim3(128),
+                          mma_smem_bytes<HD>(), s, a, static_cast<bf16*>(c->attn));
 }
 
 template <class T, int HD>
-cudaError_t run(dflare_ctx* c, const AttnArgs& a, bool mma, cudaStream_t s) {
-    const dim3 grid(a.splits, a.hkv * a.q_tiles, c->batch);
-    cudaError_t e;
-    if (mma) {
-        static bool configured = false;
-        if (!configured) {
-            e = cudaFuncSetAttribute(attn_mma_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)mma_smem_bytes<HD>());
-            if (e != cudaSuccess) return e;
-            configured = true;
-        }
-        e = launch_kernel(c->pdl, attn_mma_kernel<HD>, grid, dim3(128), mma_smem_bytes<HD>(), s, a);
-    } else {
-        e = launch_kernel(c->pdl, attn_simt_kernel<T, HD>, grid, dim3(128), 0, s, a);
-    }
+cudaError_t run_simt(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
+    cudaError_t e = launch_kernel(c->pdl, attn_simt_kernel<T, HD>,
+                                  dim3(a.splits, a.hkv * a.q_tiles, c->batch), dim3(128), 0, s, a);
     if (e != cudaSuccess) return e;
     return launch_kernel(c->pdl, attn_combine_kernel<T, HD>, dim3(a.B * a.G, a.hkv, c->batch),
                          dim3(64), 0, s, a, static_cast<T*>(c->attn));
@@ -411,10 +464,10 @@ cudaError_t run(dflare_ctx* c, const AttnArgs& a, bool mma, cudaStream_t s) {
 
 }  // namespace
 
-// Split count: enough CTAs for about two per SM over batch x H_kv x q_tiles, but no split
-// shorter than 256 keys at the host's upper bound of the context length (each split writes a
-// 64 x hd fp32 partial, as many bytes as 128 keys of K and V). The device derives the actual
-// ranges from the true lengths, so a stale bound (e.g. a replayed graph) only costs speed.
+// CUDA-core (fp32) path: enough splits for about two CTAs per SM over batch x H_kv x q_tiles,
+// none shorter than 256 keys at the host's upper bound of the context length; partials go
+// through global memory to a combine launch. The device derives the actual ranges from the true
+// lengths, so a stale bound (e.g. a replayed graph) only costs speed.
 int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub) {
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + kQT - 1) / kQT;
@@ -422,6 +475,19 @@ int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub)
     int sp = (2 * num_sms + base - 1) / base;
     sp = std::min(sp, (len_ub + g.block + 255) / 256);
     return std::max(1, sp);
+}
+
+// Tensor-core path: the splits of one (sequence, head, query tile) are one cluster of 1, 2, 4 or 8
+// CTAs: as many as needed for about two CTAs per SM, at most one per 64-key tile.
+int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int len_ub) {
+    const int G = g.n_q_heads / g.n_kv_heads;
+    const int q_tiles = (g.block * G + kQT - 1) / kQT;
+    const int base = batch * g.n_kv_heads * q_tiles;
+    const int want = (2 * num_sms + base - 1) / base;
+    const int tiles = (len_ub + g.block + kKT - 1) / kKT;
+    int sp = 1;
+    while (sp < 8 && sp < want && 2 * sp <= tiles) sp *= 2;
+    return sp;
 }
 
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
@@ -442,13 +508,14 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
     a.d_q = g.n_q_heads * g.head_dim;
     a.d_kv = g.n_kv_heads * g.head_dim;
     a.max_ctx = g.max_ctx;
-    a.splits = attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
     a.q_tiles = (a.B * a.G + kQT - 1) / kQT;
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)g.head_dim);
-    const bool f32 = g.dtype == DFLARE_F32;
-    if (g.head_dim == 64)
-        return f32 ? run<float, 64>(c, a, false, s) : run<bf16, 64>(c, a, true, s);
-    return f32 ? run<float, 128>(c, a, false, s) : run<bf16, 128>(c, a, true, s);
+    if (g.dtype == DFLARE_F32) {
+        a.splits = attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
+        return g.head_dim == 64 ? run_simt<float, 64>(c, a, s) : run_simt<float, 128>(c, a, s);
+    }
+    a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub);
+    return g.head_dim == 64 ? run_mma<64>(c, a, s) : run_mma<128>(c, a, s);
 }
 
 }  // namespace dfl

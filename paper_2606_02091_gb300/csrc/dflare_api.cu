@@ -180,8 +180,8 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     // split-KV partial buffers sized for the largest batch x splits product
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + 63) / 64;
-    size_t part_rows = 0;
-    for (int b = 1; b <= g.max_batch; ++b) {
+    size_t part_rows = 1;   // split-KV partials in global memory: the fp32 path only
+    for (int b = 1; b <= g.max_batch && g.dtype == DFLARE_F32; ++b) {
         const size_t r = (size_t)b * g.n_kv_heads * q_tiles * attention_splits(g, b, c->num_sms, g.max_ctx) * 64;
         if (r > part_rows) part_rows = r;
     }

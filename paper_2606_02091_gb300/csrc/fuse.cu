@@ -2,15 +2,16 @@
 //
 // fusion_alpha: alpha^(i) = softmax(W^fuse_{i,:}), computed once when the weights are set
 // (Sec. 4.1: the normalised weights can be cached after training).
-// fuse_layers: one CTA per new position; every thread owns 8 consecutive features, reads the T
-// target states of its features once with 16-byte loads (four layers in flight), forms the
-// weighted sums of up to 8 draft layers in registers, then RMSNorms each sum (one block
-// reduction for all layers at once). More than 8 draft layers take further passes over the same
-// rows, which the previous pass left in L2.
+// fuse_layers: one thread-block cluster per new position reads the T target rows of that position
+// exactly once and writes every draft layer's fused, normalised row.
 #include <math.h>
+
+#include <cooperative_groups.h>
 
 #include "common.cuh"
 #include "internal.h"
+
+namespace cg = cooperative_groups;
 
 namespace dfl {
 namespace {
@@ -51,26 +52,50 @@ __global__ void fuse_begin_kernel(int32_t* ctx_len, int32_t* app_base, int32_t* 
     ctx_len[b] = L + n;
 }
 
+constexpr int kFuseCH = 512;       // features per CTA (64 threads x 8)
+
+// One position is handled by a cluster of ceil(d / 512) CTAs (at most 8 for d <= 4096); CTA c owns
+// features [512 c, 512 c + 512). Each CTA stages its slice of all T target rows in shared memory
+// with cp.async (one round trip), forms the D weighted sums in registers (up to 8 draft layers
+// per pass), reduces its partial sums of squares, and the CTAs of the cluster exchange those
+// partials through distributed shared memory (summed in rank order) before normalising.
 template <class T, int DMAX>
-__global__ void __launch_bounds__(512) fuse_layers_kernel(
+__global__ void __launch_bounds__(64) fuse_layers_kernel(
     const T* __restrict__ H, const float* __restrict__ alpha, const T* __restrict__ gain,
     T* __restrict__ F, T* __restrict__ F_out, const int32_t* __restrict__ app_cnt, int D, int Tn,
     int batch, int n_max, int d, long long f_layer_rows, float eps) {
     pdl_trigger();
     pdl_wait();
+    extern __shared__ __align__(16) uint8_t smem[];
+    T* sh = reinterpret_cast<T*>(smem);          // [Tn][kFuseCH]
     __shared__ float s_alpha[16 * 64];
-    __shared__ float red[32][DMAX];
-    const int r = blockIdx.x, b = blockIdx.y;
-    for (int k = threadIdx.x; k < D * Tn; k += blockDim.x) s_alpha[k] = alpha[k];
-    __syncthreads();
-    if (r >= app_cnt[b]) return;
-    const int e0 = threadIdx.x * 8;
-    const bool act = e0 < d;
+    __shared__ float red[2][DMAX];
+    __shared__ float ss_cta[DMAX];
+    cg::cluster_group cluster = cg::this_cluster();
+    const int C = (int)cluster.num_blocks(), cr = (int)cluster.block_rank();
+    const int r = blockIdx.y, b = blockIdx.z;
+    if (r >= app_cnt[b]) return;                 // the same for every CTA of the cluster
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int f0 = cr * kFuseCH, nf = min(kFuseCH, d - f0);
     const size_t row = (size_t)b * n_max + r;
     const size_t lstride = (size_t)batch * n_max * d;
-    const T* hrow = H + row * d + (act ? e0 : 0);
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-
+    constexpr int EPC = 16 / sizeof(T);          // elements per 16-byte copy
+    const int per_row = nf / EPC;
+    const uint32_t ssh = (uint32_t)__cvta_generic_to_shared(sh);
+    for (int idx = tid; idx < Tn * per_row; idx += blockDim.x) {
+        const int j = idx / per_row, p = idx % per_row;
+        const T* src = H + (size_t)j * lstride + row * d + f0 + p * EPC;
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                         ssh + (uint32_t)((j * kFuseCH + p * EPC) * sizeof(T))),
+                     "l"(src)
+                     : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    for (int k = tid; k < D * Tn; k += blockDim.x) s_alpha[k] = alpha[k];
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    const int e0 = tid * 8;
+    const bool act = e0 < nf;
     for (int i0 = 0; i0 < D; i0 += DMAX) {
         const int nd = min(DMAX, D - i0);
         float acc[DMAX][8];
@@ -79,58 +104,47 @@ __global__ void __launch_bounds__(512) fuse_layers_kernel(
 #pragma unroll
             for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
         if (act) {
-            for (int j0 = 0; j0 < Tn; j0 += 4) {
-                float h[4][8];
+            for (int j = 0; j < Tn; ++j) {
+                float h[8];
+                load8(sh + j * kFuseCH + e0, h);
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (j0 + u < Tn) load8(hrow + (size_t)(j0 + u) * lstride, h[u]);
+                for (int i = 0; i < DMAX; ++i) {
+                    if (i < nd) {
+                        const float a = s_alpha[(i0 + i) * Tn + j];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    if (j0 + u >= Tn) break;
-#pragma unroll
-                    for (int i = 0; i < DMAX; ++i) {
-                        if (i < nd) {
-                            const float a = s_alpha[(i0 + i) * Tn + j0 + u];
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a, h[u][e], acc[i][e]);
-                        }
+                        for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a, h[e], acc[i][e]);
                     }
                 }
             }
         }
-        // sum of squares of every draft layer's fused row, one reduction for all of them
-        float ss[DMAX];
 #pragma unroll
         for (int i = 0; i < DMAX; ++i) {
             float v = 0.f;
 #pragma unroll
             for (int e = 0; e < 8; ++e) v = fmaf(acc[i][e], acc[i][e], v);
-            ss[i] = warp_sum(v);
+            v = warp_sum(v);
+            if (lane == 0) red[warp][i] = v;
         }
         __syncthreads();
-        if (lane == 0)
-#pragma unroll
-            for (int i = 0; i < DMAX; ++i) red[warp][i] = ss[i];
-        __syncthreads();
-#pragma unroll
-        for (int i = 0; i < DMAX; ++i) {
-            float s = 0.f;
-            for (int w = 0; w < nw; ++w) s += red[w][i];
-            ss[i] = s;
-        }
+        if (tid < DMAX) ss_cta[tid] = red[0][tid] + red[1][tid];
+        cluster.sync();
         if (act) {
 #pragma unroll
             for (int i = 0; i < DMAX; ++i) {
                 if (i >= nd) break;
-                const float inv = inv_rms(ss[i], d, eps);
+                float tot = 0.f;
+                for (int c = 0; c < C; ++c) tot += cluster.map_shared_rank(ss_cta, c)[i];
+                const float inv = inv_rms(tot, d, eps);
                 float g[8], o[8];
-                load8(gain + (size_t)(i0 + i) * d + e0, g);
+                load8(gain + (size_t)(i0 + i) * d + f0 + e0, g);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) o[e] = g[e] * (acc[i][e] * inv);
-                store8(F + ((size_t)(i0 + i) * f_layer_rows + row) * d + e0, o);
-                if (F_out) store8(F_out + (((size_t)(i0 + i) * batch + b) * n_max + r) * d + e0, o);
+                store8(F + ((size_t)(i0 + i) * f_layer_rows + row) * d + f0 + e0, o);
+                if (F_out)
+                    store8(F_out + (((size_t)(i0 + i) * batch + b) * n_max + r) * d + f0 + e0, o);
             }
         }
+        cluster.sync();   // peers have read ss_cta before it is reused or this CTA exits
     }
 }
 
@@ -138,15 +152,26 @@ template <class T>
 cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,
                           cudaStream_t s) {
     const dflare_config& g = c->cfg;
-    const dim3 grid(n_max, c->batch), block(((g.d / 8 + 31) / 32) * 32);
+    const int C = (g.d + kFuseCH - 1) / kFuseCH;
+    const size_t smem = (size_t)g.n_target_layers * kFuseCH * sizeof(T);
     const T* H = static_cast<const T*>(hidden);
     const T* gain = static_cast<const T*>(c->w.fuse_norm);
     T* F = static_cast<T*>(c->fused);
     T* Fo = static_cast<T*>(fused_out);
     auto kern = g.n_draft_layers <= 4 ? fuse_layers_kernel<T, 4> : fuse_layers_kernel<T, 8>;
-    return launch_kernel(c->pdl, kern, grid, block, 0, s, H, (const float*)c->alpha, gain, F, Fo,
-                         (const int32_t*)c->app_cnt, g.n_draft_layers, g.n_target_layers, c->batch,
-                         n_max, g.d, (long long)g.max_fuse_rows, g.rms_eps);
+    static bool configured = false;
+    if (!configured) {
+        for (auto k : {fuse_layers_kernel<T, 4>, fuse_layers_kernel<T, 8>}) {
+            cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)(64 * kFuseCH * sizeof(T)));
+            if (e != cudaSuccess) return e;
+        }
+        configured = true;
+    }
+    return launch_cluster(c->pdl, C, kern, dim3(C, n_max, c->batch), dim3(64), smem, s, H,
+                          (const float*)c->alpha, gain, F, Fo, (const int32_t*)c->app_cnt,
+                          g.n_draft_layers, g.n_target_layers, c->batch, n_max, g.d,
+                          (long long)g.max_fuse_rows, g.rms_eps);
 }
 
 }  // namespace
