@@ -210,12 +210,14 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
                 }
             }
             // S = Q K^T for 16 rows x 64 keys
+            // (k outer, keys inner: eight independent accumulators between dependent MMAs)
             float sc[8][4];
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+            for (int nt = 0; nt < 8; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
 #pragma unroll
-                for (int kk = 0; kk < HD / 16; kk += 2) {
+            for (int kk = 0; kk < HD / 16; kk += 2) {
+#pragma unroll
+                for (int nt = 0; nt < 8; ++nt) {
                     const int row = nt * 8 + (lane & 7);
                     const int col = kk * 16 + (lane >> 3) * 8;
                     uint32_t b0, b1, b2, b3;

@@ -1,6 +1,6 @@
 // Epilogues of the projection GEMMs, shared by the tcgen05 and the CUDA-core GEMM.
 //
-// Both GEMMs hand over a tile of fp32 accumulators for 128 consecutive output features and `nc`
+// Both GEMMs hand over a tile of fp32 accumulators for 128 consecutive output features and 16
 // consecutive token rows, laid out [accumulator][token][feature] in shared memory. Thread t
 // (0..127) writes output feature n_tile*128 + t for every token of the tile; the rotary
 // embedding pairs feature j with j +- head_dim/2, which lies in the same tile because every head
@@ -11,35 +11,52 @@
 
 namespace dfl {
 
+constexpr int kEpiChunk = 16;   // tokens per epilogue tile
+
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }
 
+// Every branch issues all of its global loads (residual values, per-token positions, rotary
+// factors) before its first store, so the loads of the 16 tokens of a chunk are in flight
+// together instead of each waiting behind the previous token's store.
 template <class T>
-__device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float* tile, int nc,
-                                               int group, int n_tile, int tok0, int t) {
+__device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float* tile, int group,
+                                               int n_tile, int tok0, int t) {
+    constexpr int NC = kEpiChunk;
     const int n = n_tile * 128 + t;
     if (n >= ep.n) return;
     const int hd = ep.head_dim, half = hd >> 1;
+    const int nvalid = min(NC, ep.m_tok - tok0);
+    if (nvalid <= 0) return;
     switch (ep.kind) {
         case EPI_STORE: {
             T* out = reinterpret_cast<T*>(ep.out);
-            for (int c = 0; c < nc && tok0 + c < ep.m_tok; ++c)
-                out[(size_t)(tok0 + c) * ep.ldo + n] = from_f<T>(tile[c * 128 + t]);
+#pragma unroll
+            for (int c = 0; c < NC; ++c)
+                if (c < nvalid) out[(size_t)(tok0 + c) * ep.ldo + n] = from_f<T>(tile[c * 128 + t]);
         } break;
         case EPI_F32: {
             float* out = reinterpret_cast<float*>(ep.out);
-            for (int c = 0; c < nc && tok0 + c < ep.m_tok; ++c)
-                out[(size_t)(tok0 + c) * ep.ldo + n] = tile[c * 128 + t];
+#pragma unroll
+            for (int c = 0; c < NC; ++c)
+                if (c < nvalid) out[(size_t)(tok0 + c) * ep.ldo + n] = tile[c * 128 + t];
         } break;
         case EPI_RESID: {
-            for (int c = 0; c < nc && tok0 + c < ep.m_tok; ++c)
-                ep.resid[(size_t)(tok0 + c) * ep.ld_resid + n] += tile[c * 128 + t];
+            float r[NC];
+#pragma unroll
+            for (int c = 0; c < NC; ++c)
+                r[c] = c < nvalid ? ep.resid[(size_t)(tok0 + c) * ep.ld_resid + n] : 0.f;
+#pragma unroll
+            for (int c = 0; c < NC; ++c)
+                if (c < nvalid) ep.resid[(size_t)(tok0 + c) * ep.ld_resid + n] = r[c] + tile[c * 128 + t];
         } break;
         case EPI_SWIGLU: {
             T* out = reinterpret_cast<T*>(ep.out);
-            const float* up = tile + nc * 128;
-            for (int c = 0; c < nc && tok0 + c < ep.m_tok; ++c)
-                out[(size_t)(tok0 + c) * ep.ldo + n] =
-                    from_f<T>(silu_f(tile[c * 128 + t]) * up[c * 128 + t]);
+            const float* up = tile + NC * 128;
+#pragma unroll
+            for (int c = 0; c < NC; ++c)
+                if (c < nvalid)
+                    out[(size_t)(tok0 + c) * ep.ldo + n] =
+                        from_f<T>(silu_f(tile[c * 128 + t]) * up[c * 128 + t]);
         } break;
         case EPI_QKV: {
             int col, ld, rot;
@@ -51,42 +68,69 @@ __device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float*
             } else {
                 col = n - ep.d_q - ep.d_kv; ld = ep.d_kv; dst = reinterpret_cast<T*>(ep.vd); rot = 0;
             }
-            const int j = col % hd;
+            const int j = col % hd, jj = j % half;
             const int tp = j < half ? t + half : t - half;
-            for (int c = 0; c < nc && tok0 + c < ep.m_tok; ++c) {
-                const int tok = tok0 + c;
+            float cs[NC], sn[NC];
+            if (rot) {
+                int pos[NC];
+#pragma unroll
+                for (int c = 0; c < NC; ++c) {
+                    const int tok = tok0 + min(c, nvalid - 1);
+                    const int b = tok / ep.block;
+                    pos[c] = ep.ctx_len[b] + (tok - b * ep.block);
+                }
+#pragma unroll
+                for (int c = 0; c < NC; ++c) {
+                    cs[c] = ep.rope_cos[(size_t)pos[c] * half + jj];
+                    sn[c] = ep.rope_sin[(size_t)pos[c] * half + jj];
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+                if (c >= nvalid) break;
                 float v = tile[c * 128 + t];
                 if (rot) {
-                    const int b = tok / ep.block, k = tok - b * ep.block;
-                    const int pos = ep.ctx_len[b] + k;
-                    const float cs = ep.rope_cos[(size_t)pos * half + (j % half)];
-                    const float sn = ep.rope_sin[(size_t)pos * half + (j % half)];
                     const float y = tile[c * 128 + tp];
-                    v = j < half ? v * cs - y * sn : v * cs + y * sn;
+                    v = j < half ? v * cs[c] - y * sn[c] : v * cs[c] + y * sn[c];
                 }
-                dst[(size_t)tok * ld + col] = from_f<T>(v);
+                dst[(size_t)(tok0 + c) * ld + col] = from_f<T>(v);
             }
         } break;
         case EPI_KV_APPEND: {
             const bool is_k = n < ep.d_kv;
             const int col = is_k ? n : n - ep.d_kv;
-            const int g = col / hd, j = col - g * hd;
+            const int g = col / hd, j = col - g * hd, jj = j % half;
             const int tp = j < half ? t + half : t - half;
             const int hkv = ep.d_kv / hd;
             T* cache = reinterpret_cast<T*>(is_k ? ep.kcache : ep.vcache);
-            for (int c = 0; c < nc && tok0 + c < ep.m_tok; ++c) {
-                const int tok = tok0 + c;
+            int pos[NC], ok[NC], bb[NC];
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+                const int tok = tok0 + min(c, nvalid - 1);
                 const int b = tok / ep.n_max, r = tok - b * ep.n_max;
-                if (r >= ep.app_cnt[b]) continue;
-                const int pos = ep.app_base[b] + r;
+                bb[c] = b;
+                ok[c] = c < nvalid && r < ep.app_cnt[b];
+                pos[c] = ep.app_base[b] + r;
+            }
+            float cs[NC], sn[NC];
+            if (is_k) {
+#pragma unroll
+                for (int c = 0; c < NC; ++c) {
+                    const int p = ok[c] ? pos[c] : 0;
+                    cs[c] = ep.rope_cos[(size_t)p * half + jj];
+                    sn[c] = ep.rope_sin[(size_t)p * half + jj];
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+                if (!ok[c]) continue;
                 float v = tile[c * 128 + t];
                 if (is_k) {
-                    const float cs = ep.rope_cos[(size_t)pos * half + (j % half)];
-                    const float sn = ep.rope_sin[(size_t)pos * half + (j % half)];
                     const float y = tile[c * 128 + tp];
-                    v = j < half ? v * cs - y * sn : v * cs + y * sn;
+                    v = j < half ? v * cs[c] - y * sn[c] : v * cs[c] + y * sn[c];
                 }
-                const size_t row = (((size_t)group * ep.max_batch + b) * hkv + g) * ep.max_ctx + pos;
+                const size_t row =
+                    (((size_t)group * ep.max_batch + bb[c]) * hkv + g) * ep.max_ctx + pos[c];
                 cache[row * hd + j] = from_f<T>(v);
             }
         } break;

@@ -61,7 +61,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 #pragma unroll
         for (int i = 0; i < 8; ++i) tile[(a * kTT + tg * 8 + i) * kTN + f] = acc[a][i];
     __syncthreads();
-    if (tid < 128) apply_epilogue<T>(ep, tile, kTT, group, n_tile, tok0, tid);
+    if (tid < 128) apply_epilogue<T>(ep, tile, group, n_tile, tok0, tid);
 }
 
 }  // namespace

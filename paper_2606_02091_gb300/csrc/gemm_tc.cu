@@ -434,8 +434,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                         for (int c = 0; c < kChunk; ++c) epi[(a * kChunk + c) * 128 + t] = v[c];
                     }
                     epi_bar();
-                    apply_epilogue<bf16>(args.ep, epi, kChunk, x.group, x.n_tile,
-                                         x.tok_tile * bn + c0, t);
+                    apply_epilogue<bf16>(args.ep, epi, x.group, x.n_tile, x.tok_tile * bn + c0, t);
                     epi_bar();
                 }
             }
