@@ -9,7 +9,8 @@
 //
 // bf16 path: 64 query rows per CTA (4 warps x 16 rows), three 64-key K/V tiles in flight with
 // cp.async, S = Q K^T (bf16) and O += P V (fp16 operands) on mma.sync m16n8k16 with P kept in
-// registers. The splits of one (sequence, head, query tile) form a thread-block cluster and
+// registers; two CTAs fit on an SM. The splits of one (sequence, head, query tile) form a
+// thread-block cluster (up to 16 CTAs) and
 // merge their partial results through distributed shared memory, so the whole attention is one
 // launch and no partial goes through HBM.
 // fp32 path: a CUDA-core version of the split with partials in global memory and a second
@@ -114,14 +115,14 @@ __device__ __forceinline__ void bf16x8_to_f16x8(void* p) {
     *reinterpret_cast<uint4*>(p) = o;
 }
 
-constexpr int kNST = 3;    // K/V tiles in flight per CTA
+constexpr int kNST = 2;    // K/V tiles in flight per CTA (two CTAs fit on an SM)
 
 // One CTA per (key split, KV head, 64-row query tile, sequence); the `splits` CTAs of one
 // (sequence, head, query tile) form a thread-block cluster. Each CTA runs online softmax over its
 // key range, leaves its unnormalised partial (O, running max, running sum) in its own shared
 // memory, and after a cluster barrier every CTA merges a slice of the 64 rows from all peers'
 // shared memory (DSMEM) and writes the bf16 result. No partials go through global memory.
-template <int HD>
+template <int HD, int S>
 __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* __restrict__ out) {
     pdl_trigger();
     pdl_wait();
@@ -134,7 +135,6 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
     float* sO = reinterpret_cast<float*>(smem);  // after the key loop: [kQT][HD] partial output
     float* sML = sO + kQT * HD;                  // [kQT][2] running max (log2 units), sum
     cg::cluster_group cluster = cg::this_cluster();
-    const int S = a.splits;
     const int s = (int)cluster.block_rank();
     const int g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -308,38 +308,40 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
         }
     }
     cluster.sync();
-    // merge: CTA s owns rows [s * RP, (s + 1) * RP) of the 64; TPR threads per row
-    const int RP = kQT / S, TPR = 128 / RP;
+    // merge: CTA s owns rows [s * RP, (s + 1) * RP) of the 64, TPR threads per row, EPT output
+    // elements per thread; every peer value is loaded before anything is stored
+    constexpr int RP = kQT / S, TPR = 128 / RP, EPT = HD / TPR;
     const int rr = s * RP + tid / TPR, lt = tid % TPR;
     const int rg = qt * kQT + rr;
     if (rg < R) {
-        float w[8], M = -INFINITY;
+        float mv[S], lv[S], vals[S][EPT];
 #pragma unroll
-        for (int p = 0; p < 8; ++p) {
-            if (p < S) {
-                const float* ml = cluster.map_shared_rank(sML, p);
-                w[p] = ml[2 * rr];
-                M = fmaxf(M, w[p]);
-            }
+        for (int p = 0; p < S; ++p) {
+            const float* ml = cluster.map_shared_rank(sML, p);
+            const float* op = cluster.map_shared_rank(sO, p) + rr * HD;
+            mv[p] = ml[2 * rr];
+            lv[p] = ml[2 * rr + 1];
+#pragma unroll
+            for (int q = 0; q < EPT; ++q) vals[p][q] = op[lt + q * TPR];
         }
+        float M = -INFINITY;
+#pragma unroll
+        for (int p = 0; p < S; ++p) M = fmaxf(M, mv[p]);
         float den = 0.f;
 #pragma unroll
-        for (int p = 0; p < 8; ++p) {
-            if (p < S) {
-                const float* ml = cluster.map_shared_rank(sML, p);
-                w[p] = (w[p] == -INFINITY) ? 0.f : exp2f(w[p] - M);
-                den = fmaf(w[p], ml[2 * rr + 1], den);
-            }
+        for (int p = 0; p < S; ++p) {
+            mv[p] = (mv[p] == -INFINITY) ? 0.f : exp2f(mv[p] - M);
+            den = fmaf(mv[p], lv[p], den);
         }
         const float inv = 1.0f / den;
         const int kpos = rg / a.G, hh = rg % a.G;
         bf16* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD;
-        for (int e = lt; e < HD; e += TPR) {
+#pragma unroll
+        for (int q = 0; q < EPT; ++q) {
             float v = 0.f;
 #pragma unroll
-            for (int p = 0; p < 8; ++p)
-                if (p < S) v = fmaf(w[p], cluster.map_shared_rank(sO, p)[rr * HD + e], v);
-            orow[e] = __float2bfloat16_rn(v * inv);
+            for (int p = 0; p < S; ++p) v = fmaf(mv[p], vals[p][q], v);
+            orow[lt + q * TPR] = __float2bfloat16_rn(v * inv);
         }
     }
     cluster.sync();    // peers may still be reading this CTA's shared memory
@@ -440,19 +442,62 @@ size_t mma_smem_bytes() {
     return (size_t)(kQT + 2 * kNST * kKT) * (HD + 8) * sizeof(bf16);
 }
 
-template <int HD>
-cudaError_t run_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
+template <int HD, int S>
+cudaError_t launch_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD>,
+        cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)mma_smem_bytes<HD>());
+        if (e == cudaSuccess && S > 8)
+            e = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
+                                     cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    return launch_cluster(c->pdl, a.splits, attn_mma_kernel<HD>,
-                          dim3(a.splits, a.hkv * a.q_tiles, c->batch), dim3(128),
-                          mma_smem_bytes<HD>(), s, a, static_cast<bf16*>(c->attn));
+    return launch_cluster(c->pdl, S, attn_mma_kernel<HD, S>, dim3(S, a.hkv * a.q_tiles, c->batch),
+                          dim3(128), mma_smem_bytes<HD>(), s, a, static_cast<bf16*>(c->attn));
+}
+
+template <int HD>
+cudaError_t run_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
+    switch (a.splits) {
+        case 1: return launch_mma<HD, 1>(c, a, s);
+        case 2: return launch_mma<HD, 2>(c, a, s);
+        case 4: return launch_mma<HD, 4>(c, a, s);
+        case 8: return launch_mma<HD, 8>(c, a, s);
+        default: return launch_mma<HD, 16>(c, a, s);
+    }
+}
+
+// Largest cluster the device schedules for the attention kernel (16 where non-portable clusters
+// of that size fit, else 8).
+template <int HD>
+int max_attention_cluster() {
+    static int cached = 0;
+    if (cached) return cached;
+    cached = 8;
+    if (cudaFuncSetAttribute(attn_mma_kernel<HD, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)mma_smem_bytes<HD>()) == cudaSuccess &&
+        cudaFuncSetAttribute(attn_mma_kernel<HD, 16>, cudaFuncAttributeNonPortableClusterSizeAllowed,
+                             1) == cudaSuccess) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(16, 1, 1);
+        cfg.blockDim = dim3(128);
+        cfg.dynamicSmemBytes = mma_smem_bytes<HD>();
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 16;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, attn_mma_kernel<HD, 16>, &cfg) == cudaSuccess && n > 0)
+            cached = 16;
+    }
+    cudaGetLastError();
+    return cached;
 }
 
 template <class T, int HD>
@@ -479,16 +524,17 @@ int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub)
     return std::max(1, sp);
 }
 
-// Tensor-core path: the splits of one (sequence, head, query tile) are one cluster of 1, 2, 4 or 8
-// CTAs: as many as needed for about two CTAs per SM, at most one per 64-key tile.
-int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int len_ub) {
+// Tensor-core path: the splits of one (sequence, head, query tile) are one cluster of 1, 2, 4, 8
+// or 16 CTAs: as many as needed for about two CTAs per SM, at most one per 64-key tile.
+int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int len_ub,
+                             int max_cluster) {
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + kQT - 1) / kQT;
     const int base = batch * g.n_kv_heads * q_tiles;
     const int want = (2 * num_sms + base - 1) / base;
     const int tiles = (len_ub + g.block + kKT - 1) / kKT;
     int sp = 1;
-    while (sp < 8 && sp < want && 2 * sp <= tiles) sp *= 2;
+    while (sp < max_cluster && sp < want && 2 * sp <= tiles) sp *= 2;
     return sp;
 }
 
@@ -516,7 +562,8 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
         a.splits = attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
         return g.head_dim == 64 ? run_simt<float, 64>(c, a, s) : run_simt<float, 128>(c, a, s);
     }
-    a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub);
+    const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
+    a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc);
     return g.head_dim == 64 ? run_mma<64>(c, a, s) : run_mma<128>(c, a, s);
 }
 

@@ -53,48 +53,57 @@ __global__ void fuse_begin_kernel(int32_t* ctx_len, int32_t* app_base, int32_t* 
 }
 
 constexpr int kFuseCH = 512;       // features per CTA (64 threads x 8)
+constexpr int kFuseGroups = 4;     // thread groups splitting the T target layers
 
 // One position is handled by a cluster of ceil(d / 512) CTAs (at most 8 for d <= 4096); CTA c owns
-// features [512 c, 512 c + 512). Each CTA stages its slice of all T target rows in shared memory
-// with cp.async (one round trip), forms the D weighted sums in registers (up to 8 draft layers
-// per pass), reduces its partial sums of squares, and the CTAs of the cluster exchange those
-// partials through distributed shared memory (summed in rank order) before normalising.
+// features [512 c, 512 c + 512). Each CTA (256 threads) stages its slice of all T target rows and
+// of the D gain rows in shared memory with cp.async (one round trip). Thread group q (64 threads,
+// 8 features each) forms the D weighted sums over target layers j = q, q + 4, ...; the four
+// partial sums are added in group order, the CTA reduces its partial sums of squares, and the
+// CTAs of the cluster exchange those partials through distributed shared memory (one gather,
+// summed in rank order) before normalising.
 template <class T, int DMAX>
-__global__ void __launch_bounds__(64) fuse_layers_kernel(
+__global__ void __launch_bounds__(256) fuse_layers_kernel(
     const T* __restrict__ H, const float* __restrict__ alpha, const T* __restrict__ gain,
     T* __restrict__ F, T* __restrict__ F_out, const int32_t* __restrict__ app_cnt, int D, int Tn,
     int batch, int n_max, int d, long long f_layer_rows, float eps) {
     pdl_trigger();
     pdl_wait();
     extern __shared__ __align__(16) uint8_t smem[];
-    T* sh = reinterpret_cast<T*>(smem);          // [Tn][kFuseCH]
+    T* sh = reinterpret_cast<T*>(smem);          // [Tn][kFuseCH] target rows, then [D][kFuseCH] gains
+    T* sg = sh + (size_t)Tn * kFuseCH;
+    float* sacc = reinterpret_cast<float*>(sg + (size_t)D * kFuseCH);  // [3][DMAX][8][64]
     __shared__ float s_alpha[16 * 64];
     __shared__ float red[2][DMAX];
-    __shared__ float ss_cta[DMAX];
+    __shared__ float ss_cta[DMAX];               // this CTA's partial sums of squares
+    __shared__ float part[8][DMAX];              // every cluster rank's partials
+    __shared__ float inv_s[DMAX];
     cg::cluster_group cluster = cg::this_cluster();
     const int C = (int)cluster.num_blocks(), cr = (int)cluster.block_rank();
     const int r = blockIdx.y, b = blockIdx.z;
     if (r >= app_cnt[b]) return;                 // the same for every CTA of the cluster
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int tid = threadIdx.x, q = tid >> 6, t64 = tid & 63;
+    const int lane = tid & 31, warp = tid >> 5;
     const int f0 = cr * kFuseCH, nf = min(kFuseCH, d - f0);
     const size_t row = (size_t)b * n_max + r;
     const size_t lstride = (size_t)batch * n_max * d;
     constexpr int EPC = 16 / sizeof(T);          // elements per 16-byte copy
-    const int per_row = nf / EPC;
+    const int per_row = nf / EPC;                // <= 64 (bf16) or 128 (fp32)
     const uint32_t ssh = (uint32_t)__cvta_generic_to_shared(sh);
-    for (int idx = tid; idx < Tn * per_row; idx += blockDim.x) {
-        const int j = idx / per_row, p = idx % per_row;
-        const T* src = H + (size_t)j * lstride + row * d + f0 + p * EPC;
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
-                         ssh + (uint32_t)((j * kFuseCH + p * EPC) * sizeof(T))),
-                     "l"(src)
-                     : "memory");
+    // all T target rows of this slice and all D gain rows, one round trip
+    for (int j = q; j < Tn + D; j += kFuseGroups) {
+        const T* src = j < Tn ? H + (size_t)j * lstride + row * d + f0 : gain + (size_t)(j - Tn) * d + f0;
+        for (int p = t64; p < per_row; p += 64)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                             ssh + (uint32_t)((j * kFuseCH + p * EPC) * sizeof(T))),
+                         "l"(src + p * EPC)
+                         : "memory");
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     for (int k = tid; k < D * Tn; k += blockDim.x) s_alpha[k] = alpha[k];
     asm volatile("cp.async.wait_group 0;" ::: "memory");
     __syncthreads();
-    const int e0 = tid * 8;
+    const int e0 = t64 * 8;
     const bool act = e0 < nf;
     for (int i0 = 0; i0 < D; i0 += DMAX) {
         const int nd = min(DMAX, D - i0);
@@ -104,39 +113,61 @@ __global__ void __launch_bounds__(64) fuse_layers_kernel(
 #pragma unroll
             for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
         if (act) {
-            for (int j = 0; j < Tn; ++j) {
-                float h[8];
+            for (int j = q; j < Tn; j += kFuseGroups) {
+                float h[8], a[DMAX];
                 load8(sh + j * kFuseCH + e0, h);
 #pragma unroll
-                for (int i = 0; i < DMAX; ++i) {
-                    if (i < nd) {
-                        const float a = s_alpha[(i0 + i) * Tn + j];
+                for (int i = 0; i < DMAX; ++i) a[i] = i < nd ? s_alpha[(i0 + i) * Tn + j] : 0.f;
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a, h[e], acc[i][e]);
-                    }
-                }
+                for (int i = 0; i < DMAX; ++i)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a[i], h[e], acc[i][e]);
             }
         }
+        // groups 1..3 hand their partial sums to group 0, which adds them in group order
+        if (q > 0) {
 #pragma unroll
-        for (int i = 0; i < DMAX; ++i) {
-            float v = 0.f;
+            for (int i = 0; i < DMAX; ++i)
 #pragma unroll
-            for (int e = 0; e < 8; ++e) v = fmaf(acc[i][e], acc[i][e], v);
-            v = warp_sum(v);
-            if (lane == 0) red[warp][i] = v;
+                for (int e = 0; e < 8; ++e) sacc[(((q - 1) * DMAX + i) * 8 + e) * 64 + t64] = acc[i][e];
+        }
+        __syncthreads();
+        if (q == 0) {
+#pragma unroll
+            for (int g2 = 0; g2 < kFuseGroups - 1; ++g2)
+#pragma unroll
+                for (int i = 0; i < DMAX; ++i)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc[i][e] += sacc[((g2 * DMAX + i) * 8 + e) * 64 + t64];
+#pragma unroll
+            for (int i = 0; i < DMAX; ++i) {
+                float v = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v = fmaf(acc[i][e], acc[i][e], v);
+                v = warp_sum(v);
+                if (lane == 0) red[warp][i] = v;
+            }
         }
         __syncthreads();
         if (tid < DMAX) ss_cta[tid] = red[0][tid] + red[1][tid];
         cluster.sync();
-        if (act) {
+        // gather every rank's partials in one round of DSMEM loads, then sum in rank order
+        for (int k = tid; k < C * nd; k += blockDim.x)
+            part[k / nd][k % nd] = cluster.map_shared_rank(ss_cta, k / nd)[k % nd];
+        __syncthreads();
+        if (tid < nd) {
+            float tot = 0.f;
+            for (int c = 0; c < C; ++c) tot += part[c][tid];
+            inv_s[tid] = inv_rms(tot, d, eps);
+        }
+        __syncthreads();
+        if (q == 0 && act) {
 #pragma unroll
             for (int i = 0; i < DMAX; ++i) {
                 if (i >= nd) break;
-                float tot = 0.f;
-                for (int c = 0; c < C; ++c) tot += cluster.map_shared_rank(ss_cta, c)[i];
-                const float inv = inv_rms(tot, d, eps);
                 float g[8], o[8];
-                load8(gain + (size_t)(i0 + i) * d + f0 + e0, g);
+                load8(sg + (i0 + i) * kFuseCH + e0, g);
+                const float inv = inv_s[i];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) o[e] = g[e] * (acc[i][e] * inv);
                 store8(F + ((size_t)(i0 + i) * f_layer_rows + row) * d + f0 + e0, o);
@@ -153,7 +184,8 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
                           cudaStream_t s) {
     const dflare_config& g = c->cfg;
     const int C = (g.d + kFuseCH - 1) / kFuseCH;
-    const size_t smem = (size_t)g.n_target_layers * kFuseCH * sizeof(T);
+    const size_t smem = (size_t)(g.n_target_layers + g.n_draft_layers) * kFuseCH * sizeof(T) +
+                        (size_t)(kFuseGroups - 1) * 8 * 8 * 64 * sizeof(float);
     const T* H = static_cast<const T*>(hidden);
     const T* gain = static_cast<const T*>(c->w.fuse_norm);
     T* F = static_cast<T*>(c->fused);
@@ -163,12 +195,13 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
     if (!configured) {
         for (auto k : {fuse_layers_kernel<T, 4>, fuse_layers_kernel<T, 8>}) {
             cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)(64 * kFuseCH * sizeof(T)));
+                                                 (int)((64 + 16) * kFuseCH * sizeof(T) +
+                                                       (kFuseGroups - 1) * 8 * 8 * 64 * 4));
             if (e != cudaSuccess) return e;
         }
         configured = true;
     }
-    return launch_cluster(c->pdl, C, kern, dim3(C, n_max, c->batch), dim3(64), smem, s, H,
+    return launch_cluster(c->pdl, C, kern, dim3(C, n_max, c->batch), dim3(256), smem, s, H,
                           (const float*)c->alpha, gain, F, Fo, (const int32_t*)c->app_cnt,
                           g.n_draft_layers, g.n_target_layers, c->batch, n_max, g.d,
                           (long long)g.max_fuse_rows, g.rms_eps);
