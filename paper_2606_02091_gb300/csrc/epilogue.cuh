@@ -70,30 +70,33 @@ __device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float*
             }
             const int j = col % hd, jj = j % half;
             const int tp = j < half ? t + half : t - half;
-            float cs[NC], sn[NC];
-            if (rot) {
-                int pos[NC];
-#pragma unroll
-                for (int c = 0; c < NC; ++c) {
-                    const int tok = tok0 + min(c, nvalid - 1);
-                    const int b = tok / ep.block;
-                    pos[c] = ep.ctx_len[b] + (tok - b * ep.block);
-                }
-#pragma unroll
-                for (int c = 0; c < NC; ++c) {
-                    cs[c] = ep.rope_cos[(size_t)pos[c] * half + jj];
-                    sn[c] = ep.rope_sin[(size_t)pos[c] * half + jj];
-                }
-            }
-#pragma unroll
-            for (int c = 0; c < NC; ++c) {
-                if (c >= nvalid) break;
-                float v = tile[c * 128 + t];
+            // eight tokens at a time: their positions and rotary factors are loaded together
+            for (int h0 = 0; h0 < nvalid; h0 += 8) {
+                float cs[8], sn[8];
                 if (rot) {
-                    const float y = tile[c * 128 + tp];
-                    v = j < half ? v * cs[c] - y * sn[c] : v * cs[c] + y * sn[c];
+                    int pos[8];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const int tok = tok0 + min(h0 + c, nvalid - 1);
+                        const int b = tok / ep.block;
+                        pos[c] = ep.ctx_len[b] + (tok - b * ep.block);
+                    }
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        cs[c] = ep.rope_cos[(size_t)pos[c] * half + jj];
+                        sn[c] = ep.rope_sin[(size_t)pos[c] * half + jj];
+                    }
                 }
-                dst[(size_t)(tok0 + c) * ld + col] = from_f<T>(v);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    if (h0 + c >= nvalid) break;
+                    float v = tile[(h0 + c) * 128 + t];
+                    if (rot) {
+                        const float y = tile[(h0 + c) * 128 + tp];
+                        v = j < half ? v * cs[c] - y * sn[c] : v * cs[c] + y * sn[c];
+                    }
+                    dst[(size_t)(tok0 + h0 + c) * ld + col] = from_f<T>(v);
+                }
             }
         } break;
         case EPI_KV_APPEND: {
@@ -103,35 +106,37 @@ __device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float*
             const int tp = j < half ? t + half : t - half;
             const int hkv = ep.d_kv / hd;
             T* cache = reinterpret_cast<T*>(is_k ? ep.kcache : ep.vcache);
-            int pos[NC], ok[NC], bb[NC];
+            for (int h0 = 0; h0 < nvalid; h0 += 8) {
+                int pos[8], ok[8], bb[8];
 #pragma unroll
-            for (int c = 0; c < NC; ++c) {
-                const int tok = tok0 + min(c, nvalid - 1);
-                const int b = tok / ep.n_max, r = tok - b * ep.n_max;
-                bb[c] = b;
-                ok[c] = c < nvalid && r < ep.app_cnt[b];
-                pos[c] = ep.app_base[b] + r;
-            }
-            float cs[NC], sn[NC];
-            if (is_k) {
-#pragma unroll
-                for (int c = 0; c < NC; ++c) {
-                    const int p = ok[c] ? pos[c] : 0;
-                    cs[c] = ep.rope_cos[(size_t)p * half + jj];
-                    sn[c] = ep.rope_sin[(size_t)p * half + jj];
+                for (int c = 0; c < 8; ++c) {
+                    const int tok = tok0 + min(h0 + c, nvalid - 1);
+                    const int b = tok / ep.n_max, r = tok - b * ep.n_max;
+                    bb[c] = b;
+                    ok[c] = h0 + c < nvalid && r < ep.app_cnt[b];
+                    pos[c] = ep.app_base[b] + r;
                 }
-            }
-#pragma unroll
-            for (int c = 0; c < NC; ++c) {
-                if (!ok[c]) continue;
-                float v = tile[c * 128 + t];
+                float cs[8], sn[8];
                 if (is_k) {
-                    const float y = tile[c * 128 + tp];
-                    v = j < half ? v * cs[c] - y * sn[c] : v * cs[c] + y * sn[c];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const int p = ok[c] ? pos[c] : 0;
+                        cs[c] = ep.rope_cos[(size_t)p * half + jj];
+                        sn[c] = ep.rope_sin[(size_t)p * half + jj];
+                    }
                 }
-                const size_t row =
-                    (((size_t)group * ep.max_batch + bb[c]) * hkv + g) * ep.max_ctx + pos[c];
-                cache[row * hd + j] = from_f<T>(v);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    if (!ok[c]) continue;
+                    float v = tile[(h0 + c) * 128 + t];
+                    if (is_k) {
+                        const float y = tile[(h0 + c) * 128 + tp];
+                        v = j < half ? v * cs[c] - y * sn[c] : v * cs[c] + y * sn[c];
+                    }
+                    const size_t row =
+                        (((size_t)group * ep.max_batch + bb[c]) * hkv + g) * ep.max_ctx + pos[c];
+                    cache[row * hd + j] = from_f<T>(v);
+                }
             }
         } break;
         default:

@@ -177,7 +177,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const uint32_t sbase = raw + pad;
     const int S = args.stages;
     float* epi = reinterpret_cast<float*>(smem + (size_t)S * args.stage_bytes);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + 2 * kChunk * 128);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + args.n_a * kChunk * 128);
     uint32_t* misc = reinterpret_cast<uint32_t*>(bars + 2 * S + 5);
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -220,6 +220,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     if (warp == 4) {
         if (lane == 0) {
             // ---------------- TMA producer
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+            if (args.n_a == 2)
+                asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA2)) : "memory");
             int stage = 0;
             uint32_t phase = 0, issued = 0, issued_phase = 0;
             bool ok = true;
@@ -516,15 +520,18 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
             best = spn;
         }
     }
-    // default: four 64-wide k-blocks per stage (512 contiguous bytes of every weight row per
-    // stage; 128-byte rows per request leave DRAM bandwidth unused), fewer when the stage would
-    // not fit twice in shared memory
+    // Shared-memory budget: up to 227 KB (one CTA per SM; measured faster than two smaller CTAs
+    // per SM, with or without programmatic dependent launch). Stage size: four 64-wide k-blocks
+    // (512 contiguous bytes of every weight row; 128-byte rows per request leave DRAM bandwidth
+    // unused), fewer when two stages do not fit.
+    const int epi_bytes = a.n_a * kChunk * 128 * 4;
+    const int fixed = 1024 + epi_bytes + 8 * (2 * kMaxStages + 5) + 16;
+    const int budget = g.max_smem > 0 ? std::min(g.max_smem, kSmemLimit) : kSmemLimit;
     if (g.kbs > 0) {
         a.kbs = g.kbs;
     } else {
         a.kbs = 4;
-        while (a.kbs > 1 && 2 * a.kbs * (kBM * kBK * 2 * a.n_a + a.bn * kBK * 2) >
-                                kSmemLimit - (1024 + 2 * kChunk * 128 * 4 + 8 * (2 * kMaxStages + 5) + 16))
+        while (a.kbs > 1 && 2 * a.kbs * (kBM * kBK * 2 * a.n_a + a.bn * kBK * 2) > budget - fixed)
             a.kbs >>= 1;
     }
     a.kb_per_split = (a.k_blocks + best - 1) / best;
@@ -536,9 +543,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     a.stage_bytes = (uint32_t)a.kbs * (a_bytes * a.n_a + a.b_bytes);
     a.tx_bytes = a.stage_bytes;
     a.evict_first = g.evict_first >= 0 ? 1 : 0;
-    const int epi_bytes = 2 * kChunk * 128 * 4;
-    const int fixed = 1024 + epi_bytes + 8 * (2 * kMaxStages + 5) + 16;
-    a.stages = std::min(kMaxStages, (kSmemLimit - fixed) / (int)a.stage_bytes);
+    a.stages = std::min(kMaxStages, (budget - fixed) / (int)a.stage_bytes);
     if (a.stages < 2) {
         if (why) *why = "tcgen05 GEMM: tile does not fit in shared memory";
         return cudaErrorInvalidValue;
