@@ -220,6 +220,32 @@ dflare_status dflare_synthetic_target(const int32_t* draft_tokens_dev, const uin
                                       int32_t* step_dev, uint32_t threshold, int batch, int block,
                                       int32_t* target_argmax_dev, void* stream);
 
+/* Largest number of rows dflare_argmax_noalloc accepts. */
+#define DFLARE_NOALLOC_MAX_ROWS 4096
+
+/*
+ * Greedy argmax over rows of fp32 logits that allocates nothing (the paper has no counterpart:
+ * this is a library utility, with the same tie rule as the drafted tokens -- the lowest token id
+ * among equal maxima).
+ *   logits_dev  [rows][vocab] fp32 (caller-owned, device)
+ *   tokens_dev  [rows] int32 out (caller-owned, device)
+ * It is for callers that cannot allocate device memory: serving loops that fix their memory
+ * budget at start-up and forbid allocation afterwards, code that must avoid the implicit
+ * device synchronisation of cudaMalloc/cudaFree, or allocator-free embeddings. The call uses a
+ * fixed scratch array compiled into the library (one 8-byte slot per row plus a counter,
+ * DFLARE_NOALLOC_MAX_ROWS rows, held by every GPU that loads the library until the process
+ * exits); it calls no cudaMalloc, cudaFree or allocating library routine.
+ * - rows > DFLARE_NOALLOC_MAX_ROWS returns DFLARE_ECAPACITY (message in dflare_last_error(NULL)).
+ * - The first call on a device looks up the scratch array's device address with that device
+ *   current; make that first call before capturing a stream into a CUDA graph.
+ * - Every call on a device shares the same scratch array, which keeps the last call's contents;
+ *   each call clears the part it uses on `stream` before its kernel. Calls that overlap on the
+ *   GPU (on different streams, or from several host threads) race on the scratch and give wrong
+ *   tokens: serialise them.
+ */
+dflare_status dflare_argmax_noalloc(const float* logits_dev, int rows, int vocab,
+                                    int32_t* tokens_dev, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -13,7 +13,7 @@ from . import _lib
 from ._lib import (  # noqa: F401
     DFlareError, DFLARE_BF16, DFLARE_F32, FLAG_NO_BLOCK_ROPE, FLAG_RAW_FUSION, FLAG_SIMT_GEMM,
     FLAG_SERIAL_LAUNCH,
-    DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT, EXPORTS, WEIGHT_FIELDS, load,
+    DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT, EXPORTS, WEIGHT_FIELDS, NOALLOC_MAX_ROWS, load,
 )
 
 
@@ -151,6 +151,18 @@ class DFlare:
         if st not in (_lib.DFLARE_OK, _lib.DFLARE_EDEVICE):
             self._check(st)
         return bits.value
+
+
+def argmax_noalloc(logits, tokens_out, stream=None):
+    """Greedy argmax of [rows][vocab] fp32 device logits into int32 tokens_out without any device
+    allocation (see dflare_argmax_noalloc: fixed scratch, at most NOALLOC_MAX_ROWS rows)."""
+    import torch
+    _need_cuda("logits", logits, torch.float32)
+    _need_cuda("tokens_out", tokens_out, torch.int32)
+    rows, vocab = logits.shape[0], logits.shape[-1]
+    rows = logits.numel() // vocab
+    _lib.check(load().dflare_argmax_noalloc(_ptr(logits), rows, vocab, _ptr(tokens_out),
+                                            _stream(stream)))
 
 
 def synthetic_target(draft_tokens, u, r, last, step, threshold, batch, block, target_out,

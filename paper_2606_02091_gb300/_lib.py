@@ -29,7 +29,9 @@ STATUS_NAMES = {0: "DFLARE_OK", 1: "DFLARE_EINVAL", 2: "DFLARE_ECAPACITY", 3: "D
 EXPORTS = ("dflare_create", "dflare_destroy", "dflare_set_weights", "dflare_reset",
            "dflare_fuse_context", "dflare_draft_block", "dflare_verify_accept", "dflare_read_kv",
            "dflare_ctx_lens", "dflare_device_error", "dflare_last_error",
-           "dflare_synthetic_target", "dflare_set_trace")
+           "dflare_synthetic_target", "dflare_set_trace", "dflare_argmax_noalloc")
+
+NOALLOC_MAX_ROWS = 4096
 
 TRACE_FN = ctypes.CFUNCTYPE(None, ctypes.c_void_p, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p)
 
@@ -85,6 +87,7 @@ def load():
         "dflare_last_error": [vp],
         "dflare_synthetic_target": [vp, vp, vp, vp, i32, vp, u32, i32, i32, vp, vp],
         "dflare_set_trace": [vp, TRACE_FN, vp],
+        "dflare_argmax_noalloc": [vp, i32, i32, vp, vp],
     }
     for name, args in sig.items():
         f = getattr(L, name)

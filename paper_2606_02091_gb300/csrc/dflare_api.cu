@@ -149,6 +149,10 @@ const uint8_t* at(const void* base, size_t elems, size_t esz) {
 
 }  // namespace
 
+namespace dfl {
+void noalloc_set_error(const std::string& message) { g_create_error = message; }
+}  // namespace dfl
+
 extern "C" {
 
 dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {

@@ -151,6 +151,9 @@ inline cudaError_t launch_cluster(bool pdl, int cluster_x, void (*kernel)(KArgs.
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// Sets the message dflare_last_error(NULL) returns (for entry points without a context).
+void noalloc_set_error(const std::string& message);
+
 // launchers (each returns the first CUDA error it meets)
 cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why);
 cudaError_t launch_gemm_simt(dflare_ctx* c, const GemmDesc& g, cudaStream_t s);
