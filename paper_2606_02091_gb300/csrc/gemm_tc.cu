@@ -11,18 +11,22 @@
 // walks the units. Per CTA (192 threads):
 //   warp 4    TMA producer: per stage, kbs consecutive 128x64 bf16 weight tiles (+ the up tiles
 //             for SwiGLU) and the matching bn x 64 activation tiles, 128-byte swizzled; weights
-//             carry an L2 evict-first hint (each byte is read once per step).
+//             carry an L2 evict-first hint (each byte is read once per step). Weights do not
+//             depend on the previous kernel: the first ring of stages gets its weight tiles
+//             before griddepcontrol.wait, the activation tiles after it.
 //   warp 5    allocates TMEM, issues tcgen05.mma (one thread), commits stages back to the
 //             producer and finished accumulators to the epilogue; two accumulator buffers let
 //             the next unit's MMAs overlap the current unit's epilogue.
 //   warps 0-3 epilogue: tcgen05.ld of the accumulator (thread t = TMEM lane t = feature t),
 //             split-K reduction through a global workspace (the last CTA of a tile sums the
 //             partials in split order, so results are deterministic), then the fused epilogue.
+//             Residual rows are loaded before the accumulator is waited for.
 // Every wait on an mbarrier is bounded (2 s); on a timeout the CTA sets DFLARE_DEVERR_TIMEOUT,
 // stops issuing work, drains what it issued and frees its TMEM.
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstring>
 #include <mutex>
 
 #include "epilogue.cuh"
@@ -37,15 +41,17 @@ constexpr int kChunk = 16;
 constexpr int kMaxStages = 8;
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 constexpr int kSmemLimit = 227 * 1024;
+constexpr uint32_t kABytes = kBM * kBK * 2;   // one 128 x 64 bf16 weight tile
 
 struct TcArgs {
+    CUtensorMap map_a, map_a2, map_b;   // weights, up weights (SwiGLU), activations
     int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks;
     int bn, n_a, stages, n_bufs, tmem_cols;
     int kbs;                   // 64-wide k-blocks per pipeline stage
     uint32_t b_bytes;          // bytes of one activation sub-tile (bn x 64 bf16)
     int evict_first;           // stream the weights with an L2 evict-first policy
     uint32_t idesc;
-    uint32_t stage_bytes, tx_bytes;
+    uint32_t stage_bytes;
     float* ws;
     uint32_t* tile_cnt;
     uint32_t* err;
@@ -150,10 +156,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
 }
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+// The kernel's loop constants, copied out of the parameter block into registers (the block is
+// addressed for the tensor maps, so every asm with a memory clobber would otherwise reload them).
+struct Geom {
+    int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks, n_a, kbs, bn, n_bufs;
+    uint32_t b_bytes, stage_bytes, idesc;
+};
 struct Unit {
     int group, n_tile, tok_tile, split, tile_id, kb0, kb1;
 };
-__device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
+__device__ __forceinline__ Unit decode_unit(const Geom& a, int u) {
     Unit x;
     x.split = u % a.splits;
     x.tile_id = u / a.splits;
@@ -167,17 +185,48 @@ __device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
     return x;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
-               const __grid_constant__ CUtensorMap tmB, const TcArgs args) {
+// EPI_RESID with the residual values already in registers: resid[tok][n] += acc.
+__device__ __forceinline__ void load_resid(const EpiParams& ep, int n_tile, int tok0, int t, float* r) {
+    const int n = n_tile * 128 + t;
+    const int nvalid = min(kChunk, ep.m_tok - tok0);
+#pragma unroll
+    for (int c = 0; c < kChunk; ++c)
+        r[c] = (n < ep.n && c < nvalid) ? ep.resid[(size_t)(tok0 + c) * ep.ld_resid + n] : 0.f;
+}
+__device__ __forceinline__ void resid_epilogue(const EpiParams& ep, const float* tile, int n_tile,
+                                               int tok0, int t, const float* r) {
+    const int n = n_tile * 128 + t;
+    if (n >= ep.n) return;
+    const int nvalid = min(kChunk, ep.m_tok - tok0);
+#pragma unroll
+    for (int c = 0; c < kChunk; ++c)
+        if (c < nvalid) ep.resid[(size_t)(tok0 + c) * ep.ld_resid + n] = r[c] + tile[c * 128 + t];
+}
+
+__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs args) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
     uint8_t* smem = smem_raw + pad;
     const uint32_t sbase = raw + pad;
+    Geom G;
+    G.n_units = args.n_units;
+    G.n_tiles = args.n_tiles;
+    G.tok_tiles = args.tok_tiles;
+    G.splits = args.splits;
+    G.kb_per_split = args.kb_per_split;
+    G.k_blocks = args.k_blocks;
+    G.n_a = args.n_a;
+    G.kbs = args.kbs;
+    G.bn = args.bn;
+    G.n_bufs = args.n_bufs;
+    G.b_bytes = args.b_bytes;
+    G.stage_bytes = args.stage_bytes;
+    G.idesc = args.idesc;
+    uint32_t* const err = args.err;
     const int S = args.stages;
-    float* epi = reinterpret_cast<float*>(smem + (size_t)S * args.stage_bytes);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + args.n_a * kChunk * 128);
+    float* epi = reinterpret_cast<float*>(smem + (size_t)S * G.stage_bytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + G.n_a * kChunk * 128);
     uint32_t* misc = reinterpret_cast<uint32_t*>(bars + 2 * S + 5);
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -185,10 +234,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * S + b); };
     auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * S + 2 + b); };
     const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
-    const uint32_t a_bytes = kBM * kBK * 2;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     pdl_trigger();
+    if (warp == 4 && lane == 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&args.map_a)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&args.map_b)) : "memory");
+        if (G.n_a == 2)
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&args.map_a2)) : "memory");
+    }
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_bar(s), 1);
@@ -216,21 +270,23 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     tc_fence_after();
     const uint32_t tmem = misc[0];
     volatile int* abort_flag = reinterpret_cast<volatile int*>(&misc[1]);
+    const int acc_cols = G.n_a * G.bn;
 
     if (warp == 4) {
         if (lane == 0) {
             // ---------------- TMA producer
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
-            if (args.n_a == 2)
-                asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA2)) : "memory");
+            const CUtensorMap* mA = &args.map_a;
+            const CUtensorMap* mA2 = &args.map_a2;
+            const CUtensorMap* mB = &args.map_b;
             int stage = 0;
             uint32_t phase = 0, issued = 0, issued_phase = 0;
             bool ok = true;
             uint64_t policy = 0;
-            if (args.evict_first)
+            const bool evict_first = args.evict_first != 0;
+            if (evict_first)
                 asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
-            const uint32_t a_sub = a_bytes, b_base = a_bytes * args.n_a * args.kbs;
+            const uint32_t b_base = kABytes * G.n_a * G.kbs;
+            const uint32_t tx = kABytes * G.n_a + G.b_bytes;
             // Weights do not depend on the previous kernel: the first ring of stages gets its
             // weight tiles before griddepcontrol.wait, the activation tiles after it.
             int pend_kx[kMaxStages], pend_nk[kMaxStages], pend_tok[kMaxStages], pend_grp[kMaxStages];
@@ -239,34 +295,31 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             bool waited = false;
             auto load_b = [&](uint32_t st, int kx0, int nk, int tok_tile, int group, uint32_t bar) {
                 for (int j = 0; j < nk; ++j)
-                    tma_load_3d(st + b_base + j * args.b_bytes, &tmB, kx0 + j * kBK,
-                                tok_tile * args.bn, group, bar);
+                    tma_load_3d(st + b_base + j * G.b_bytes, mB, kx0 + j * kBK, tok_tile * G.bn, group, bar);
             };
-            for (int u = blockIdx.x; u < args.n_units && ok; u += gridDim.x) {
-                const Unit x = decode_unit(args, u);
-                for (int kb = x.kb0; kb < x.kb1; kb += args.kbs) {
-                    const int nk = min(args.kbs, x.kb1 - kb);
-                    if (!bar_wait(empty_bar(stage), phase ^ 1u, abort_flag, args.err)) {
+            for (int u = blockIdx.x; u < G.n_units && ok; u += gridDim.x) {
+                const Unit x = decode_unit(G, u);
+                for (int kb = x.kb0; kb < x.kb1; kb += G.kbs) {
+                    const int nk = min(G.kbs, x.kb1 - kb);
+                    if (!bar_wait(empty_bar(stage), phase ^ 1u, abort_flag, err)) {
                         ok = false;
                         break;
                     }
-                    const uint32_t st = sbase + (uint32_t)stage * args.stage_bytes;
-                    mbar_expect_tx(full_bar(stage),
-                                   (uint32_t)nk * (a_bytes * args.n_a + args.b_bytes));
+                    const uint32_t st = sbase + (uint32_t)stage * G.stage_bytes;
+                    mbar_expect_tx(full_bar(stage), (uint32_t)nk * tx);
                     for (int j = 0; j < nk; ++j) {
                         const int kx = (kb + j) * kBK;
-                        if (args.evict_first) {
-                            tma_load_3d_hint(st + j * a_sub, &tmA, kx, x.n_tile * kBM, x.group,
+                        if (evict_first) {
+                            tma_load_3d_hint(st + j * kABytes, mA, kx, x.n_tile * kBM, x.group,
                                              full_bar(stage), policy);
-                            if (args.n_a == 2)
-                                tma_load_3d_hint(st + (args.kbs + j) * a_sub, &tmA2, kx,
-                                                 x.n_tile * kBM, x.group, full_bar(stage), policy);
+                            if (G.n_a == 2)
+                                tma_load_3d_hint(st + (G.kbs + j) * kABytes, mA2, kx, x.n_tile * kBM,
+                                                 x.group, full_bar(stage), policy);
                         } else {
-                            tma_load_3d(st + j * a_sub, &tmA, kx, x.n_tile * kBM, x.group,
-                                        full_bar(stage));
-                            if (args.n_a == 2)
-                                tma_load_3d(st + (args.kbs + j) * a_sub, &tmA2, kx, x.n_tile * kBM,
-                                            x.group, full_bar(stage));
+                            tma_load_3d(st + j * kABytes, mA, kx, x.n_tile * kBM, x.group, full_bar(stage));
+                            if (G.n_a == 2)
+                                tma_load_3d(st + (G.kbs + j) * kABytes, mA2, kx, x.n_tile * kBM, x.group,
+                                            full_bar(stage));
                         }
                     }
                     if (waited) {
@@ -281,7 +334,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                             pdl_wait();
                             waited = true;
                             for (int i = 0; i < npend; ++i)
-                                load_b(sbase + pend_st[i] * args.stage_bytes, pend_kx[i], pend_nk[i],
+                                load_b(sbase + pend_st[i] * G.stage_bytes, pend_kx[i], pend_nk[i],
                                        pend_tok[i], pend_grp[i], full_bar(pend_st[i]));
                         }
                     }
@@ -296,15 +349,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (!waited) {
                 pdl_wait();
                 for (int i = 0; i < npend; ++i)
-                    load_b(sbase + pend_st[i] * args.stage_bytes, pend_kx[i], pend_nk[i], pend_tok[i],
+                    load_b(sbase + pend_st[i] * G.stage_bytes, pend_kx[i], pend_nk[i], pend_tok[i],
                            pend_grp[i], full_bar(pend_st[i]));
             }
             // make sure no copy is still landing in shared memory when the CTA exits
             for (int s = 0; s < S; ++s)
                 if (issued & (1u << s)) {
                     volatile int never = 0;
-                    bar_wait(full_bar(s), (issued_phase >> s) & 1u, ok ? &never : abort_flag,
-                             args.err);
+                    bar_wait(full_bar(s), (issued_phase >> s) & 1u, ok ? &never : abort_flag, err);
                 }
         }
     } else if (warp == 5) {
@@ -312,32 +364,30 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             // ---------------- MMA issuer
             int stage = 0, acc = 0;
             uint32_t phase = 0, acc_phase = 0;
-            const int acc_cols = args.n_a * args.bn;
             bool ok = true;
-            for (int u = blockIdx.x; u < args.n_units && ok; u += gridDim.x) {
-                const Unit x = decode_unit(args, u);
-                if (!bar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, args.err)) break;
+            const uint32_t b_base = kABytes * G.n_a * G.kbs;
+            for (int u = blockIdx.x; u < G.n_units && ok; u += gridDim.x) {
+                const Unit x = decode_unit(G, u);
+                if (!bar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d0 = tmem + (uint32_t)(acc * acc_cols);
-                for (int kb = x.kb0; kb < x.kb1; kb += args.kbs) {
-                    const int nk = min(args.kbs, x.kb1 - kb);
-                    if (!bar_wait(full_bar(stage), phase, abort_flag, args.err)) {
+                for (int kb = x.kb0; kb < x.kb1; kb += G.kbs) {
+                    const int nk = min(G.kbs, x.kb1 - kb);
+                    if (!bar_wait(full_bar(stage), phase, abort_flag, err)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t st = sbase + (uint32_t)stage * args.stage_bytes;
-                    const uint32_t b_base = a_bytes * args.n_a * args.kbs;
+                    const uint32_t st = sbase + (uint32_t)stage * G.stage_bytes;
                     for (int j = 0; j < nk; ++j) {
-                        const uint64_t da = smem_desc(st + j * a_bytes);
-                        const uint64_t da2 = smem_desc(st + (args.kbs + j) * a_bytes);
-                        const uint64_t db = smem_desc(st + b_base + j * args.b_bytes);
+                        const uint64_t da = smem_desc(st + j * kABytes);
+                        const uint64_t da2 = smem_desc(st + (G.kbs + j) * kABytes);
+                        const uint64_t db = smem_desc(st + b_base + j * G.b_bytes);
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k) {
                             const uint32_t accum = (kb > x.kb0 || j > 0 || k > 0) ? 1u : 0u;
-                            umma_bf16(d0, da + 2 * k, db + 2 * k, args.idesc, accum);
-                            if (args.n_a == 2)
-                                umma_bf16(d0 + args.bn, da2 + 2 * k, db + 2 * k, args.idesc, accum);
+                            umma_bf16(d0, da + 2 * k, db + 2 * k, G.idesc, accum);
+                            if (G.n_a == 2) umma_bf16(d0 + G.bn, da2 + 2 * k, db + 2 * k, G.idesc, accum);
                         }
                     }
                     umma_commit(empty_bar(stage));
@@ -348,7 +398,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 }
                 if (!ok) break;
                 umma_commit(tfull_bar(acc));
-                if (args.n_bufs == 2) {
+                if (G.n_bufs == 2) {
                     acc ^= 1;
                     if (acc == 0) acc_phase ^= 1u;
                 } else {
@@ -358,7 +408,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             // all issued MMAs complete before TMEM is released
             umma_commit(drain_bar);
             volatile int never = 0;
-            bar_wait(drain_bar, 0, &never, args.err);
+            bar_wait(drain_bar, 0, &never, err);
         }
     } else {
         // ---------------- epilogue warps 0-3 (thread t <-> TMEM lane t <-> feature t of a tile)
@@ -366,17 +416,22 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const int t = threadIdx.x;
         int acc = 0;
         uint32_t acc_phase = 0;
-        const int acc_cols = args.n_a * args.bn;
-        const int bn = args.bn, na = args.n_a;
-        for (int u = blockIdx.x; u < args.n_units; u += gridDim.x) {
-            const Unit x = decode_unit(args, u);
-            if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, args.err)) break;
+        const int bn = G.bn, na = G.n_a;
+        float* const ws = args.ws;
+        uint32_t* const tile_cnt = args.tile_cnt;
+        const bool resid = args.ep.kind == EPI_RESID && bn == kChunk;
+        for (int u = blockIdx.x; u < G.n_units; u += gridDim.x) {
+            const Unit x = decode_unit(G, u);
+            // the residual rows do not depend on the accumulator: load them before waiting
+            float rr[kChunk];
+            if (resid) load_resid(args.ep, x.n_tile, x.tok_tile * bn, t, rr);
+            if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, err)) break;
             tc_fence_after();
             const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
             bool final_tile = true;
-            if (args.splits > 1) {
+            if (G.splits > 1) {
                 // partial layout per (tile, split): [accumulator][16-token chunk][feature][16]
-                float* dst = args.ws + (size_t)(x.tile_id * args.splits + x.split) * na * bn * 128;
+                float* dst = ws + (size_t)(x.tile_id * G.splits + x.split) * na * bn * 128;
                 for (int a = 0; a < na; ++a)
                     for (int c0 = 0; c0 < bn; c0 += kChunk) {
                         float v[kChunk];
@@ -384,69 +439,72 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                         float4* d4 = reinterpret_cast<float4*>(
                             dst + ((size_t)(a * (bn / kChunk) + c0 / kChunk) * 128 + t) * kChunk);
 #pragma unroll
-                        for (int q = 0; q < kChunk / 4; ++q)
-                            d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                        for (int k = 0; k < kChunk / 4; ++k)
+                            d4[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
                     }
                 tc_fence_before();
                 mbar_arrive(tempty_bar(acc));
-                __threadfence();
+                // the CTA barrier orders every thread's partial before thread 0's release; its
+                // acquire (when last) orders the other partials before the reads below
                 epi_bar();
                 if (t == 0) {
-                    const uint32_t prev = atomicAdd(&args.tile_cnt[x.tile_id], 1u);
-                    misc[2] = (prev == (uint32_t)(args.splits - 1)) ? 1u : 0u;
-                    if (prev == (uint32_t)(args.splits - 1)) args.tile_cnt[x.tile_id] = 0;
+                    const uint32_t prev = atom_add_acq_rel(&tile_cnt[x.tile_id], 1u);
+                    misc[2] = (prev == (uint32_t)(G.splits - 1)) ? 1u : 0u;
+                    if (prev == (uint32_t)(G.splits - 1)) tile_cnt[x.tile_id] = 0;
                 }
                 epi_bar();
                 final_tile = misc[2] != 0;
-                __threadfence();
             }
             if (final_tile) {
                 for (int c0 = 0; c0 < bn; c0 += kChunk) {
                     for (int a = 0; a < na; ++a) {
                         float v[kChunk];
-                        if (args.splits == 1) {
+                        if (G.splits == 1) {
                             tmem_ld16(taddr + (uint32_t)(a * bn + c0), v);
                         } else {
                             // sum the splits in split order (deterministic); four 16-byte loads
                             // per split, several splits in flight
                             float4 acc4[kChunk / 4];
 #pragma unroll
-                            for (int q = 0; q < kChunk / 4; ++q) acc4[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+                            for (int k = 0; k < kChunk / 4; ++k) acc4[k] = make_float4(0.f, 0.f, 0.f, 0.f);
                             const size_t off = ((size_t)(a * (bn / kChunk) + c0 / kChunk) * 128 + t) * kChunk;
 #pragma unroll 4
-                            for (int s = 0; s < args.splits; ++s) {
+                            for (int s = 0; s < G.splits; ++s) {
                                 const float4* src = reinterpret_cast<const float4*>(
-                                    args.ws + (size_t)(x.tile_id * args.splits + s) * na * bn * 128 + off);
+                                    ws + (size_t)(x.tile_id * G.splits + s) * na * bn * 128 + off);
 #pragma unroll
-                                for (int q = 0; q < kChunk / 4; ++q) {
-                                    const float4 w4 = __ldcg(src + q);
-                                    acc4[q].x += w4.x;
-                                    acc4[q].y += w4.y;
-                                    acc4[q].z += w4.z;
-                                    acc4[q].w += w4.w;
+                                for (int k = 0; k < kChunk / 4; ++k) {
+                                    const float4 w4 = __ldcg(src + k);
+                                    acc4[k].x += w4.x;
+                                    acc4[k].y += w4.y;
+                                    acc4[k].z += w4.z;
+                                    acc4[k].w += w4.w;
                                 }
                             }
 #pragma unroll
-                            for (int q = 0; q < kChunk / 4; ++q) {
-                                v[4 * q] = acc4[q].x;
-                                v[4 * q + 1] = acc4[q].y;
-                                v[4 * q + 2] = acc4[q].z;
-                                v[4 * q + 3] = acc4[q].w;
+                            for (int k = 0; k < kChunk / 4; ++k) {
+                                v[4 * k] = acc4[k].x;
+                                v[4 * k + 1] = acc4[k].y;
+                                v[4 * k + 2] = acc4[k].z;
+                                v[4 * k + 3] = acc4[k].w;
                             }
                         }
 #pragma unroll
                         for (int c = 0; c < kChunk; ++c) epi[(a * kChunk + c) * 128 + t] = v[c];
                     }
                     epi_bar();
-                    apply_epilogue<bf16>(args.ep, epi, x.group, x.n_tile, x.tok_tile * bn + c0, t);
+                    if (resid)
+                        resid_epilogue(args.ep, epi, x.n_tile, x.tok_tile * bn + c0, t, rr);
+                    else
+                        apply_epilogue<bf16>(args.ep, epi, x.group, x.n_tile, x.tok_tile * bn + c0, t);
                     epi_bar();
                 }
             }
-            if (args.splits == 1) {
+            if (G.splits == 1) {
                 tc_fence_before();
                 mbar_arrive(tempty_bar(acc));
             }
-            if (args.n_bufs == 2) {
+            if (G.n_bufs == 2) {
                 acc ^= 1;
                 if (acc == 0) acc_phase ^= 1u;
             } else {
@@ -497,7 +555,8 @@ bool make_map(CUtensorMap* m, const void* base, int k, int rows, int groups, lon
 
 cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why) {
     if (g.m_tok <= 0 || g.n <= 0) return cudaSuccess;
-    TcArgs a{};
+    TcArgs a;
+    memset(&a, 0, sizeof(a));
     a.n_a = g.a2 ? 2 : 1;
     a.bn = g.m_tok <= 256 ? ((g.m_tok + 15) / 16) * 16 : 256;
     a.tok_tiles = (g.m_tok + a.bn - 1) / a.bn;
@@ -534,14 +593,17 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         while (a.kbs > 1 && 2 * a.kbs * (kBM * kBK * 2 * a.n_a + a.bn * kBK * 2) > budget - fixed)
             a.kbs >>= 1;
     }
+    if (g.force_splits > 0) best = std::min(g.force_splits, a.k_blocks);
     a.kb_per_split = (a.k_blocks + best - 1) / best;
     a.kb_per_split = (a.kb_per_split + a.kbs - 1) / a.kbs * a.kbs;
     a.splits = (a.k_blocks + a.kb_per_split - 1) / a.kb_per_split;
+    if (a.splits > 1 && ((size_t)tiles * a.splits * a.n_a * a.bn * 128 > c->ws_floats || tiles > c->tile_cnt_n)) {
+        if (why) *why = "tcgen05 GEMM: split-K workspace too small";
+        return cudaErrorInvalidValue;
+    }
     a.n_units = tiles * a.splits;
-    const uint32_t a_bytes = kBM * kBK * 2;
     a.b_bytes = (uint32_t)a.bn * kBK * 2;
-    a.stage_bytes = (uint32_t)a.kbs * (a_bytes * a.n_a + a.b_bytes);
-    a.tx_bytes = a.stage_bytes;
+    a.stage_bytes = (uint32_t)a.kbs * (kABytes * a.n_a + a.b_bytes);
     a.evict_first = g.evict_first >= 0 ? 1 : 0;
     a.stages = std::min(kMaxStages, (budget - fixed) / (int)a.stage_bytes);
     if (a.stages < 2) {
@@ -561,11 +623,9 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     a.tile_cnt = c->tile_cnt;
     a.err = c->err;
     a.ep = g.ep;
-
-    CUtensorMap ma, ma2, mb;
-    if (!make_map(&ma, g.a, g.k, g.n, g.groups, g.n, kBM) ||
-        !make_map(&ma2, g.a2 ? g.a2 : g.a, g.k, g.n, g.groups, g.n, kBM) ||
-        !make_map(&mb, g.b, g.k, g.m_tok, g.groups, g.b_group_rows, a.bn)) {
+    if (!make_map(&a.map_a, g.a, g.k, g.n, g.groups, g.n, kBM) ||
+        !make_map(&a.map_a2, g.a2 ? g.a2 : g.a, g.k, g.n, g.groups, g.n, kBM) ||
+        !make_map(&a.map_b, g.b, g.k, g.m_tok, g.groups, g.b_group_rows, a.bn)) {
         if (why) *why = "cuTensorMapEncodeTiled failed (alignment or driver entry point)";
         return cudaErrorInvalidValue;
     }
@@ -577,7 +637,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         configured = 1;
     }
     const int grid = std::min(a.n_units, sms);
-    return launch_kernel(c->pdl, gemm_tc_kernel, dim3(grid), dim3(kThreads), smem, s, ma, ma2, mb, a);
+    return launch_kernel(c->pdl, gemm_tc_kernel, dim3(grid), dim3(kThreads), smem, s, a);
 }
 
 }  // namespace dfl

@@ -61,6 +61,7 @@ struct GemmDesc {
     int kbs = 0;           // tcgen05 GEMM: 64-wide k-blocks per pipeline stage (0 = default)
     int max_smem = 0;      // tcgen05 GEMM: shared-memory budget per CTA in bytes (0 = default)
     int evict_first = 0;   // tcgen05 GEMM: weights with an L2 evict-first policy (0 = yes, -1 = no)
+    int force_splits = 0;  // tcgen05 GEMM: K splits (0 = chosen from the wave count)
 };
 
 }  // namespace dfl
