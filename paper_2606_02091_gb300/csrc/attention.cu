@@ -42,6 +42,8 @@ struct AttnArgs {
     const int32_t* ctx_len;
     float* part_o;        // [batch][H_kv][q_tiles][splits][64][hd]
     float* part_ml;       // [batch][H_kv][q_tiles][splits][64][2]
+    uint32_t* err;        // device error word (a tile wait that timed out)
+    int block_rows;       // rows of one K^d / V^d tensor-map box (min(64, max_batch * B))
     int B, G, hkv, d_q, d_kv, max_ctx, splits, q_tiles;
     float scale_log2;     // log2(e) / sqrt(hd)
 };
@@ -115,46 +117,128 @@ __device__ __forceinline__ void bf16x8_to_f16x8(void* p) {
     *reinterpret_cast<uint4*>(p) = o;
 }
 
-constexpr int kNST = 2;    // K/V tiles in flight per CTA (two CTAs fit on an SM)
+constexpr int kNST = 2;                   // K/V tiles in flight per CTA (two CTAs fit on an SM)
+constexpr uint64_t kWaitNs = 2000000000ull;  // bound on every wait for a tile
+
+// Tensor maps of one layer (bf16, 128-byte swizzle, boxes of 64 keys x 64 head dims):
+// K and V cache [max_batch * H_kv][max_ctx][hd] and the block's K^d, V^d [H_kv][max_batch * B][hd]
+// (row stride d_kv).
+struct AttnMaps {
+    CUtensorMap kc, vc, kd, vd;
+};
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+// Byte offset of the 16-byte chunk c8 (head dims 8*c8 .. 8*c8+7) of key row r in a tile stored as
+// [hd/64 halves][64 rows][128 bytes] with the 128-byte swizzle (chunk index XOR row % 8).
+__device__ __forceinline__ uint32_t swz(int r, int c8) {
+    return (uint32_t)((c8 >> 3) * 8192 + r * 128 + (((c8 & 7) ^ (r & 7)) << 4));
+}
+__device__ __forceinline__ bool tile_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok = 0;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (ok) return true;
+        if (globaltimer_ns() - t0 > kWaitNs) return false;
+    }
+}
+__device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* m, int x, int y, int z,
+                                         uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
 
 // One CTA per (key split, KV head, 64-row query tile, sequence); the `splits` CTAs of one
-// (sequence, head, query tile) form a thread-block cluster. Each CTA runs online softmax over its
-// key range, leaves its unnormalised partial (O, running max, running sum) in its own shared
-// memory, and after a cluster barrier every CTA merges a slice of the 64 rows from all peers'
-// shared memory (DSMEM) and writes the bf16 result. No partials go through global memory.
+// (sequence, head, query tile) form a thread-block cluster. The keys are cut into tiles of 64:
+// ceil(L / 64) context tiles, then one tile of the block's own B keys (K^d, V^d); the splits take
+// contiguous runs of tiles whose counts differ by at most one. One thread streams the tiles with TMA into a ring of kNST swizzled stages;
+// every thread waits on the stage's mbarrier. Each CTA runs online softmax over its keys and
+// pushes its partial (O / l in fp16, running max, running sum) row by row into the shared memory
+// of the CTA that merges that row (DSMEM stores); after one cluster barrier every CTA merges its
+// slice of the 64 rows from its own shared memory and writes the bf16 result. No partials go
+// through global memory.
 template <int HD, int S>
-__global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* __restrict__ out) {
+__global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ AttnMaps maps,
+                                                       const AttnArgs a, bf16* __restrict__ out) {
     pdl_trigger();
-    pdl_wait();
-    constexpr int LD = HD + 8;                 // padded smem row (elements)
+    constexpr int LD = HD + 8;                 // padded Q row (elements)
     constexpr int PIECES = HD / 8;             // 16-byte pieces per row
-    extern __shared__ __align__(16) uint8_t smem[];
-    bf16* Qs = reinterpret_cast<bf16*>(smem);
-    bf16* Ks = Qs + kQT * LD;                  // [kNST][kKT][LD]
-    bf16* Vs = Ks + kNST * kKT * LD;           // [kNST][kKT][LD]
-    float* sO = reinterpret_cast<float*>(smem);  // after the key loop: [kQT][HD] partial output
-    float* sML = sO + kQT * HD;                  // [kQT][2] running max (log2 units), sum
+    constexpr uint32_t TB = HD * 128;          // bytes of one 64-key K (or V) tile
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    bf16* Qs = reinterpret_cast<bf16*>(smem + kNST * 2 * TB);   // [kQT][LD]
+    // partials pushed here by the cluster's CTAs: row lr of this CTA's slice from split p at
+    // [p * RP + lr], O / l in fp16 and (running max in log2 units, running sum)
+    __half* rO = reinterpret_cast<__half*>(Qs + kQT * LD);     // [kQT][HD]
+    float* rML = reinterpret_cast<float*>(rO + kQT * HD);        // [kQT][2]
+    uint64_t* full = reinterpret_cast<uint64_t*>(rML + 2 * kQT);
+    constexpr int RP = kQT / S;                                  // merged rows per CTA
     cg::cluster_group cluster = cg::this_cluster();
     const int s = (int)cluster.block_rank();
     const int g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = a.B * a.G;
-    int j_begin, j_end, L;
-    key_range(a, b, s, j_begin, j_end, L);
+    const uint32_t sbase = smem_addr(smem), fbar = smem_addr(full);
+    if (tid == 0) {
+        for (int i = 0; i < kNST; ++i)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(fbar + 8u * i) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.kc)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.vc)) : "memory");
+    }
+    __syncthreads();
+    // every CTA of the cluster has started before any pushes into another's shared memory (the
+    // matching wait comes after the key loop)
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    pdl_wait();
+    const int L = a.ctx_len[b];
+    // the sequence's tiles: ceil(L / 64) context tiles, then the block tile; split s takes a
+    // contiguous run of them (the counts differ by at most one)
+    const int n_ctx_tiles = (L + kKT - 1) / kKT, T = n_ctx_tiles + 1;
+    const int t0 = s * (T / S) + min(s, T % S);
+    const int n_tiles = T / S + (s < T % S ? 1 : 0);
+    const int n_ct = max(0, min(t0 + n_tiles, n_ctx_tiles) - t0);   // context tiles of this CTA
+    // tile t -> stage t % kNST: K at [stage][0, TB), V at [stage][TB, 2 TB)
+    auto issue = [&](int t) {
+        const int st = t % kNST;
+        const uint32_t kdst = sbase + (uint32_t)st * 2 * TB, bar = fbar + 8u * st;
+        const uint32_t bytes = t < n_ct ? 2 * TB : 2u * (HD / 64) * (uint32_t)a.block_rows * 128u;
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                     : "memory");
+        for (int h = 0; h < HD / 64; ++h) {
+            if (t < n_ct) {
+                const int y = (t0 + t) * kKT, z = b * a.hkv + g;
+                tma_tile(kdst + h * 8192, &maps.kc, h * 64, y, z, bar);
+                tma_tile(kdst + TB + h * 8192, &maps.vc, h * 64, y, z, bar);
+            } else {
+                tma_tile(kdst + h * 8192, &maps.kd, h * 64, b * a.B, g, bar);
+                tma_tile(kdst + TB + h * 8192, &maps.vd, h * 64, b * a.B, g, bar);
+            }
+        }
+    };
+    int issued = 0, consumed = 0;
+    if (tid == 0)
+        for (; issued < min(kNST - 1, n_tiles); ++issued) issue(issued);
 
     float o[HD / 8][4];
 #pragma unroll
     for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    if (j_begin < j_end) {
+    bool timed_out = false;
+    if (n_tiles > 0) {
         const bf16* q = static_cast<const bf16*>(a.q);
-        const bf16* kd = static_cast<const bf16*>(a.kd);
-        const bf16* vd = static_cast<const bf16*>(a.vd);
-        const bf16* kc = static_cast<const bf16*>(a.kc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
-        const bf16* vc = static_cast<const bf16*>(a.vc) + ((size_t)b * a.hkv + g) * a.max_ctx * HD;
-        const uint32_t sQ = (uint32_t)__cvta_generic_to_shared(Qs);
-        const uint32_t sK = (uint32_t)__cvta_generic_to_shared(Ks);
-        const uint32_t sV = (uint32_t)__cvta_generic_to_shared(Vs);
+        const uint32_t sQ = smem_addr(Qs);
         // query rows of this tile: row r -> block position r / G, head g*G + r % G
         for (int idx = tid; idx < kQT * PIECES; idx += blockDim.x) {
             const int r = idx / PIECES, pc = idx % PIECES;
@@ -164,51 +248,40 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
             const bf16* src = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + pc * 8;
             cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
         }
-        // keys j < L come from the cache, j >= L from the block's own K^d / V^d
-        auto load_tile = [&](int j0, int buf) {
-            for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
-                const int r = idx / PIECES, pc = idx % PIECES;
-                const int j = j0 + r;
-                const bool ok = j < j_end;
-                const bf16 *ksrc, *vsrc;
-                if (j < L) {
-                    ksrc = kc + (size_t)j * HD + pc * 8;
-                    vsrc = vc + (size_t)j * HD + pc * 8;
-                } else {
-                    const int k = ok ? j - L : 0;
-                    ksrc = kd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
-                    vsrc = vd + ((size_t)b * a.B + k) * a.d_kv + (size_t)g * HD + pc * 8;
-                }
-                const uint32_t off = (uint32_t)((buf * kKT + r) * LD + pc * 8) * 2;
-                cp_async16(sK + off, ok ? (const void*)ksrc : (const void*)kc, ok);
-                cp_async16(sV + off, ok ? (const void*)vsrc : (const void*)vc, ok);
-            }
-        };
-        const int n_tiles = (j_end - j_begin + kKT - 1) / kKT;
-        for (int p = 0; p < kNST - 1; ++p) {
-            if (p < n_tiles) load_tile(j_begin + p * kKT, p);
-            cp_commit();
-        }
+        cp_commit();
         uint32_t qa[HD / 16][4];
         for (int t = 0; t < n_tiles; ++t) {
-            const int buf = t % kNST;
-            if (t + kNST - 1 < n_tiles) load_tile(j_begin + (t + kNST - 1) * kKT, (t + kNST - 1) % kNST);
-            cp_commit();
-            cp_wait<kNST - 1>();
-            // this thread's copies of tile t have landed: convert its V pieces to fp16
-            for (int idx = tid; idx < kKT * PIECES; idx += blockDim.x) {
-                const int r = idx / PIECES, pc = idx % PIECES;
-                bf16x8_to_f16x8(Vs + (buf * kKT + r) * LD + pc * 8);
+            const int st = t % kNST;
+            if (tid == 0 && issued < n_tiles) issue(issued++);   // the stage freed at the end of t-1
+            const bool landed = tile_wait(fbar + 8u * st, (uint32_t)(t / kNST) & 1u);
+            if (__syncthreads_or(!landed)) {   // one decision for the whole CTA
+                timed_out = true;
+                break;
             }
+            ++consumed;
+            const int valid = t < n_ct ? min(kKT, L - (t0 + t) * kKT) : a.B;
+            // V to fp16 in place; rows past the tile's valid keys become zeros (their P is 0)
+            uint8_t* vt = smem + (size_t)st * 2 * TB + TB;
+            for (int k = tid; k < (int)(TB / 16); k += blockDim.x) {
+                const int r = (k & 511) >> 3;
+                if (r < valid) {
+                    bf16x8_to_f16x8(vt + (size_t)k * 16);
+                } else {
+                    *reinterpret_cast<uint4*>(vt + (size_t)k * 16) = make_uint4(0u, 0u, 0u, 0u);
+                }
+            }
+            // these generic-proxy writes come before the TMA that refills the stage later
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            if (t == 0) cp_wait<0>();
             __syncthreads();
             if (t == 0) {
 #pragma unroll
                 for (int kk = 0; kk < HD / 16; ++kk) {
                     const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
-                    ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2],
-                            qa[kk][3]);
+                    ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
                 }
             }
+            const uint32_t sK = sbase + (uint32_t)st * 2 * TB, sV = sK + TB;
             // S = Q K^T for 16 rows x 64 keys
             // (k outer, keys inner: eight independent accumulators between dependent MMAs)
             float sc[8][4];
@@ -219,22 +292,20 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
 #pragma unroll
                 for (int nt = 0; nt < 8; ++nt) {
                     const int row = nt * 8 + (lane & 7);
-                    const int col = kk * 16 + (lane >> 3) * 8;
+                    const int c8 = kk * 2 + (lane >> 3);
                     uint32_t b0, b1, b2, b3;
-                    ldsm_x4(sK + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
+                    ldsm_x4(sK + swz(row, c8), b0, b1, b2, b3);
                     mma16816(sc[nt], qa[kk], b0, b1);
                     mma16816(sc[nt], qa[kk + 1], b2, b3);
                 }
             }
-            // mask keys past the range, scale into the log2 domain, online softmax
-            const int jt = j_begin + t * kKT;
+            // mask keys past the tile's valid ones, scale into the log2 domain, online softmax
             float mx0 = m0, mx1 = m1;
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
-                    const int j = jt + nt * 8 + (lane & 3) * 2 + e;
-                    const bool ok = j < j_end;
+                    const bool ok = nt * 8 + (lane & 3) * 2 + e < valid;
                     sc[nt][e] = ok ? sc[nt][e] * a.scale_log2 : -INFINITY;
                     sc[nt][2 + e] = ok ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
                     mx0 = fmaxf(mx0, sc[nt][e]);
@@ -246,14 +317,14 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
                 mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
                 mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
             }
-            const float c0 = exp2f(m0 - mx0), c1 = exp2f(m1 - mx1);
+            const float cr0 = exp2f(m0 - mx0), cr1 = exp2f(m1 - mx1);
             m0 = mx0;
             m1 = mx1;
-            l0 *= c0;
-            l1 *= c1;
+            l0 *= cr0;
+            l1 *= cr1;
 #pragma unroll
             for (int i = 0; i < HD / 8; ++i) {
-                o[i][0] *= c0; o[i][1] *= c0; o[i][2] *= c1; o[i][3] *= c1;
+                o[i][0] *= cr0; o[i][1] *= cr0; o[i][2] *= cr1; o[i][3] *= cr1;
             }
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
@@ -275,9 +346,9 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
 #pragma unroll
                 for (int nt = 0; nt < HD / 8; nt += 2) {
                     const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-                    const int col = (nt + (lane >> 4)) * 8;
+                    const int c8 = nt + (lane >> 4);
                     uint32_t b0, b1, b2, b3;
-                    ldsm_x4_t(sV + (uint32_t)((buf * kKT + row) * LD + col) * 2, b0, b1, b2, b3);
+                    ldsm_x4_t(sV + swz(row, c8), b0, b1, b2, b3);
                     mma16816_f16(o[nt], pa, b0, b1);
                     mma16816_f16(o[nt + 1], pa, b2, b3);
                 }
@@ -291,60 +362,74 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a, bf16* _
             l1 += __shfl_xor_sync(0xffffffffu, l1, off);
         }
     }
-    __syncthreads();   // the tiles' shared memory now holds this CTA's partial result
+    if (timed_out) {
+        if (tid == 0) atomicOr(a.err, DFLARE_DEVERR_TIMEOUT);
+        // copies still in flight land before this shared memory is reused or released
+        if (tid == 0)
+            for (int t = consumed; t < issued; ++t) tile_wait(fbar + 8u * (t % kNST), (uint32_t)(t / kNST) & 1u);
+    }
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+    // push the partial: query row r belongs to the merge slice of CTA r / RP, which keeps it at
+    // [s * RP + r % RP]; O is normalised by l first (|O / l| <= max |V|, safe in fp16). The rows
+    // are staged in this CTA's (now idle) tile memory so that the remote stores are 16 bytes wide.
     {
+        __half* stg = reinterpret_cast<__half*>(smem);   // [kQT][HD]
         const int r0 = warp * 16 + (lane >> 2), r1 = r0 + 8;
+        const float i0 = l0 > 0.f ? 1.0f / l0 : 0.f, i1 = l1 > 0.f ? 1.0f / l1 : 0.f;
 #pragma unroll
         for (int nt = 0; nt < HD / 8; ++nt) {
             const int col = nt * 8 + (lane & 3) * 2;
-            *reinterpret_cast<float2*>(sO + r0 * HD + col) = make_float2(o[nt][0], o[nt][1]);
-            *reinterpret_cast<float2*>(sO + r1 * HD + col) = make_float2(o[nt][2], o[nt][3]);
+            *reinterpret_cast<__half2*>(stg + r0 * HD + col) = __floats2half2_rn(o[nt][0] * i0, o[nt][1] * i0);
+            *reinterpret_cast<__half2*>(stg + r1 * HD + col) = __floats2half2_rn(o[nt][2] * i1, o[nt][3] * i1);
         }
         if ((lane & 3) == 0) {
-            sML[2 * r0] = m0;
-            sML[2 * r0 + 1] = l0;
-            sML[2 * r1] = m1;
-            sML[2 * r1 + 1] = l1;
+            *reinterpret_cast<float2*>(cluster.map_shared_rank(rML, r0 / RP) + 2 * (s * RP + r0 % RP)) =
+                make_float2(m0, l0);
+            *reinterpret_cast<float2*>(cluster.map_shared_rank(rML, r1 / RP) + 2 * (s * RP + r1 % RP)) =
+                make_float2(m1, l1);
+        }
+        __syncthreads();
+        for (int k = tid; k < kQT * PIECES; k += blockDim.x) {
+            const int r = k / PIECES, pc = k % PIECES;
+            *reinterpret_cast<uint4*>(cluster.map_shared_rank(rO, r / RP) + (size_t)(s * RP + r % RP) * HD + pc * 8) =
+                *reinterpret_cast<const uint4*>(stg + r * HD + pc * 8);
         }
     }
+    // every partial has arrived; after this barrier no CTA touches another's shared memory
     cluster.sync();
-    // merge: CTA s owns rows [s * RP, (s + 1) * RP) of the 64, TPR threads per row, EPT output
-    // elements per thread; every peer value is loaded before anything is stored
-    constexpr int RP = kQT / S, TPR = 128 / RP, EPT = HD / TPR;
-    const int rr = s * RP + tid / TPR, lt = tid % TPR;
-    const int rg = qt * kQT + rr;
+    // merge: TPR threads per row of this CTA's slice, EPT contiguous output elements per thread,
+    // out = sum_p w_p (O_p / l_p) / sum_p w_p with w_p = l_p 2^(m_p - max m)
+    constexpr int TPR = 128 / RP, EPT = HD / TPR;
+    static_assert(EPT % 2 == 0, "merge slice must be a whole number of half2");
+    const int lr = tid / TPR, lt = tid % TPR;
+    const int rg = qt * kQT + s * RP + lr;
     if (rg < R) {
-        float mv[S], lv[S], vals[S][EPT];
-#pragma unroll
-        for (int p = 0; p < S; ++p) {
-            const float* ml = cluster.map_shared_rank(sML, p);
-            const float* op = cluster.map_shared_rank(sO, p) + rr * HD;
-            mv[p] = ml[2 * rr];
-            lv[p] = ml[2 * rr + 1];
-#pragma unroll
-            for (int q = 0; q < EPT; ++q) vals[p][q] = op[lt + q * TPR];
-        }
+        float w[S];
         float M = -INFINITY;
 #pragma unroll
-        for (int p = 0; p < S; ++p) M = fmaxf(M, mv[p]);
+        for (int p = 0; p < S; ++p) M = fmaxf(M, rML[2 * (p * RP + lr)]);
         float den = 0.f;
 #pragma unroll
         for (int p = 0; p < S; ++p) {
-            mv[p] = (mv[p] == -INFINITY) ? 0.f : exp2f(mv[p] - M);
-            den = fmaf(mv[p], lv[p], den);
+            const float mp = rML[2 * (p * RP + lr)], lp = rML[2 * (p * RP + lr) + 1];
+            w[p] = mp == -INFINITY ? 0.f : lp * exp2f(mp - M);
+            den += w[p];
         }
         const float inv = 1.0f / den;
         const int kpos = rg / a.G, hh = rg % a.G;
-        bf16* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD;
+        bf16* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + lt * EPT;
 #pragma unroll
-        for (int q = 0; q < EPT; ++q) {
-            float v = 0.f;
+        for (int q = 0; q < EPT; q += 2) {
+            float v0 = 0.f, v1 = 0.f;
 #pragma unroll
-            for (int p = 0; p < S; ++p) v = fmaf(mv[p], vals[p][q], v);
-            orow[lt + q * TPR] = __float2bfloat16_rn(v * inv);
+            for (int p = 0; p < S; ++p) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(rO + (size_t)(p * RP + lr) * HD + lt * EPT + q));
+                v0 = fmaf(w[p], f.x, v0);
+                v1 = fmaf(w[p], f.y, v1);
+            }
+            *reinterpret_cast<__nv_bfloat162*>(orow + q) = __floats2bfloat162_rn(v0 * inv, v1 * inv);
         }
     }
-    cluster.sync();    // peers may still be reading this CTA's shared memory
 }
 
 // ------------------------------------------------------------------ CUDA-core path
@@ -438,12 +523,13 @@ __global__ void attn_combine_kernel(const AttnArgs a, T* __restrict__ out) {
 }
 
 template <int HD>
-size_t mma_smem_bytes() {
-    return (size_t)(kQT + 2 * kNST * kKT) * (HD + 8) * sizeof(bf16);
+size_t mma_smem_bytes() {   // alignment pad, K/V stages, padded Q tile, pushed partials, barriers
+    return 1024 + (size_t)kNST * 2 * HD * 128 + (size_t)kQT * (HD + 8) * sizeof(bf16) +
+           (size_t)kQT * HD * sizeof(__half) + (size_t)kQT * 2 * sizeof(float) + 8 * kNST;
 }
 
 template <int HD, int S>
-cudaError_t launch_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
+cudaError_t launch_mma(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
     static bool configured = false;
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
@@ -456,17 +542,17 @@ cudaError_t launch_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
         configured = true;
     }
     return launch_cluster(c->pdl, S, attn_mma_kernel<HD, S>, dim3(S, a.hkv * a.q_tiles, c->batch),
-                          dim3(128), mma_smem_bytes<HD>(), s, a, static_cast<bf16*>(c->attn));
+                          dim3(128), mma_smem_bytes<HD>(), s, maps, a, static_cast<bf16*>(c->attn));
 }
 
 template <int HD>
-cudaError_t run_mma(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
+cudaError_t run_mma(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
     switch (a.splits) {
-        case 1: return launch_mma<HD, 1>(c, a, s);
-        case 2: return launch_mma<HD, 2>(c, a, s);
-        case 4: return launch_mma<HD, 4>(c, a, s);
-        case 8: return launch_mma<HD, 8>(c, a, s);
-        default: return launch_mma<HD, 16>(c, a, s);
+        case 1: return launch_mma<HD, 1>(c, maps, a, s);
+        case 2: return launch_mma<HD, 2>(c, maps, a, s);
+        case 4: return launch_mma<HD, 4>(c, maps, a, s);
+        case 8: return launch_mma<HD, 8>(c, maps, a, s);
+        default: return launch_mma<HD, 16>(c, maps, a, s);
     }
 }
 
@@ -540,7 +626,7 @@ int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int
 
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
     const dflare_config& g = c->cfg;
-    AttnArgs a;
+    AttnArgs a{};
     a.q = c->q;
     a.kd = c->kd;
     a.vd = c->vd;
@@ -562,9 +648,37 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
         a.splits = attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
         return g.head_dim == 64 ? run_simt<float, 64>(c, a, s) : run_simt<float, 128>(c, a, s);
     }
+    a.err = c->err;
+    // tensor maps of every layer's K/V cache and of K^d / V^d, built once per context
+    if (c->attn_maps.empty()) {
+        std::vector<CUtensorMap> m((size_t)2 * g.n_draft_layers + 2);
+        const uint64_t hd = (uint64_t)g.head_dim;
+        const uint32_t box[3] = {64u, (uint32_t)kKT, 1u};
+        const uint32_t bbox[3] = {64u, (uint32_t)std::min(kKT, g.max_batch * g.block), 1u};
+        for (int i = 0; i < g.n_draft_layers; ++i)
+            for (int kv = 0; kv < 2; ++kv) {
+                const uint8_t* base = static_cast<const uint8_t*>(kv ? c->vcache : c->kcache) + i * layer_elems * c->esz;
+                const uint64_t dims[3] = {hd, (uint64_t)g.max_ctx, (uint64_t)g.max_batch * g.n_kv_heads};
+                const uint64_t strides[2] = {hd * 2, (uint64_t)g.max_ctx * hd * 2};
+                if (!encode_tma_bf16(&m[2 * i + kv], base, 3, dims, strides, box)) return cudaErrorInvalidValue;
+            }
+        for (int kv = 0; kv < 2; ++kv) {
+            const uint64_t dims[3] = {hd, (uint64_t)g.max_batch * g.block, (uint64_t)g.n_kv_heads};
+            const uint64_t strides[2] = {(uint64_t)a.d_kv * 2, hd * 2};
+            if (!encode_tma_bf16(&m[2 * g.n_draft_layers + kv], kv ? c->vd : c->kd, 3, dims, strides, bbox))
+                return cudaErrorInvalidValue;
+        }
+        c->attn_maps.swap(m);
+    }
+    AttnMaps maps;
+    maps.kc = c->attn_maps[2 * layer];
+    maps.vc = c->attn_maps[2 * layer + 1];
+    maps.kd = c->attn_maps[2 * g.n_draft_layers];
+    maps.vd = c->attn_maps[2 * g.n_draft_layers + 1];
+    a.block_rows = std::min(kKT, g.max_batch * g.block);
     const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
     a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc);
-    return g.head_dim == 64 ? run_mma<64>(c, a, s) : run_mma<128>(c, a, s);
+    return g.head_dim == 64 ? run_mma<64>(c, maps, a, s) : run_mma<128>(c, maps, a, s);
 }
 
 }  // namespace dfl

@@ -5,6 +5,7 @@
 #include <stdint.h>
 
 #include <string>
+#include <vector>
 
 #include "dflare.h"
 
@@ -96,6 +97,8 @@ struct dflare_ctx {
     float* attn_o = nullptr;       // split-KV partial outputs
     float* attn_ml = nullptr;      // split-KV partial (max, sum)
     int attn_splits = 1;
+    // tensor maps of the bf16 attention: per layer K and V cache, then K^d and V^d (built on first use)
+    std::vector<CUtensorMap> attn_maps;
     float* ws = nullptr;           // split-K workspace
     size_t ws_floats = 0;
     uint32_t* tile_cnt = nullptr;  // split-K arrival counters
@@ -157,6 +160,10 @@ void noalloc_set_error(const std::string& message);
 
 // launchers (each returns the first CUDA error it meets)
 cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why);
+// bf16 tensor map with a 128-byte swizzle and zero fill outside the tensor (dims innermost first;
+// strides_bytes for dims 1..rank-1); false when the driver rejects it.
+bool encode_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                     const uint64_t* strides_bytes, const uint32_t* box);
 cudaError_t launch_gemm_simt(dflare_ctx* c, const GemmDesc& g, cudaStream_t s);
 cudaError_t launch_fusion_alpha(dflare_ctx* c, cudaStream_t s);
 cudaError_t launch_fuse_begin(dflare_ctx* c, const int32_t* n_new, int n_max, cudaStream_t s);
