@@ -218,9 +218,10 @@ class Cudart:
         assert self.lib.cudaEventCreate(ctypes.byref(e)) == 0
         return e
 
-    def record(self, e, stream):
-        # cudaEventRecordExternal: inside stream capture this becomes an event-record node
-        assert self.lib.cudaEventRecordWithFlags(e, stream, 1) == 0
+    def record(self, e, stream, captured=True):
+        # cudaEventRecordExternal: inside stream capture this becomes an event-record node; an
+        # eager launch takes the default flags
+        assert self.lib.cudaEventRecordWithFlags(e, stream, 1 if captured else 0) == 0
 
     def elapsed(self, a, b):
         ms = ctypes.c_float()
@@ -282,6 +283,20 @@ def gemm_traffic(w):
     return d.get("dram_bytes_per_step")
 
 
+def replica_aggregate(ms, units_per_step, steps, dist=None, device="cuda"):
+    """Weak-scaling aggregate of independent replicas (one per rank, no data-path exchange):
+    the job's time is the slowest rank's, its throughput every rank's units over that time.
+    Returns (max ms over ranks, units per second of the whole job)."""
+    world = 1
+    if dist is not None and dist.is_initialized():
+        import torch
+        t = torch.tensor([float(ms)], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        world = dist.get_world_size()
+    return ms, world * units_per_step * steps / (ms / 1e3)
+
+
 def run_ours(args):
     import torch
     import paper_2606_02091_gb300 as P
@@ -313,8 +328,11 @@ def run_ours(args):
                             flags=P.FLAG_SERIAL_LAUNCH if args.serial_launch else 0)
     lib.set_weights(dev_w)
     lib.reset(w.batch)
-    # context fill in chunks (the target's prompt states)
+    # context fill in chunks (the target's prompt states): once untimed, then again from an empty
+    # context with CUDA events around the fusion and context-projection launches (Sec. 8 K1/K2
+    # are measured at fill, where n = L positions per call)
     dt_np = np.uint16 if s.dtype == "bf16" else np.float32
+    fill_chunks = []
     for pos0 in range(0, max(w.ctx_lens), chunk):
         ns = [max(0, min(chunk, L - pos0)) for L in w.ctx_lens]
         H = np.zeros((s.n_target_layers, w.batch, chunk, s.d), dt_np)
@@ -322,10 +340,38 @@ def run_ours(args):
             if n:
                 H[:, b, :n] = synth.hidden_states(w, b, pos0, n)
         Ht = torch.from_numpy(H)
-        Ht = (Ht.view(torch.bfloat16) if dt_np == np.uint16 else Ht).cuda()
-        lib.fuse_context(Ht, torch.tensor(ns, dtype=torch.int32, device="cuda"))
-        del Ht
-    torch.cuda.synchronize()
+        fill_chunks.append(((Ht.view(torch.bfloat16) if dt_np == np.uint16 else Ht).cuda(),
+                            torch.tensor(ns, dtype=torch.int32, device="cuda")))
+    fill_ev = []
+    crf = Cudart()
+
+    @P._lib.TRACE_FN
+    def fill_cb(user, name, phase, stream):
+        e = crf.event()
+        crf.record(e, stream, captured=False)
+        fill_ev.append((name.decode(), phase, e))
+
+    for timed in (False, True):
+        lib.reset(w.batch)
+        if timed:
+            P.load().dflare_set_trace(lib.raw, fill_cb, None)
+        for Ht, nt in fill_chunks:
+            lib.fuse_context(Ht, nt)
+        if timed:
+            P.load().dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
+        torch.cuda.synchronize()
+    del fill_chunks
+    fill_us = {}
+    open_f = {}
+    for name, phase, e in fill_ev:
+        if phase == 0:
+            open_f[name] = e
+        else:
+            fill_us[name] = fill_us.get(name, 0.0) + 1e3 * crf.elapsed(open_f.pop(name), e)
+    n_fill = sum(w.ctx_lens)
+    e_sz = 2 if s.dtype == "bf16" else 4
+    fuse_bytes = n_fill * (s.n_target_layers + s.n_draft_layers) * s.d * e_sz
+    kv_flops = 2.0 * n_fill * s.n_draft_layers * 2 * s.d_kv * s.d
     # per-step buffers: target states of up to B newly committed positions, draws of the
     # synthetic target for n_tab steps, and the loop state (accept_len doubles as next n_new)
     Hs = np.zeros((s.n_target_layers, w.batch, s.block, s.d), dt_np)
@@ -406,12 +452,8 @@ def run_ours(args):
     lens1 = lib.ctx_lens()
     # each step fuses the previous step's tau: the context grows by the accepted positions
     mean_tau = (sum(lens1) - sum(lens0)) / (K * w.batch)
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
     drafted_per_step = w.batch * (s.block - 1)
-    value = world * drafted_per_step * K / (ms / 1e3)
+    ms, value = replica_aggregate(ms, drafted_per_step, K, dist)
 
     # ---------------- per-kernel durations (CUDA events around every launch, graph replays)
     cr = Cudart()
@@ -533,6 +575,17 @@ def run_ours(args):
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "ms_per_step": 1e3 * max(e2e_ms / 1e3, wall) / E,
                 "steps": E, "timing": "eager public calls, pinned-host copies in the region"},
+        "fill": {"positions": n_fill, "calls": len(range(0, max(w.ctx_lens), chunk)),
+                 "fuse_layers_us": fill_us.get("fuse_layers"),
+                 "fuse_layers_gbs": fuse_bytes / (fill_us["fuse_layers"] * 1e-6) / 1e9
+                 if fill_us.get("fuse_layers") else None,
+                 "fuse_layers_frac_of_hbm": fuse_bytes / (fill_us["fuse_layers"] * 1e-6) / 1e9 / hbm
+                 if fill_us.get("fuse_layers") else None,
+                 "kv_ctx_us": fill_us.get("gemm_kv_ctx"),
+                 "kv_ctx_tflops": kv_flops / (fill_us["gemm_kv_ctx"] * 1e-6) / 1e12
+                 if fill_us.get("gemm_kv_ctx") else None,
+                 "note": "context fill of every sequence from empty, CUDA events around each launch "
+                         "(fusion: (T + D) d bytes per position; K/V projection: 2 n D 2 d_kv d flop)"},
         "gpu_launches": int(round(launches_per_step * K)),
         "launches_per_step": launches_per_step,
         "clocks": clk,

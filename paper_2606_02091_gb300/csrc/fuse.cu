@@ -2,9 +2,13 @@
 //
 // fusion_alpha: alpha^(i) = softmax(W^fuse_{i,:}), computed once when the weights are set
 // (Sec. 4.1: the normalised weights can be cached after training).
-// fuse_layers: one thread-block cluster per new position reads the T target rows of that position
-// exactly once and writes every draft layer's fused, normalised row.
+// fuse_layers: the T target rows of every new position are read once and every draft layer's
+// fused, normalised row is written: a thread-block cluster per position for a handful of
+// positions (one block step), one CTA per position when there are enough to fill the GPU
+// (context fill).
 #include <math.h>
+
+#include <algorithm>
 
 #include <cooperative_groups.h>
 
@@ -179,6 +183,174 @@ __global__ void __launch_bounds__(256) fuse_layers_kernel(
     }
 }
 
+// Many positions (context fill): a persistent grid of CTAs of d/8 threads walks the positions (no
+// cluster). The T target rows of each position (d contiguous elements each) stream through shared
+// memory as 1-D bulk copies issued by one thread, kRB rows per stage, kNS - 1 stages in flight; the
+// stage sequence runs on across positions, so the next position's first rows load while the
+// current one is reduced and stored. Completion is tracked by an mbarrier per stage (bounded
+// waits). Thread t forms the D (<= DMAX) draft-layer sums of features [8t, 8t + 8) in registers,
+// and the CTA reduces the D sums of squares in one pass (warp shuffles, then the warps' partials
+// in order).
+constexpr int kRB = 8;   // target rows per stage
+constexpr int kNS = 2;   // stages (kNS - 1 in flight while one is summed)
+template <class T, int DMAX>
+__global__ void __launch_bounds__(512) fuse_rows_kernel(
+    const T* __restrict__ H, const float* __restrict__ alpha, const T* __restrict__ gain,
+    T* __restrict__ F, T* __restrict__ F_out, const int32_t* __restrict__ app_cnt, int D, int Tn,
+    int batch, int n_max, int d, long long f_layer_rows, float eps, uint32_t* err) {
+    pdl_trigger();
+    extern __shared__ __align__(128) uint8_t stage_mem[];   // [kNS][kRB][d]
+    __shared__ float s_alpha[16 * 64];
+    __shared__ float red[16][DMAX];
+    __shared__ float inv_s[DMAX];
+    __shared__ __align__(8) uint64_t bar[kNS];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(&bar[0]);
+    const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(stage_mem);
+    if (tid == 0) {
+        for (int i = 0; i < kNS; ++i)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar0 + 8u * i) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    pdl_wait();
+    for (int k = tid; k < D * Tn; k += blockDim.x) s_alpha[k] = alpha[k];
+    __syncthreads();
+    const int e0 = tid * 8;
+    const bool act = e0 < d;
+    const int n_pos = batch * n_max;
+    const size_t lstride = (size_t)n_pos * d;
+    const uint32_t row_bytes = (uint32_t)(d * sizeof(T));
+    const T* stg = reinterpret_cast<const T*>(stage_mem);
+    const int nst = (Tn + kRB - 1) / kRB;   // stages per position
+    // this CTA's positions pid = blockIdx.x + k * gridDim.x that have rows to append
+    auto next_pos = [&](int pid) {
+        for (pid += gridDim.x; pid < n_pos; pid += gridDim.x)
+            if (pid % n_max < app_cnt[pid / n_max]) return pid;
+        return n_pos;
+    };
+    int first = (int)blockIdx.x;
+    if (first < n_pos && !(first % n_max < app_cnt[first / n_max])) first = next_pos(first);
+    // stage stream: (position, stage within the position); g counts stages (buffer g % kNS)
+    int ipos = first, ik = 0, g_issue = 0;
+    auto issue_next = [&]() {   // thread 0 only
+        if (ipos >= n_pos) return;
+        const int st = g_issue % kNS, j0 = ik * kRB, nr = min(kRB, Tn - j0);
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar0 + 8u * st),
+                     "r"((uint32_t)nr * row_bytes)
+                     : "memory");
+        for (int u = 0; u < nr; ++u)
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    sbase + (uint32_t)(st * kRB + u) * row_bytes),
+                "l"(H + (size_t)(j0 + u) * lstride + (size_t)ipos * d), "r"(row_bytes), "r"(bar0 + 8u * st)
+                : "memory");
+        ++g_issue;
+        if (++ik == nst) {
+            ik = 0;
+            ipos = next_pos(ipos);
+        }
+    };
+    if (tid == 0)
+        for (int i = 0; i < kNS - 1; ++i) issue_next();
+    int g = 0;   // stages consumed
+    bool ok = true;
+    for (int pid = first; pid < n_pos && ok; pid = next_pos(pid)) {
+        const int b = pid / n_max, r = pid % n_max;
+        float acc[DMAX][8];
+#pragma unroll
+        for (int i = 0; i < DMAX; ++i)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
+        for (int k = 0; k < nst; ++k, ++g) {
+            const int st = g % kNS;
+            if (tid == 0) issue_next();   // stage g + kNS - 1, into the buffer freed after g - 1
+            bool landed = false;
+            {
+                const uint64_t t0 = globaltimer_ns();
+                while (true) {
+                    uint32_t done;
+                    asm volatile(
+                        "{\n\t.reg .pred p;\n\t"
+                        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                        "selp.u32 %0, 1, 0, p;\n\t}"
+                        : "=r"(done)
+                        : "r"(bar0 + 8u * st), "r"((uint32_t)((g / kNS) & 1))
+                        : "memory");
+                    if (done) { landed = true; break; }
+                    if (globaltimer_ns() - t0 > 2000000000ull) break;
+                }
+            }
+            if (__syncthreads_or(!landed)) {
+                if (tid == 0) {
+                    atomicOr(err, DFLARE_DEVERR_TIMEOUT);
+                    // copies still in flight land before the CTA exits (again bounded)
+                    for (int q = g; q < g_issue; ++q) {
+                        const uint64_t t1 = globaltimer_ns();
+                        uint32_t done = 0;
+                        while (!done && globaltimer_ns() - t1 < 2000000000ull)
+                            asm volatile(
+                                "{\n\t.reg .pred p;\n\t"
+                                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                                "selp.u32 %0, 1, 0, p;\n\t}"
+                                : "=r"(done)
+                                : "r"(bar0 + 8u * (q % kNS)), "r"((uint32_t)((q / kNS) & 1))
+                                : "memory");
+                    }
+                }
+                ok = false;
+                break;
+            }
+            if (act) {
+#pragma unroll
+                for (int u = 0; u < kRB; ++u) {
+                    const int j = k * kRB + u;
+                    if (j >= Tn) break;
+                    float h[8];
+                    load8(stg + (size_t)(st * kRB + u) * d + e0, h);
+#pragma unroll
+                    for (int i = 0; i < DMAX; ++i) {
+                        if (i < D) {
+                            const float a = s_alpha[i * Tn + j];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a, h[e], acc[i][e]);
+                        }
+                    }
+                }
+            }
+            __syncthreads();   // stage st is read before it is refilled
+        }
+        if (!ok) break;
+#pragma unroll
+        for (int i = 0; i < DMAX; ++i) {
+            float v = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v = fmaf(acc[i][e], acc[i][e], v);
+            v = warp_sum(v);
+            if (lane == 0) red[warp][i] = v;
+        }
+        __syncthreads();
+        if (tid < D) {
+            float tot = 0.f;
+            for (int w = 0; w < nw; ++w) tot += red[w][tid];
+            inv_s[tid] = inv_rms(tot, d, eps);
+        }
+        __syncthreads();
+        if (act) {
+#pragma unroll
+            for (int i = 0; i < DMAX; ++i) {
+                if (i >= D) break;
+                float gg[8], o[8];
+                load8(gain + (size_t)i * d + e0, gg);
+                const float inv = inv_s[i];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) o[e] = gg[e] * (acc[i][e] * inv);
+                store8(F + ((size_t)i * f_layer_rows + pid) * d + e0, o);
+                if (F_out) store8(F_out + (((size_t)i * batch + b) * n_max + r) * d + e0, o);
+            }
+        }
+    }
+}
+
 template <class T>
 cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,
                           cudaStream_t s) {
@@ -190,6 +362,34 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
     const T* gain = static_cast<const T*>(c->w.fuse_norm);
     T* F = static_cast<T*>(c->fused);
     T* Fo = static_cast<T*>(fused_out);
+    const int rthreads = ((g.d / 8 + 31) / 32) * 32;
+    const size_t rsmem_need = (size_t)kNS * kRB * g.d * sizeof(T);
+    if ((long long)c->batch * n_max >= 2LL * c->num_sms && rsmem_need <= 220 * 1024 &&
+        g.n_draft_layers <= 8) {
+        // enough positions to fill the GPU: one CTA per position
+        auto rk = g.n_draft_layers <= 4 ? fuse_rows_kernel<T, 4>
+                  : g.n_draft_layers == 5 ? fuse_rows_kernel<T, 5> : fuse_rows_kernel<T, 8>;
+        const int threads = rthreads;
+        const size_t rsmem = rsmem_need;
+        static bool rconf = false;
+        if (!rconf) {
+            for (auto k : {fuse_rows_kernel<T, 4>, fuse_rows_kernel<T, 5>, fuse_rows_kernel<T, 8>}) {
+                cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                     220 * 1024);
+                if (e != cudaSuccess) return e;
+            }
+            rconf = true;
+        }
+        // persistent: as many CTAs as fit at once (two per SM at d = 2560), at most one per position
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rk, threads, rsmem) != cudaSuccess || per_sm < 1)
+            per_sm = 1;
+        const int grid = (int)std::min<long long>((long long)c->batch * n_max, (long long)per_sm * c->num_sms);
+        return launch_kernel(c->pdl, rk, dim3(grid), dim3(threads), rsmem, s, H,
+                             (const float*)c->alpha, gain, F, Fo, (const int32_t*)c->app_cnt,
+                             g.n_draft_layers, g.n_target_layers, c->batch, n_max, g.d,
+                             (long long)g.max_fuse_rows, g.rms_eps, c->err);
+    }
     auto kern = g.n_draft_layers <= 4 ? fuse_layers_kernel<T, 4> : fuse_layers_kernel<T, 8>;
     static bool configured = false;
     if (!configured) {

@@ -23,6 +23,18 @@ SMALL_HD64 = synth.Workload(
     synth.Shape(d=384, n_draft_layers=2, n_target_layers=4, n_q_heads=8, n_kv_heads=2,
                 head_dim=64, ffn=640, vocab=2048, block=8),
     (65, 300), 0.75, seed=12)
+# many token rows per projection: batch 16 x block 16 = 256 rows (the widest GEMM token tile and
+# a 240-row LM head), and block 32 (31 mask rows, two 64-row query tiles per KV head)
+WIDE_B16 = synth.Workload(
+    "wide_bf16_b16",
+    synth.Shape(d=384, n_draft_layers=2, n_target_layers=3, n_q_heads=8, n_kv_heads=2,
+                head_dim=64, ffn=640, vocab=1024, block=16),
+    tuple(9 + (37 * b) % 61 for b in range(16)), 0.8, seed=13)
+BLOCK32 = synth.Workload(
+    "block32_bf16",
+    synth.Shape(d=256, n_draft_layers=2, n_target_layers=3, n_q_heads=8, n_kv_heads=2,
+                head_dim=128, ffn=512, vocab=1500, block=32),
+    (90, 17), 0.8, seed=14)
 TINY = synth.preset("tiny_f32")
 
 

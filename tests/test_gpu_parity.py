@@ -8,8 +8,8 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import (SMALL_HD128, SMALL_HD64, TINY, GpuRun, f64, oracle_for, rel_err,
-                           tolerance)
+from tests.harness import (BLOCK32, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16, GpuRun, f64, oracle_for,
+                           rel_err, tolerance)
 
 pytestmark = pytest.mark.gpu
 GAP = 1e-2
@@ -195,3 +195,21 @@ def test_simt_gemm_agrees_with_tcgen05_gemm():
     tb, lb, hb = b.draft(x_t)
     assert rel_err(ha, hb) <= tolerance(w)
     assert rel_err(la, lb) <= tolerance(w)
+
+
+@pytest.mark.parametrize("w", [WIDE_B16, BLOCK32], ids=lambda w: w.name)
+def test_wide_token_tiles_match_oracle(w):
+    """256 token rows per projection (batch 16, the widest tcgen05 token tile) and block 32: fused
+    context, cached K/V and the draft block against the oracle."""
+    g = GpuRun(w)
+    o = oracle_for(w, g.W)
+    fused = f64(g.fuse(w.ctx_lens))
+    for b, n in enumerate(w.ctx_lens):
+        F = o.fuse_context(b, synth.hidden_states(w, b, 0, n))
+        assert rel_err(fused[:, b, :n], F) <= tolerance(w), b
+        k, v = g.lib.read_kv(w.shape.n_draft_layers - 1, b, 0, n)
+        assert rel_err(f64(k), o.ctx_k[b][w.shape.n_draft_layers - 1]) <= tolerance(w), b
+    x_t = synth.initial_tokens(w)
+    tok, logits, hidden = g.draft(x_t)
+    _check_draft(w, tok, logits, hidden, [o.draft_block(b, int(x_t[b])) for b in range(w.batch)])
+    assert g.lib.device_error() == 0
