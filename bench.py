@@ -51,6 +51,8 @@ def parse():
     p.add_argument("--fill-chunk", type=int, default=2048)
     p.add_argument("--serial-launch", action="store_true",
                    help="no programmatic dependent launch between kernels (A/B measurement)")
+    p.add_argument("--no-variants", action="store_true",
+                   help="skip the context-fusion comparison with the ablations and DFlash's FC")
     return p.parse_args()
 
 
@@ -283,6 +285,84 @@ def gemm_traffic(w):
     return d.get("dram_bytes_per_step")
 
 
+FUSION_VARIANTS = (("dflare", ()), ("minus_kvproj", ("FLAG_SHARED_KV",)),
+                   ("plus_fc", ("FLAG_FUSION_FC",)), ("dflash_fc", ("FLAG_DFLASH_FC",)))
+
+
+def fusion_variants(w, dev_w, fill_chunks, hid_step, n_step, reps=100):
+    """Time one dflare_fuse_context call (fusion, optional FC, context K/V projection) of DFlare
+    and of each variant: at decode (n_step new positions per sequence, a CUDA graph of one call
+    replayed `reps` times between events) and at a context fill (the fill chunks, once untimed,
+    then timed from an empty context)."""
+    import torch
+    import paper_2606_02091_gb300 as P
+    from paper_2606_02091_gb300 import DFlare
+    s = w.shape
+    esz = 2 if s.dtype == "bf16" else 4
+    extra = {}
+    for k, v in synth.variant_weights(w).items():
+        t = torch.from_numpy(v)
+        extra[k] = (t.view(torch.bfloat16) if v.dtype == np.uint16 else t).cuda()
+    n_fill = sum(w.ctx_lens)
+    fill_rows = max(Ht.shape[2] for Ht, _ in fill_chunks)
+    n_new = torch.full((w.batch,), n_step, dtype=torch.int32, device="cuda")
+    out = {}
+    for name, flags in FUSION_VARIANTS:
+        flag = 0
+        for f in flags:
+            flag |= getattr(P, f)
+        lib = DFlare.from_shape(s, max_batch=w.batch, max_ctx=max(w.ctx_lens) + n_step * (reps + 8),
+                                max_fuse_rows=w.batch * max(fill_rows, s.block), flags=flag)
+        lib.set_weights({**dev_w, **extra})
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        fill_ms = None
+        for timed in (False, True):
+            lib.reset(w.batch)
+            torch.cuda.synchronize()
+            ev[0].record()
+            for Ht, nt in fill_chunks:
+                lib.fuse_context(Ht, nt)
+            ev[1].record()
+            torch.cuda.synchronize()
+            fill_ms = ev[0].elapsed_time(ev[1])
+        lib.reset(w.batch)
+        cs = torch.cuda.Stream()
+        cs.wait_stream(torch.cuda.current_stream())
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cs):
+            lib.fuse_context(hid_step, n_new)
+            torch.cuda.synchronize()
+            with torch.cuda.graph(graph, stream=cs):
+                lib.fuse_context(hid_step, n_new)
+        torch.cuda.synchronize()
+        lib.reset(w.batch)
+        for _ in range(3):
+            graph.replay()
+        torch.cuda.synchronize()
+        ev[2].record()
+        for _ in range(reps):
+            graph.replay()
+        ev[3].record()
+        torch.cuda.synchronize()
+        if lib.device_error():
+            raise RuntimeError(f"device error in the {name} fusion variant")
+        step_us = 1e3 * ev[2].elapsed_time(ev[3]) / reps
+        wbytes = {"dflare": s.n_draft_layers * 2 * s.d_kv * s.d,
+                  "minus_kvproj": s.n_draft_layers * 2 * s.d_kv * s.d,
+                  "plus_fc": s.n_draft_layers * (2 * s.d_kv + s.d) * s.d,
+                  "dflash_fc": s.n_target_layers * s.d * s.d + s.n_draft_layers * 2 * s.d_kv * s.d}
+        out[name] = {"step_us": step_us, "fill_us": 1e3 * fill_ms,
+                     "weight_bytes_per_call": wbytes[name] * esz}
+        del graph
+        lib.close()
+    out["note"] = (f"one dflare_fuse_context call per entry: decode = {n_step} new positions per "
+                   f"sequence (CUDA graph of one call, {reps} replays); fill = {n_fill} positions "
+                   "from empty. dflare: Eq. 3 + Eq. 4; minus_kvproj / plus_fc: the Sec. 6.3 "
+                   "ablations; dflash_fc: Eq. 1 (one GEMM over the T stacked target layers) + "
+                   "Eq. 2's shared K/V projection")
+    return out
+
+
 def replica_aggregate(ms, units_per_step, steps, dist=None, device="cuda"):
     """Weak-scaling aggregate of independent replicas (one per rank, no data-path exchange):
     the job's time is the slowest rank's, its throughput every rank's units over that time.
@@ -360,7 +440,6 @@ def run_ours(args):
         if timed:
             P.load().dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
         torch.cuda.synchronize()
-    del fill_chunks
     fill_us = {}
     open_f = {}
     for name, phase, e in fill_ev:
@@ -590,6 +669,10 @@ def run_ours(args):
         "launches_per_step": launches_per_step,
         "clocks": clk,
     }
+    if not args.no_variants:
+        line["fusion_variants"] = fusion_variants(w, dev_w, fill_chunks, hid_step,
+                                                  max(1, int(round(mean_tau))))
+    del fill_chunks
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, dt, tau = oracle_steps(w, W, args.cpu_steps)
         line["cpu_baseline"] = {

@@ -65,6 +65,21 @@ typedef enum { DFLARE_BF16 = 0, DFLARE_F32 = 1 } dflare_dtype;
                                            instead of with programmatic dependent launch (which
                                            lets a kernel's prologue and weight prefetch overlap the
                                            previous kernel's tail); for measurements */
+#define DFLARE_FLAG_SHARED_KV     0x10u /* the "-KVProj" ablation of Sec. 6.3 (Table 2): context
+                                           keys/values use the layer's own W_K^d / W_V^d (rows
+                                           [d_q, d_q + 2 d_kv) of w_qkv) instead of W^t of Eq. 4;
+                                           w_kv_ctx is not read and may be NULL */
+#define DFLARE_FLAG_FUSION_FC     0x20u /* the "+FC" ablation of Sec. 6.3 (Table 2): one more
+                                           fully-connected layer per draft layer after the fusion,
+                                           F'^(i) = F^(i) W_fc^(i)T + b_fc^(i) (weights fusion_fc_w,
+                                           fusion_fc_b), which then feeds Eq. 4 in place of F^(i) */
+#define DFLARE_FLAG_DFLASH_FC     0x40u /* the DFlash baseline of Sec. 2.2-2.3: one context feature
+                                           c_t = W_fc [h_t^(1); ...; h_t^(T)] + b_fc (Eq. 1) for
+                                           every draft layer, projected by the layer's own W_K /
+                                           W_V as in Eq. 2 (weights dflash_fc_w, dflash_fc_b);
+                                           fuse_logits, fuse_norm and w_kv_ctx are not read and
+                                           may be NULL. Cannot be combined with RAW_FUSION or
+                                           FUSION_FC (DFLARE_EINVAL) */
 
 /* Device error word bits (dflare_device_error) */
 #define DFLARE_DEVERR_TOKEN     0x1u    /* a token id outside [0, vocab) was read (clamped to 0) */
@@ -112,6 +127,12 @@ typedef struct {
     const void* final_norm;    /* [d] T: RMSNorm before the LM head */
     const void* embed;         /* [V][d] T: token embedding shared with the target (Sec. 3.3) */
     const void* lm_head;       /* [V][d] T: LM head shared with the target (Sec. 3.3) */
+    /* read only under the flag named; NULL otherwise */
+    const void* fusion_fc_w;   /* [D][d][d] T: DFLARE_FLAG_FUSION_FC, per-layer FC after Eq. 3 */
+    const void* fusion_fc_b;   /* [D][d] T: DFLARE_FLAG_FUSION_FC, its bias */
+    const void* dflash_fc_w;   /* [d][T*d] T: DFLARE_FLAG_DFLASH_FC, W_fc of Eq. 1 (column j*d+e
+                                  multiplies element e of target layer j's state) */
+    const void* dflash_fc_b;   /* [d] T: DFLARE_FLAG_DFLASH_FC, b_fc of Eq. 1 */
 } dflare_weights;
 
 typedef struct dflare_ctx dflare_ctx;
@@ -141,7 +162,10 @@ dflare_status dflare_reset(dflare_ctx* ctx, int batch, void* stream);
  *   n_new_dev          [batch] int32: positions to append per sequence, each in [0, n_max]
  *                      (typically the previous step's accept_len, or the prompt length first).
  *   n_max              row stride of target_hidden; batch * n_max <= max_fuse_rows.
- *   fused_out_dev      optional [D][batch][n_max][d] T: the fused context f^(i) (Eq. 3).
+ *   fused_out_dev      optional [D][batch][n_max][d] T: the context representation each layer
+ *                      projects: f^(i) of Eq. 3 (with DFLARE_FLAG_FUSION_FC: the FC's output
+ *                      F'^(i)); with DFLARE_FLAG_DFLASH_FC only slot 0 is written, with c_t of
+ *                      Eq. 1, which every layer shares. Rows r >= n_new[b] are unspecified.
  * Sequence b's new rows get positions ctx_len[b] .. ctx_len[b]+n_new[b]-1; keys are rotated at
  * those positions and cached; ctx_len[b] grows by n_new[b]. A sequence that would exceed max_ctx
  * appends nothing and sets DFLARE_DEVERR_CAPACITY.
@@ -194,7 +218,8 @@ dflare_status dflare_device_error(dflare_ctx* ctx, uint32_t* bits_host, void* st
 
 /* Optional tracing. When set, fn(user, name, phase, stream) is called on the host right before
  * (phase 0) and right after (phase 1) the library enqueues each of its kernel launches on
- * `stream` (name: "fuse_begin", "fuse_layers", "gemm_kv_ctx", "embed", "rmsnorm", "gemm_qkv",
+ * `stream` (name: "fuse_begin", "fuse_layers", "gemm_fusion_fc", "gemm_dflash_fc",
+ * "gemm_kv_ctx", "embed", "rmsnorm", "gemm_qkv",
  * "attention", "gemm_o", "gemm_gate_up", "gemm_down", "gemm_lm_head", "argmax", "verify").
  * A caller can record CUDA events there, also while the stream is being captured into a graph.
  * fn = NULL turns tracing off. */

@@ -18,6 +18,8 @@ and notation (arxiv 2606.02091):
   layer to layer; logits are taken at the mask positions and greedy drafting takes the argmax.
 * Sec. 3.2 (verification phase): accept the longest prefix of drafts that matches the target's
   own predictions, plus one token from the target.
+* Variants measured against DFlare: the ablations of Sec. 6.3 / Table 2 ("-Softmax", "-KVProj",
+  "+FC") and DFlash's FC fusion (Eq. 1) with one shared KV projection (Eq. 2).
 
 Where the paper is silent the oracle takes these readings (each is also listed in the design doc):
 pre-norm residual blocks (RMSNorm -> attention -> residual; RMSNorm -> SwiGLU MLP -> residual)
@@ -147,6 +149,30 @@ def context_kv(F_i, w_kv_ctx_i, positions, n_kv_heads: int, head_dim: int, theta
     return store(rope(k, positions, theta)), store(v)
 
 
+# --------------------------------------------------------------------------- Sec. 6.3 / Eq. 1 variants
+
+def fusion_fc(F_i, w_fc_i, b_fc_i, store=exact):
+    """The "+FC" ablation of Sec. 6.3 (Table 2): one more fully-connected layer applied to the
+    fused context of draft layer i before it is projected, F'^(i)_t = W_fc^(i) f_t^(i) + b_fc^(i).
+
+    F_i: [n][d]; w_fc_i: [d][d] (out x in); b_fc_i: [d]. Returns F'^(i): [n][d].
+    """
+    F_i = np.asarray(F_i, F64)
+    return store(F_i @ np.asarray(w_fc_i, F64).T + np.asarray(b_fc_i, F64))
+
+
+def dflash_context(hidden, w_fc, b_fc, store=exact):
+    """DFlash's context feature (Eq. 1): c_t = W_fc [h_t^(1); ...; h_t^(T)] + b_fc.
+
+    hidden: [T][n][d]; w_fc: [d][T d], so column j d + e multiplies element e of h_t^(j+1);
+    b_fc: [d]. Returns C: [n][d], one row per position, shared by every draft layer (Eq. 2).
+    """
+    hidden = np.asarray(hidden, F64)
+    T = hidden.shape[0]
+    concat = np.concatenate([hidden[j] for j in range(T)], axis=-1)   # [n][T d]
+    return store(concat @ np.asarray(w_fc, F64).T + np.asarray(b_fc, F64))
+
+
 # --------------------------------------------------------------------------- Sec. 3.2 block
 
 def silu(x):
@@ -261,17 +287,34 @@ class DraftOracle:
     weights: dict of input arrays in the library's stacked layout (bf16 bit patterns or fp32),
     as produced by ``synth.weights``. shape: the drafter's architecture. storage: "bf16" applies
     bf16 storage rounding (the bf16 path's reference), "exact" none (the fp32 path's).
+
+    Variants (Sec. 6.3, Table 2, and the DFlash design of Sec. 2.2-2.3):
+    softmax_fusion=False  "-Softmax": alpha = W^fuse as it is;
+    shared_kv=True        "-KVProj": context rows are projected by the layer's own W_K^d, W_V^d
+                          (the K and V rows of w_qkv) instead of W_K^t, W_V^t;
+    fusion_fc=True        "+FC": F'^(i) = W_fc^(i) F^(i) + b_fc^(i) (weights fusion_fc_w,
+                          fusion_fc_b) replaces F^(i) before the projection;
+    dflash_fc=True        DFlash: every layer projects the same c_t of Eq. 1 (weights
+                          dflash_fc_w, dflash_fc_b) with its own W_K, W_V (Eq. 2); the layer-wise
+                          fusion and W^t are not used.
     """
 
     def __init__(self, weights: dict, shape, batch: int, storage: str = "exact",
-                 softmax_fusion: bool = True, rope_block: bool = True):
+                 softmax_fusion: bool = True, rope_block: bool = True, shared_kv: bool = False,
+                 fusion_fc: bool = False, dflash_fc: bool = False):
+        if dflash_fc and (fusion_fc or not softmax_fusion):
+            raise ValueError("dflash_fc replaces the layer-wise fusion")
         self.w = weights
         self.s = shape
         self.batch = batch
         self.store = round_bf16 if storage == "bf16" else exact
         self.rope_block = rope_block
+        self.shared_kv = shared_kv or dflash_fc
+        self.fusion_fc = fusion_fc
+        self.dflash_fc = dflash_fc
         self._cache = {}
-        self.alpha = fusion_weights(weights["fuse_logits"], softmax=softmax_fusion)
+        self.alpha = None if dflash_fc else fusion_weights(weights["fuse_logits"],
+                                                           softmax=softmax_fusion)
         D = shape.n_draft_layers
         empty = np.zeros((0, shape.n_kv_heads, shape.head_dim))
         self.ctx_k = [[empty] * D for _ in range(batch)]
@@ -294,16 +337,28 @@ class DraftOracle:
 
     def fuse_context(self, b: int, hidden):
         """Fuse n newly committed positions of sequence b (hidden: [T][n][d] input bytes) and
-        append their keys/values to every layer's context cache. Returns F [D][n][d]."""
+        append their keys/values to every layer's context cache. Returns the representation
+        each layer projects, [D][n][d]: F^(i) (Eq. 3), F'^(i) under "+FC", c (Eq. 1) under
+        DFlash."""
         s = self.s
+        D = s.n_draft_layers
         h = decode(hidden, s.dtype)
         n = h.shape[1]
-        F = fuse_context(h, self.alpha, self._dec("fuse_norm"), s.rms_eps, self.store)
+        if self.dflash_fc:
+            C = dflash_context(h, self._dec("dflash_fc_w"), self._dec("dflash_fc_b"), self.store)
+            F = np.stack([C] * D)
+        else:
+            F = fuse_context(h, self.alpha, self._dec("fuse_norm"), s.rms_eps, self.store)
+            if self.fusion_fc:
+                F = np.stack([fusion_fc(F[i], self._dec("fusion_fc_w", i),
+                                        self._dec("fusion_fc_b", i), self.store)
+                              for i in range(D)])
         L = self.ctx_len(b)
         pos = np.arange(L, L + n)
-        for i in range(s.n_draft_layers):
-            k, v = context_kv(F[i], self._dec("w_kv_ctx", i), pos, s.n_kv_heads, s.head_dim,
-                              s.rope_theta, self.store)
+        for i in range(D):
+            # [W_K ; W_V] of the context rows: W^t (Eq. 4), or the block's own W^d (Eq. 2)
+            w_kv = self._dec("w_qkv", i)[s.d_q:] if self.shared_kv else self._dec("w_kv_ctx", i)
+            k, v = context_kv(F[i], w_kv, pos, s.n_kv_heads, s.head_dim, s.rope_theta, self.store)
             self.ctx_k[b][i] = np.concatenate([self.ctx_k[b][i], k])
             self.ctx_v[b][i] = np.concatenate([self.ctx_v[b][i], v])
         return F

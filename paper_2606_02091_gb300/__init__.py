@@ -12,7 +12,7 @@ import ctypes
 from . import _lib
 from ._lib import (  # noqa: F401
     DFlareError, DFLARE_BF16, DFLARE_F32, FLAG_NO_BLOCK_ROPE, FLAG_RAW_FUSION, FLAG_SIMT_GEMM,
-    FLAG_SERIAL_LAUNCH,
+    FLAG_SERIAL_LAUNCH, FLAG_SHARED_KV, FLAG_FUSION_FC, FLAG_DFLASH_FC,
     DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT, EXPORTS, WEIGHT_FIELDS, NOALLOC_MAX_ROWS, load,
 )
 
@@ -90,10 +90,15 @@ class DFlare:
         return self._ctx
 
     def set_weights(self, weights: dict, stream=None):
-        """weights: name -> CUDA tensor in the layout of ``dflare_weights`` (kept alive here)."""
+        """weights: name -> CUDA tensor in the layout of ``dflare_weights`` (kept alive here).
+
+        A missing or None entry is passed as NULL; the library rejects a NULL weight that the
+        context's flags read."""
         w = _lib.Weights()
         for name in WEIGHT_FIELDS:
-            t = weights[name]
+            t = weights.get(name)
+            if t is None:
+                continue
             _need_cuda(name, t)
             setattr(w, name, t.data_ptr())
         self._weights = dict(weights)

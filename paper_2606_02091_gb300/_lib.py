@@ -20,6 +20,9 @@ FLAG_NO_BLOCK_ROPE = 0x1
 FLAG_RAW_FUSION = 0x2
 FLAG_SIMT_GEMM = 0x4
 FLAG_SERIAL_LAUNCH = 0x8
+FLAG_SHARED_KV = 0x10
+FLAG_FUSION_FC = 0x20
+FLAG_DFLASH_FC = 0x40
 DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT = 0x1, 0x2, 0x4
 
 STATUS_NAMES = {0: "DFLARE_OK", 1: "DFLARE_EINVAL", 2: "DFLARE_ECAPACITY", 3: "DFLARE_ECUDA",
@@ -47,7 +50,8 @@ class Config(ctypes.Structure):
 
 
 WEIGHT_FIELDS = ("fuse_logits", "fuse_norm", "w_kv_ctx", "attn_norm", "w_qkv", "w_o", "mlp_norm",
-                 "w_gate", "w_up", "w_down", "final_norm", "embed", "lm_head")
+                 "w_gate", "w_up", "w_down", "final_norm", "embed", "lm_head",
+                 "fusion_fc_w", "fusion_fc_b", "dflash_fc_w", "dflash_fc_b")
 
 
 class Weights(ctypes.Structure):

@@ -61,8 +61,12 @@ bool check_config(const dflare_config* g, std::string* why) {
     if (!(g->rope_theta > 0.f) || !isfinite(g->rope_theta)) return bad("rope_theta must be finite and > 0");
     if (g->dtype != DFLARE_BF16 && g->dtype != DFLARE_F32) return bad("dtype must be DFLARE_BF16 or DFLARE_F32");
     if (g->flags & ~(DFLARE_FLAG_NO_BLOCK_ROPE | DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_SIMT_GEMM |
-                     DFLARE_FLAG_SERIAL_LAUNCH))
+                     DFLARE_FLAG_SERIAL_LAUNCH | DFLARE_FLAG_SHARED_KV | DFLARE_FLAG_FUSION_FC |
+                     DFLARE_FLAG_DFLASH_FC))
         return bad("unknown flag bits");
+    if ((g->flags & DFLARE_FLAG_DFLASH_FC) &&
+        (g->flags & (DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_FUSION_FC)))
+        return bad("DFLARE_FLAG_DFLASH_FC replaces the layer-wise fusion: no RAW_FUSION or FUSION_FC");
     return true;
 }
 
@@ -206,6 +210,7 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     ALLOC(c->app_cnt, g.max_batch * sizeof(int32_t));
     ALLOC(c->alpha, D * g.n_target_layers * sizeof(float));
     ALLOC(c->fused, D * (size_t)g.max_fuse_rows * d * esz);
+    if (g.flags & DFLARE_FLAG_FUSION_FC) ALLOC(c->fused_fc, D * (size_t)g.max_fuse_rows * d * esz);
     ALLOC(c->x, rows * d * sizeof(float));
     ALLOC(c->xn, rows * d * esz);
     ALLOC(c->q, rows * d_q * esz);
@@ -271,19 +276,29 @@ dflare_status dflare_destroy(dflare_ctx* c) {
 dflare_status dflare_set_weights(dflare_ctx* c, const dflare_weights* w, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
     if (!w) return fail(c, DFLARE_EINVAL, "weights is NULL");
-    const void* ptrs[] = {w->fuse_logits, w->fuse_norm, w->w_kv_ctx, w->attn_norm, w->w_qkv,
-                          w->w_o, w->mlp_norm, w->w_gate, w->w_up, w->w_down, w->final_norm,
-                          w->embed, w->lm_head};
-    const char* names[] = {"fuse_logits", "fuse_norm", "w_kv_ctx", "attn_norm", "w_qkv", "w_o",
-                           "mlp_norm", "w_gate", "w_up", "w_down", "final_norm", "embed", "lm_head"};
-    for (int i = 0; i < 13; ++i) {
-        if (!ptrs[i]) return fail(c, DFLARE_EINVAL, std::string("weight ") + names[i] + " is NULL");
-        if (reinterpret_cast<uintptr_t>(ptrs[i]) % 16 != 0)
-            return fail(c, DFLARE_EINVAL, std::string("weight ") + names[i] + " is not 16-byte aligned");
+    const unsigned fl = c->cfg.flags;
+    const bool dflash = fl & DFLARE_FLAG_DFLASH_FC;
+    // (pointer, name, read under the context's flags)
+    struct Need { const void* p; const char* name; bool used; } need[] = {
+        {w->fuse_logits, "fuse_logits", !dflash},
+        {w->fuse_norm, "fuse_norm", !dflash},
+        {w->w_kv_ctx, "w_kv_ctx", !dflash && !(fl & DFLARE_FLAG_SHARED_KV)},
+        {w->attn_norm, "attn_norm", true}, {w->w_qkv, "w_qkv", true}, {w->w_o, "w_o", true},
+        {w->mlp_norm, "mlp_norm", true}, {w->w_gate, "w_gate", true}, {w->w_up, "w_up", true},
+        {w->w_down, "w_down", true}, {w->final_norm, "final_norm", true}, {w->embed, "embed", true},
+        {w->lm_head, "lm_head", true},
+        {w->fusion_fc_w, "fusion_fc_w", (fl & DFLARE_FLAG_FUSION_FC) != 0},
+        {w->fusion_fc_b, "fusion_fc_b", (fl & DFLARE_FLAG_FUSION_FC) != 0},
+        {w->dflash_fc_w, "dflash_fc_w", dflash}, {w->dflash_fc_b, "dflash_fc_b", dflash}};
+    for (const Need& n : need) {
+        if (!n.used) continue;
+        if (!n.p) return fail(c, DFLARE_EINVAL, std::string("weight ") + n.name + " is NULL");
+        if (reinterpret_cast<uintptr_t>(n.p) % 16 != 0)
+            return fail(c, DFLARE_EINVAL, std::string("weight ") + n.name + " is not 16-byte aligned");
     }
     c->w = *w;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    CUDA_TRY(launch_fusion_alpha(c, s));
+    if (!dflash) CUDA_TRY(launch_fusion_alpha(c, s));
     c->weights_set = true;
     return DFLARE_OK;
 }
@@ -312,22 +327,85 @@ dflare_status dflare_fuse_context(dflare_ctx* c, const void* hidden, const int32
         return fail(c, DFLARE_EINVAL, "target_hidden and fused_out must be 16-byte aligned");
     const dflare_config& g = c->cfg;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int m_tok = c->batch * n_max;
+    const size_t d_q = (size_t)g.n_q_heads * g.head_dim, d_kv = (size_t)g.n_kv_heads * g.head_dim;
     {
         Trace t(c, "fuse_begin", s);
         CUDA_TRY(launch_fuse_begin(c, n_new, n_max, s));
     }
-    {
-        Trace t(c, "fuse_layers", s);
-        CUDA_TRY(launch_fuse_layers(c, hidden, n_max, fused_out, s));
+    // ctx_src: what the context K/V projection reads, [groups][ctx_rows][d]
+    const void* ctx_src = c->fused;
+    long long ctx_rows = g.max_fuse_rows;
+    int ctx_shared = 0;
+    if (g.flags & DFLARE_FLAG_DFLASH_FC) {
+        // Eq. 1: c_t = W_fc [h^(1); ...; h^(T)] + b_fc as one GEMM whose contraction runs over
+        // the T stacked target layers of target_hidden; one c for every draft layer
+        GemmDesc fc{};
+        fc.a = c->w.dflash_fc_w;
+        fc.b = hidden;
+        fc.groups = 1;
+        fc.n = g.d;
+        fc.k = g.n_target_layers * g.d;
+        fc.m_tok = m_tok;
+        fc.b_group_rows = m_tok;
+        fc.b_kgroup = g.d;
+        fc.ep = epi_base(c);
+        fc.ep.kind = EPI_STORE;
+        fc.ep.m_tok = m_tok;
+        fc.ep.n = g.d;
+        fc.ep.out = fused_out ? fused_out : c->fused;
+        fc.ep.ldo = g.d;
+        fc.ep.bias = c->w.dflash_fc_b;
+        dflare_status st = traced_gemm(c, "gemm_dflash_fc", fc, s);
+        if (st != DFLARE_OK) return st;
+        ctx_src = fc.ep.out;
+        ctx_rows = m_tok;
+        ctx_shared = 1;
+    } else {
+        const bool fc_after = g.flags & DFLARE_FLAG_FUSION_FC;
+        {
+            Trace t(c, "fuse_layers", s);
+            CUDA_TRY(launch_fuse_layers(c, hidden, n_max, fc_after ? nullptr : fused_out, s));
+        }
+        if (fc_after) {
+            // "+FC": F'^(i) = F^(i) W_fc^(i)T + b_fc^(i), one d x d GEMM per draft layer
+            GemmDesc fc{};
+            fc.a = c->w.fusion_fc_w;
+            fc.b = c->fused;
+            fc.groups = g.n_draft_layers;
+            fc.n = g.d;
+            fc.k = g.d;
+            fc.m_tok = m_tok;
+            fc.b_group_rows = g.max_fuse_rows;
+            fc.ep = epi_base(c);
+            fc.ep.kind = EPI_STORE;
+            fc.ep.m_tok = m_tok;
+            fc.ep.n = g.d;
+            fc.ep.out = fused_out ? fused_out : c->fused_fc;
+            fc.ep.ldo = g.d;
+            fc.ep.out_gstride = (fused_out ? (long long)m_tok : g.max_fuse_rows) * g.d;
+            fc.ep.bias = c->w.fusion_fc_b;
+            dflare_status st = traced_gemm(c, "gemm_fusion_fc", fc, s);
+            if (st != DFLARE_OK) return st;
+            ctx_src = fc.ep.out;
+            ctx_rows = fused_out ? (long long)m_tok : g.max_fuse_rows;
+        }
     }
     GemmDesc gd{};
-    gd.a = c->w.w_kv_ctx;
-    gd.b = c->fused;
+    if (g.flags & (DFLARE_FLAG_SHARED_KV | DFLARE_FLAG_DFLASH_FC)) {
+        // W_K^d / W_V^d: rows [d_q, d_q + 2 d_kv) of each layer's w_qkv
+        gd.a = at(c->w.w_qkv, d_q * g.d, c->esz);
+        gd.a_group_rows = (long long)(d_q + 2 * d_kv);
+    } else {
+        gd.a = c->w.w_kv_ctx;
+    }
+    gd.b = ctx_src;
+    gd.b_shared = ctx_shared;
     gd.groups = g.n_draft_layers;
-    gd.n = 2 * g.n_kv_heads * g.head_dim;
+    gd.n = (int)(2 * d_kv);
     gd.k = g.d;
-    gd.m_tok = c->batch * n_max;
-    gd.b_group_rows = g.max_fuse_rows;
+    gd.m_tok = m_tok;
+    gd.b_group_rows = ctx_rows;
     gd.ep = epi_base(c);
     gd.ep.kind = EPI_KV_APPEND;
     gd.ep.m_tok = gd.m_tok;

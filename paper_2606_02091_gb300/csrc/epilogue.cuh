@@ -20,7 +20,9 @@ __device__ __forceinline__ float silu_f(float g) { return __fdividef(g, 1.0f + _
 // Every branch issues all of its global loads (residual values, per-token positions, rotary
 // factors) before its first store, so the loads of the 16 tokens of a chunk are in flight
 // together instead of each waiting behind the previous token's store.
-template <class T>
+// kAux: compile the biased, group-strided store (EPI_STORE of the fusion variants); without it
+// EPI_STORE writes group 0's layout with no bias.
+template <class T, bool kAux = true>
 __device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float* tile, int group,
                                                int n_tile, int tok0, int t) {
     constexpr int NC = kEpiChunk;
@@ -31,10 +33,20 @@ __device__ __forceinline__ void apply_epilogue(const EpiParams& ep, const float*
     if (nvalid <= 0) return;
     switch (ep.kind) {
         case EPI_STORE: {
-            T* out = reinterpret_cast<T*>(ep.out);
+            if constexpr (kAux) {
+                T* out = reinterpret_cast<T*>(ep.out) + (size_t)group * ep.out_gstride;
+                const float bv =
+                    ep.bias ? to_f(reinterpret_cast<const T*>(ep.bias)[(size_t)group * ep.n + n]) : 0.f;
 #pragma unroll
-            for (int c = 0; c < NC; ++c)
-                if (c < nvalid) out[(size_t)(tok0 + c) * ep.ldo + n] = from_f<T>(tile[c * 128 + t]);
+                for (int c = 0; c < NC; ++c)
+                    if (c < nvalid)
+                        out[(size_t)(tok0 + c) * ep.ldo + n] = from_f<T>(tile[c * 128 + t] + bv);
+            } else {
+                T* out = reinterpret_cast<T*>(ep.out);
+#pragma unroll
+                for (int c = 0; c < NC; ++c)
+                    if (c < nvalid) out[(size_t)(tok0 + c) * ep.ldo + n] = from_f<T>(tile[c * 128 + t]);
+            }
         } break;
         case EPI_F32: {
             float* out = reinterpret_cast<float*>(ep.out);

@@ -14,8 +14,9 @@ constexpr int kTK = 16;    // K chunk
 template <class T>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ A2,
                                                         const T* __restrict__ Bm, int n, int k,
-                                                        int m_tok, long long b_group_rows,
-                                                        int n_tiles, EpiParams ep) {
+                                                        int m_tok, long long a_group_rows,
+                                                        long long b_group_rows, int b_shared,
+                                                        int b_kgroup, int n_tiles, EpiParams ep) {
     pdl_trigger();
     pdl_wait();
     __shared__ float sA[2][kTN][kTK + 1];
@@ -26,9 +27,9 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
     const int na = A2 ? 2 : 1;
     const int tid = threadIdx.x;
     const int f = tid & 127, tg = tid >> 7;   // feature f, tokens tg*8 .. tg*8+7
-    const T* Ag = A + (size_t)group * n * k;
-    const T* A2g = A2 ? A2 + (size_t)group * n * k : nullptr;
-    const T* Bg = Bm + (size_t)group * b_group_rows * k;
+    const T* Ag = A + (size_t)group * a_group_rows * k;
+    const T* A2g = A2 ? A2 + (size_t)group * a_group_rows * k : nullptr;
+    const T* Bg = Bm + (size_t)(b_shared ? 0 : group) * b_group_rows * k;
     float acc[2][8];
 #pragma unroll
     for (int a = 0; a < 2; ++a)
@@ -46,7 +47,16 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
         for (int idx = tid; idx < kTT * kTK; idx += 256) {
             const int r = idx / kTK, cc = idx % kTK;
             const int tok = tok0 + r, col = k0 + cc;
-            sB[r][cc] = (tok < m_tok && col < k) ? to_f(Bg[(size_t)tok * k + col]) : 0.f;
+            float v = 0.f;
+            if (tok < m_tok && col < k) {
+                if (b_kgroup > 0) {   // contraction over stacked activation groups (Eq. 1)
+                    const int z = col / b_kgroup;
+                    v = to_f(Bm[((size_t)z * b_group_rows + tok) * b_kgroup + (col - z * b_kgroup)]);
+                } else {
+                    v = to_f(Bg[(size_t)tok * k + col]);
+                }
+            }
+            sB[r][cc] = v;
         }
         __syncthreads();
         for (int a = 0; a < na; ++a)
@@ -69,14 +79,16 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 cudaError_t launch_gemm_simt(dflare_ctx* c, const GemmDesc& g, cudaStream_t s) {
     if (g.m_tok <= 0 || g.n <= 0) return cudaSuccess;
     const int n_tiles = (g.n + kTN - 1) / kTN;
+    if (g.b_kgroup > 0 && (g.k % g.b_kgroup != 0 || g.groups != 1)) return cudaErrorInvalidValue;
     dim3 grid(n_tiles * g.groups, (g.m_tok + kTT - 1) / kTT);
+    const long long a_gr = g.a_group_rows > 0 ? g.a_group_rows : g.n;
     if (c->cfg.dtype == DFLARE_F32)
         return launch_kernel(c->pdl, gemm_simt_kernel<float>, grid, dim3(256), 0, s,
                              (const float*)g.a, (const float*)g.a2, (const float*)g.b, g.n, g.k,
-                             g.m_tok, g.b_group_rows, n_tiles, g.ep);
+                             g.m_tok, a_gr, g.b_group_rows, g.b_shared, g.b_kgroup, n_tiles, g.ep);
     return launch_kernel(c->pdl, gemm_simt_kernel<bf16>, grid, dim3(256), 0, s, (const bf16*)g.a,
-                         (const bf16*)g.a2, (const bf16*)g.b, g.n, g.k, g.m_tok, g.b_group_rows,
-                         n_tiles, g.ep);
+                         (const bf16*)g.a2, (const bf16*)g.b, g.n, g.k, g.m_tok, a_gr,
+                         g.b_group_rows, g.b_shared, g.b_kgroup, n_tiles, g.ep);
 }
 
 }  // namespace dfl

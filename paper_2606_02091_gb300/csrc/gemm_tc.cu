@@ -56,6 +56,9 @@ struct TcArgs {
     uint32_t* tile_cnt;
     uint32_t* err;
     EpiParams ep;
+    // activation addressing of the kAux instance only
+    int b_kg;                  // > 0: activation group z holds contraction indices [z b_kg, (z+1) b_kg)
+    int b_gsel;                // 1: activation group = weight group; 0: one activation group for all
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -203,6 +206,11 @@ __device__ __forceinline__ void resid_epilogue(const EpiParams& ep, const float*
         if (c < nvalid) ep.resid[(size_t)(tok0 + c) * ep.ld_resid + n] = r[c] + tile[c * 128 + t];
 }
 
+// kAux = false: the projections of the draft step (every activation group belongs to its weight
+// group; the epilogues without bias). kAux = true adds the activation addressing of the fusion
+// variants (a shared activation group, a contraction across stacked groups) and the biased store;
+// it is a separate instance so that the draft step's code is not touched by it.
+template <bool kAux>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs args) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -294,8 +302,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             int npend = 0;
             bool waited = false;
             auto load_b = [&](uint32_t st, int kx0, int nk, int tok_tile, int group, uint32_t bar) {
-                for (int j = 0; j < nk; ++j)
-                    tma_load_3d(st + b_base + j * G.b_bytes, mB, kx0 + j * kBK, tok_tile * G.bn, group, bar);
+                if constexpr (kAux) {
+                    for (int j = 0; j < nk; ++j) {
+                        int bx = kx0 + j * kBK, bz = group * args.b_gsel;
+                        if (args.b_kg > 0) {   // contraction over stacked activation groups (Eq. 1)
+                            bz = bx / args.b_kg;
+                            bx -= bz * args.b_kg;
+                        }
+                        tma_load_3d(st + b_base + j * G.b_bytes, mB, bx, tok_tile * G.bn, bz, bar);
+                    }
+                } else {
+                    for (int j = 0; j < nk; ++j)
+                        tma_load_3d(st + b_base + j * G.b_bytes, mB, kx0 + j * kBK, tok_tile * G.bn, group, bar);
+                }
             };
             for (int u = blockIdx.x; u < G.n_units && ok; u += gridDim.x) {
                 const Unit x = decode_unit(G, u);
@@ -496,7 +515,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     if (resid)
                         resid_epilogue(args.ep, epi, x.n_tile, x.tok_tile * bn + c0, t, rr);
                     else
-                        apply_epilogue<bf16>(args.ep, epi, x.group, x.n_tile, x.tok_tile * bn + c0, t);
+                        apply_epilogue<bf16, kAux>(args.ep, epi, x.group, x.n_tile, x.tok_tile * bn + c0, t);
                     epi_bar();
                 }
             }
@@ -640,21 +659,35 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     a.tile_cnt = c->tile_cnt;
     a.err = c->err;
     a.ep = g.ep;
-    if (!make_map(&a.map_a, g.a, g.k, g.n, g.groups, g.n, kBM) ||
-        !make_map(&a.map_a2, g.a2 ? g.a2 : g.a, g.k, g.n, g.groups, g.n, kBM) ||
-        !make_map(&a.map_b, g.b, g.k, g.m_tok, g.groups, g.b_group_rows, a.bn)) {
+    // weights: groups of n rows, a_group_rows apart; activations: one group per weight group, one
+    // group shared by all (b_shared), or k / b_kgroup groups that the contraction runs across
+    const long long a_gr = g.a_group_rows > 0 ? g.a_group_rows : g.n;
+    a.b_kg = g.b_kgroup;
+    a.b_gsel = g.b_shared ? 0 : 1;
+    const int b_k = g.b_kgroup > 0 ? g.b_kgroup : g.k;
+    const int b_groups = g.b_kgroup > 0 ? g.k / g.b_kgroup : (g.b_shared ? 1 : g.groups);
+    const long long b_gr = g.b_group_rows > 0 ? g.b_group_rows : g.m_tok;
+    if (g.b_kgroup > 0 && (g.b_kgroup % kBK != 0 || g.k % g.b_kgroup != 0 || g.groups != 1)) {
+        if (why) *why = "tcgen05 GEMM: b_kgroup must be a multiple of 64 that divides k, with one group";
+        return cudaErrorInvalidValue;
+    }
+    if (!make_map(&a.map_a, g.a, g.k, g.n, g.groups, a_gr, kBM) ||
+        !make_map(&a.map_a2, g.a2 ? g.a2 : g.a, g.k, g.n, g.groups, a_gr, kBM) ||
+        !make_map(&a.map_b, g.b, b_k, g.m_tok, b_groups, b_gr, a.bn)) {
         if (why) *why = "cuTensorMapEncodeTiled failed (alignment or driver entry point)";
         return cudaErrorInvalidValue;
     }
-    static int configured = 0;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kSmemLimit);
+    const bool aux = g.b_kgroup > 0 || g.b_shared || g.ep.bias || g.ep.out_gstride;
+    static int configured[2] = {0, 0};
+    if (!configured[aux]) {
+        cudaError_t e = cudaFuncSetAttribute(aux ? gemm_tc_kernel<true> : gemm_tc_kernel<false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
         if (e != cudaSuccess) return e;
-        configured = 1;
+        configured[aux] = 1;
     }
     const int grid = std::min(a.n_units, sms);
-    return launch_kernel(c->pdl, gemm_tc_kernel, dim3(grid), dim3(kThreads), smem, s, a);
+    return launch_kernel(c->pdl, aux ? gemm_tc_kernel<true> : gemm_tc_kernel<false>, dim3(grid),
+                         dim3(kThreads), smem, s, a);
 }
 
 }  // namespace dfl

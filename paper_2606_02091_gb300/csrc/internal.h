@@ -13,7 +13,7 @@ namespace dfl {
 
 // Epilogue kinds of the projection GEMMs (applied to a 128-feature x token tile in fp32).
 enum EpiKind : int {
-    EPI_STORE = 0,      // out[tok][n] = acc                      (storage type)
+    EPI_STORE = 0,      // out[g][tok][n] = acc (+ bias[g][n])    (storage type)
     EPI_F32 = 1,        // out[tok][n] = acc                      (fp32: logits)
     EPI_RESID = 2,      // resid[tok][n] += acc                   (fp32 residual stream)
     EPI_QKV = 3,        // Q / K^d / V^d with rotary embedding on Q and K^d at the block positions
@@ -46,6 +46,8 @@ struct EpiParams {
     const float* rope_cos;   // [positions][hd/2]
     const float* rope_sin;
     int rope;              // apply the rotary embedding (EPI_QKV)
+    long long out_gstride; // EPI_STORE: elements between the groups' outputs
+    const void* bias;      // EPI_STORE: optional [groups][n] storage-type bias added to acc
 };
 
 // One projection GEMM: out = epilogue(B x A^T) per group, where A holds `groups` stacked weight
@@ -58,6 +60,11 @@ struct GemmDesc {
     int groups;
     int n, k, m_tok;
     long long b_group_rows;
+    long long a_group_rows = 0;  // rows between weight groups (0 = n)
+    int b_shared = 0;      // 1: every group reads the same activations (group 0 of b)
+    int b_kgroup = 0;      // > 0 (groups == 1): b holds k / b_kgroup stacked [m_tok][b_kgroup]
+                           // blocks, b_group_rows rows apart, and contraction index kk reads
+                           // block kk / b_kgroup at column kk % b_kgroup
     EpiParams ep;
     int kbs = 0;           // tcgen05 GEMM: 64-wide k-blocks per pipeline stage (0 = default)
     int max_smem = 0;      // tcgen05 GEMM: shared-memory budget per CTA in bytes (0 = default)
@@ -85,6 +92,7 @@ struct dflare_ctx {
     int32_t* app_cnt = nullptr;    // [max_batch]
     float* alpha = nullptr;        // [D][T]
     void* fused = nullptr;         // [D][max_fuse_rows][d]
+    void* fused_fc = nullptr;      // [D][max_fuse_rows][d], DFLARE_FLAG_FUSION_FC only
     float* x = nullptr;            // [max_batch*B][d] residual stream
     void* xn = nullptr;            // [max_batch*B][d] normalised activations
     void* q = nullptr;             // [max_batch*B][d_q]

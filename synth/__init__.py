@@ -17,6 +17,7 @@ from .recipes import (  # noqa: F401
     preset,
     sweep_point,
     weights,
+    variant_weights,
     hidden_states,
     initial_tokens,
     target_draws,

@@ -140,6 +140,21 @@ def weights(w: Workload) -> dict:
     }
 
 
+def variant_weights(w: Workload) -> dict:
+    """Extra weights of the "+FC" ablation and of DFlash's FC fusion, stacked like ``weights``:
+    fusion_fc_w [D][d][d] and dflash_fc_w [d][T d] ~ N(0, (1/sqrt(fan_in))^2) (a unit-scale
+    output for unit-scale inputs), the biases fusion_fc_b [D][d] and dflash_fc_b [d] ~
+    N(0, 0.02^2)."""
+    s = w.shape
+    D, T, d = s.n_draft_layers, s.n_target_layers, s.d
+    return {
+        "fusion_fc_w": _mat(w, "fusion_fc_w", (D, d, d), std=d ** -0.5),
+        "fusion_fc_b": _mat(w, "fusion_fc_b", (D, d)),
+        "dflash_fc_w": _mat(w, "dflash_fc_w", (d, T * d), std=(T * d) ** -0.5),
+        "dflash_fc_b": _mat(w, "dflash_fc_b", (d,)),
+    }
+
+
 def layer_scales(w: Workload) -> np.ndarray:
     """Per-target-layer scale s_j ~ U(0.5, 4) (ones when the workload does not scale)."""
     T = w.shape.n_target_layers

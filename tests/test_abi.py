@@ -52,7 +52,8 @@ def _cfg(**kw):
     ("n_target_layers", 0), ("n_target_layers", 65), ("head_dim", 96), ("n_q_heads", 3),
     ("n_kv_heads", 0), ("ffn", 100), ("vocab", 1), ("mask_token_id", 4096), ("mask_token_id", -1),
     ("block", 0), ("block", 33), ("max_batch", 0), ("max_batch", 65), ("max_ctx", 0),
-    ("max_fuse_rows", 0), ("rms_eps", -1.0), ("rope_theta", 0.0), ("dtype", 2), ("flags", 0x80), ("flags", 0x10),
+    ("max_fuse_rows", 0), ("rms_eps", -1.0), ("rope_theta", 0.0), ("dtype", 2), ("flags", 0x80), ("flags", 0x100),
+    ("flags", 0x40 | 0x2), ("flags", 0x40 | 0x20),   # DFlash FC with -Softmax / +FC
 ])
 def test_create_rejects_bad_config_on_host(lib, field, value):
     ctx = ctypes.c_void_p()
@@ -60,6 +61,19 @@ def test_create_rejects_bad_config_on_host(lib, field, value):
     assert st == 1                                       # DFLARE_EINVAL, no device touched
     assert not ctx
     assert lib.dflare_last_error(None).startswith(b"invalid config")
+
+
+def test_binding_structs_follow_the_header():
+    """The ctypes mirrors of dflare_weights and dflare_config list the header's fields in the
+    header's order, and the flag constants carry the header's values."""
+    from paper_2606_02091_gb300 import _lib
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    for struct, mirror in (("dflare_weights", _lib.Weights), ("dflare_config", _lib.Config)):
+        body = re.search(r"typedef struct \{([^}]*)\}\s*" + struct + ";", src).group(1)
+        fields = re.findall(r"(\w+)\s*;", body)
+        assert fields == [f for f, _ in mirror._fields_], struct
+    flags = dict(re.findall(r"#define DFLARE_FLAG_(\w+)\s+(0x[0-9a-fA-F]+)u", open(HEADER).read()))
+    assert flags and all(getattr(_lib, "FLAG_" + k) == int(v, 16) for k, v in flags.items())
 
 
 def test_create_null_out(lib):

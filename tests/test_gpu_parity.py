@@ -213,3 +213,49 @@ def test_wide_token_tiles_match_oracle(w):
     tok, logits, hidden = g.draft(x_t)
     _check_draft(w, tok, logits, hidden, [o.draft_block(b, int(x_t[b])) for b in range(w.batch)])
     assert g.lib.device_error() == 0
+
+
+# (flag name, oracle options): the Sec. 6.3 ablations and DFlash's FC fusion (Eq. 1, Eq. 2)
+VARIANTS = [
+    ("FLAG_SHARED_KV", dict(shared_kv=True)),
+    ("FLAG_FUSION_FC", dict(fusion_fc=True)),
+    ("FLAG_DFLASH_FC", dict(dflash_fc=True)),
+    ("FLAG_SHARED_KV|FLAG_FUSION_FC", dict(shared_kv=True, fusion_fc=True)),
+]
+
+
+@pytest.mark.parametrize("w", [TINY, SMALL_HD128, WIDE_B16], ids=lambda w: w.name)
+@pytest.mark.parametrize("flags,kw", VARIANTS, ids=[v[0] for v in VARIANTS])
+def test_variant_matches_oracle(w, flags, kw):
+    """Each variant against the oracle: the projected context representation (fused_out), the
+    cached context keys/values of every layer and one drafted block. A second context, filled
+    without fused_out, checks the library's internal buffers."""
+    import paper_2606_02091_gb300 as P
+    flag = 0
+    for f in flags.split("|"):
+        flag |= getattr(P, f)
+    W = dict(synth.weights(w))
+    W.update(synth.variant_weights(w))
+    o = oracle_for(w, W, **kw)
+    F = [o.fuse_context(b, synth.hidden_states(w, b, 0, n)) for b, n in enumerate(w.ctx_lens)]
+    x_t = synth.initial_tokens(w)
+    o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
+    tol = tolerance(w)
+    for want_fused in (True, False):
+        g = GpuRun(w, flags=flag, weights=W)
+        fused = g.fuse(w.ctx_lens, want_fused=want_fused)
+        assert g.lib.ctx_lens() == list(w.ctx_lens)
+        if fused is not None:
+            got = f64(fused)
+            slots = 1 if kw.get("dflash_fc") else w.shape.n_draft_layers
+            for b, n in enumerate(w.ctx_lens):
+                err = rel_err(got[:slots, b, :n], F[b][:slots])
+                assert err <= tol, (b, err)
+        for b, n in enumerate(w.ctx_lens):
+            for i in range(w.shape.n_draft_layers):
+                k, v = g.lib.read_kv(i, b, 0, n)
+                assert rel_err(f64(k), o.ctx_k[b][i]) <= tol, (want_fused, b, i, "K")
+                assert rel_err(f64(v), o.ctx_v[b][i]) <= tol, (want_fused, b, i, "V")
+        tok, logits, hidden = g.draft(x_t)
+        _check_draft(w, tok, logits, hidden, o_res)
+        assert g.lib.device_error() == 0

@@ -164,3 +164,34 @@ def test_round_bf16_truncating(monkeypatch):
         return np.ldexp(np.trunc(np.ldexp(m, 8)), e - 8)
     _patch(monkeypatch, "round_bf16", bad)
     assert _fails(TF.test_round_bf16_matches_torch_cast)
+
+
+def test_dflash_concat_in_reverse_layer_order(monkeypatch):
+    from tests import test_oracle_variants as TW
+
+    def bad(hidden, w_fc, b_fc, store=D.exact):
+        hidden = np.asarray(hidden, float)
+        cat = np.concatenate([hidden[j] for j in reversed(range(hidden.shape[0]))], axis=-1)
+        return store(cat @ np.asarray(w_fc, float).T + b_fc)
+    _patch(monkeypatch, "dflash_context", bad)
+    assert _fails(TW.test_dflash_context_brute_force)
+
+
+def test_dflash_without_bias(monkeypatch):
+    from tests import test_oracle_variants as TW
+
+    def bad(hidden, w_fc, b_fc, store=D.exact):
+        hidden = np.asarray(hidden, float)
+        cat = np.concatenate(list(hidden), axis=-1)
+        return store(cat @ np.asarray(w_fc, float).T)
+    _patch(monkeypatch, "dflash_context", bad)
+    assert _fails(TW.test_dflash_context_one_hot_block_selects_a_layer)
+
+
+def test_fusion_fc_transposed_weight(monkeypatch):
+    from tests import test_oracle_variants as TW
+
+    def bad(F_i, w_fc_i, b_fc_i, store=D.exact):
+        return store(np.asarray(F_i, float) @ np.asarray(w_fc_i, float) + b_fc_i)
+    _patch(monkeypatch, "fusion_fc", bad)
+    assert _fails(TW.test_fusion_fc_brute_force_and_identity)
