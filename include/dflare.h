@@ -203,6 +203,21 @@ dflare_status dflare_verify_accept(dflare_ctx* ctx, const int32_t* draft_tokens_
                                    const int32_t* target_argmax_dev, int32_t* accept_len_dev,
                                    int32_t* next_token_dev, void* stream);
 
+/*
+ * Prefix acceptance from the target's logits (Sec. 3.2, verification phase, with the target's
+ * greedy predictions taken here): g_k = argmax_v target_logits[b][k][v] (lowest id among equal
+ * maxima; NaN entries are never chosen, a row of NaN gives id 0), then exactly
+ * dflare_verify_accept on g.
+ *   draft_tokens_dev     [batch][B-1] int32: d_1 .. d_{B-1}.
+ *   target_logits_dev    [batch][B][V] fp32, 16-byte aligned: the target's logits after block
+ *                        rows 0 .. B-1 (row k predicts position t+k+1).
+ *   accept_len_dev, next_token_dev  as in dflare_verify_accept.
+ * Uses the context's own scratch, so calls on one context must be stream-ordered.
+ */
+dflare_status dflare_verify_logits(dflare_ctx* ctx, const int32_t* draft_tokens_dev,
+                                   const float* target_logits_dev, int32_t* accept_len_dev,
+                                   int32_t* next_token_dev, void* stream);
+
 /* Copy n cached context rows [pos0, pos0+n) of draft layer `layer`, sequence `seq`, into
  * k_out_dev / v_out_dev, each [n][n_kv_heads][head_dim] T (keys already rotated). Either output
  * may be NULL. Rows past the current context hold stale data. */
@@ -220,7 +235,8 @@ dflare_status dflare_device_error(dflare_ctx* ctx, uint32_t* bits_host, void* st
  * (phase 0) and right after (phase 1) the library enqueues each of its kernel launches on
  * `stream` (name: "fuse_begin", "fuse_layers", "gemm_fusion_fc", "gemm_dflash_fc",
  * "gemm_kv_ctx", "embed", "rmsnorm", "gemm_qkv",
- * "attention", "gemm_o", "gemm_gate_up", "gemm_down", "gemm_lm_head", "argmax", "verify").
+ * "attention", "gemm_o", "gemm_gate_up", "gemm_down", "gemm_lm_head", "argmax", "argmax_target",
+ * "verify").
  * A caller can record CUDA events there, also while the stream is being captured into a graph.
  * fn = NULL turns tracing off. */
 typedef void (*dflare_trace_fn)(void* user, const char* name, int phase, void* stream);

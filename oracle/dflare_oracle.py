@@ -20,6 +20,9 @@ and notation (arxiv 2606.02091):
   own predictions, plus one token from the target.
 * Variants measured against DFlare: the ablations of Sec. 6.3 / Table 2 ("-Softmax", "-KVProj",
   "+FC") and DFlash's FC fusion (Eq. 1) with one shared KV projection (Eq. 2).
+* Sampled decoding (Table 1, temperature 1): drafts drawn from softmax(logits / T) and verified
+  by the speculative-sampling rejection rule (the rule is not stated in the paper; see the
+  sampling section below).
 
 Where the paper is silent the oracle takes these readings (each is also listed in the design doc):
 pre-norm residual blocks (RMSNorm -> attention -> residual; RMSNorm -> SwiGLU MLP -> residual)
@@ -266,6 +269,12 @@ def verify_accept(draft, target):
     return a + 1, int(target[a])
 
 
+def verify_from_logits(draft, target_logits):
+    """Verification with the target's greedy predictions taken from its logits (Sec. 3.2):
+    g_k = argmax_v target_logits[k][v] (lowest id among equal maxima), then ``verify_accept``."""
+    return verify_accept(draft, argmax_lowest(target_logits))
+
+
 def synthetic_target(draft, u, r, last, threshold: int):
     """Stand-in for the target's verification argmax (not part of the method).
 
@@ -277,6 +286,115 @@ def synthetic_target(draft, u, r, last, threshold: int):
     r = np.asarray(r, np.int64)
     g = np.where(u < threshold, draft, r + (r >= draft))
     return np.concatenate([g, [int(last)]]).astype(np.int64)
+
+
+# --------------------------------------------------------------------------- sampling (Table 1, temperature 1)
+#
+# Table 1 also reports sampled decoding (temperature 1) without stating its acceptance rule. The
+# oracle takes the rule of the speculative-sampling works the paper builds on: draft token d_k is
+# accepted with probability min(1, p(d_k) / q(d_k)), where p is the target's and q the draft's
+# distribution at that position; at the first rejection the replacement token is drawn from
+# max(0, p - q) renormalised, and when every draft is accepted the extra token is drawn from the
+# target's distribution after the last block row. Draws use the Gumbel-max form
+# argmax_v (log w_v + G_v), G_v = -log(-log u_v), which samples v with probability w_v / sum w.
+#
+# Random numbers: the uniforms of stream (purpose, step, row) are lanes of Philox4x64-10
+# (Salmon, Moraes, Dror, Shaw, SC'11): element v is lane v mod 4 of the block at counter
+# (1 + v div 4, row, step, purpose) under key (seed, 0), mapped to ((x >> 41) + 1/2) 2^-23, a
+# value in (0, 1) that fp32 represents exactly.
+
+RNG_DRAFT, RNG_ACCEPT, RNG_RESIDUAL = 1, 2, 3
+_M64 = (1 << 64) - 1
+PHILOX_MUL = (0xD2E7470EE14C6C93, 0xCA5A826395121157)
+PHILOX_WEYL = (0x9E3779B97F4A7C15, 0xBB67AE8584CAA73B)
+
+
+def philox4x64(counter, key, rounds: int = 10):
+    """One Philox4x64 block from its definition (Python integers): each round multiplies words 0
+    and 2 by the two round multipliers (128-bit products split into high and low halves) and
+    mixes them with words 1 and 3 and the key; the key is advanced by the two Weyl constants
+    between rounds."""
+    c = [int(x) & _M64 for x in counter]
+    k = [int(x) & _M64 for x in key]
+    for r in range(rounds):
+        if r:
+            k = [(k[0] + PHILOX_WEYL[0]) & _M64, (k[1] + PHILOX_WEYL[1]) & _M64]
+        p0 = PHILOX_MUL[0] * c[0]
+        p1 = PHILOX_MUL[1] * c[2]
+        c = [(p1 >> 64) ^ c[1] ^ k[0], p1 & _M64, (p0 >> 64) ^ c[3] ^ k[1], p0 & _M64]
+    return c
+
+
+def uniforms(seed: int, purpose: int, step: int, row: int, n: int):
+    """u_0 .. u_{n-1} of stream (purpose, step, row), float64 values in (0, 1).
+
+    numpy's Philox bit generator computes the same Philox4x64-10 blocks; it advances the counter
+    before its first block, so it starts from word 0 = 0 to produce block 1 first.
+    """
+    u64 = lambda *v: np.array([int(x) & _M64 for x in v], dtype=np.uint64)
+    g = np.random.Philox(counter=u64(0, row, step, purpose), key=u64(seed, 0))
+    x = g.random_raw(int(n)) if n else np.zeros(0, np.uint64)
+    return ((x >> np.uint64(41)).astype(F64) + 0.5) * 2.0 ** -23
+
+
+def softmax_t(logits, temperature: float):
+    """softmax(logits / T) over the last axis (max-subtracted)."""
+    z = np.asarray(logits, F64) / temperature
+    z = np.exp(z - z.max(axis=-1, keepdims=True))
+    return z / z.sum(axis=-1, keepdims=True)
+
+
+def gumbel_draw(log_w, u):
+    """argmax_v (log_w[v] - log(-log u[v])): a draw of v with probability proportional to
+    exp(log_w[v]); entries with log_w = -inf are never drawn (lowest id among equal scores)."""
+    score = np.asarray(log_w, F64) - np.log(-np.log(np.asarray(u, F64)))
+    return int(np.argmax(score))
+
+
+def sample_token(logits, temperature: float, u):
+    """A draft token at temperature T: a draw from softmax(logits / T)."""
+    return gumbel_draw(np.asarray(logits, F64) / temperature, u)
+
+
+def accept_prob(p, q, d: int):
+    """min(1, p(d) / q(d)): the probability of keeping draft token d."""
+    return min(1.0, float(p[d]) / float(q[d]))
+
+
+def residual_dist(p, q):
+    """max(0, p - q) renormalised, the replacement distribution after a rejection (p itself when
+    the difference vanishes everywhere)."""
+    w = np.maximum(np.asarray(p, F64) - np.asarray(q, F64), 0.0)
+    tot = w.sum()
+    return w / tot if tot > 0 else np.asarray(p, F64)
+
+
+def speculative_verify(draft, target_logits, draft_logits, temperature: float, r, u_res):
+    """Sampled verification of one block.
+
+    draft: d_1 .. d_{B-1}; target_logits: [B][V], row k-1 predicts the position of d_k (row B-1
+    the position after the block); draft_logits: [B-1][V], the draft's logits at the position of
+    d_k; r: B-1 acceptance uniforms; u_res: V uniforms for the replacement or extra token.
+    d_k is kept when r_k q(d_k) < p(d_k), i.e. r_k < p(d_k)/q(d_k). Returns (tau, next_token).
+    """
+    target_logits = np.asarray(target_logits, F64)
+    B = target_logits.shape[0]
+    a = 0
+    while a < B - 1:
+        p = softmax_t(target_logits[a], temperature)
+        q = softmax_t(draft_logits[a], temperature)
+        d = int(draft[a])
+        if r[a] * q[d] < p[d]:
+            a += 1
+        else:
+            break
+    if a < B - 1:
+        w = residual_dist(softmax_t(target_logits[a], temperature),
+                          softmax_t(draft_logits[a], temperature))
+    else:
+        w = softmax_t(target_logits[B - 1], temperature)
+    with np.errstate(divide="ignore"):
+        return a + 1, gumbel_draw(np.log(w), u_res)
 
 
 # --------------------------------------------------------------------------- the whole path

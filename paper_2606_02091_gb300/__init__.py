@@ -136,6 +136,17 @@ class DFlare:
                                                  _ptr(accept_len), _ptr(next_token),
                                                  _stream(stream)))
 
+    def verify_logits(self, draft_tokens, target_logits, accept_len, next_token, stream=None):
+        """target_logits [batch][B][V] fp32: the target's argmax is taken on the device."""
+        import torch
+        _need_cuda("target_logits", target_logits, torch.float32)
+        for n, t in (("draft_tokens", draft_tokens), ("accept_len", accept_len),
+                     ("next_token", next_token)):
+            _need_cuda(n, t, torch.int32)
+        self._check(self._L.dflare_verify_logits(self._ctx, _ptr(draft_tokens), _ptr(target_logits),
+                                                 _ptr(accept_len), _ptr(next_token),
+                                                 _stream(stream)))
+
     def read_kv(self, layer, seq, pos0, n, stream=None):
         import torch
         dt = torch.bfloat16 if self.dtype == "bf16" else torch.float32

@@ -57,7 +57,8 @@ __device__ __forceinline__ uint32_t order_key(float v) {
 
 // Grid (chunks, rows): each CTA reduces one vocabulary chunk of one row (lowest index among
 // equal maxima) and folds (ordered value, ~index) into the row's slot with a 64-bit atomicMax;
-// the last CTA to arrive writes the token ids.
+// the last CTA to arrive writes the token ids. NaN entries are never chosen; a row with no value
+// above -inf gets its first -inf entry (id 0 when every entry is NaN).
 __global__ void __launch_bounds__(256) argmax_noalloc_kernel(const float* __restrict__ logits,
                                                              int V, int rows, int chunk,
                                                              unsigned long long* slot,
@@ -95,8 +96,17 @@ __global__ void __launch_bounds__(256) argmax_noalloc_kernel(const float* __rest
     __syncthreads();
     if (last) {
         __threadfence();
-        for (int r = threadIdx.x; r < rows; r += blockDim.x)
-            tokens[r] = (int32_t)(0xFFFFFFFFu - (uint32_t)(atomicAdd(&slot[r], 0ull) & 0xFFFFFFFFull));
+        for (int r = threadIdx.x; r < rows; r += blockDim.x) {
+            const unsigned long long key = atomicAdd(&slot[r], 0ull);
+            int32_t tok = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+            if (key == 0ull) {   // no entry above -inf: a serial scan, only for such rows
+                const float* pr = logits + (size_t)r * V;
+                tok = 0;
+                for (int i = 0; i < V; ++i)
+                    if (pr[i] == -INFINITY) { tok = i; break; }
+            }
+            tokens[r] = tok;
+        }
     }
 }
 

@@ -224,7 +224,8 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     ALLOC(c->attn_ml, part_rows * 2 * sizeof(float));
     ALLOC(c->ws, c->ws_floats * sizeof(float));
     ALLOC(c->tile_cnt, (size_t)c->tile_cnt_n * sizeof(uint32_t));
-    ALLOC(c->amax_slot, mrows * sizeof(unsigned long long));
+    ALLOC(c->amax_slot, rows * sizeof(unsigned long long));
+    ALLOC(c->tgt_tok, rows * sizeof(int32_t));
     ALLOC(c->amax_cnt, sizeof(uint32_t));
     const size_t half = g.head_dim / 2, npos = (size_t)g.max_ctx + B;
     ALLOC(c->rope_cos, npos * half * sizeof(float));
@@ -235,7 +236,7 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     struct Z { void* p; size_t n; } zs[] = {
         {c->ctx_len, g.max_batch * sizeof(int32_t)}, {c->app_base, g.max_batch * sizeof(int32_t)},
         {c->app_cnt, g.max_batch * sizeof(int32_t)}, {c->tile_cnt, (size_t)c->tile_cnt_n * 4},
-        {c->amax_slot, mrows * 8}, {c->amax_cnt, 4}, {c->err, 4},
+        {c->amax_slot, rows * 8}, {c->amax_cnt, 4}, {c->err, 4},
         {c->fused, D * (size_t)g.max_fuse_rows * d * esz}, {c->x, rows * d * 4}};
     for (auto& z : zs) {
         e = cudaMemset(z.p, 0, z.n);
@@ -547,7 +548,7 @@ dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32
     if (st != DFLARE_OK) return st;
     {
         Trace t(c, "argmax", s);
-        CUDA_TRY(launch_argmax(c, mrows, draft_tokens, s));
+        CUDA_TRY(launch_argmax(c, c->logits, mrows, draft_tokens, s));
     }
     if (logits_out)
         CUDA_TRY(cudaMemcpyAsync(logits_out, c->logits, (size_t)mrows * g.vocab * 4,
@@ -563,6 +564,23 @@ dflare_status dflare_verify_accept(dflare_ctx* c, const int32_t* draft, const in
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     Trace t(c, "verify", s);
     CUDA_TRY(launch_verify(c, draft, target, accept_len, next_token, s));
+    return DFLARE_OK;
+}
+
+dflare_status dflare_verify_logits(dflare_ctx* c, const int32_t* draft, const float* target_logits,
+                                   int32_t* accept_len, int32_t* next_token, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!target_logits || !accept_len || !next_token || (!draft && c->cfg.block > 1))
+        return fail(c, DFLARE_EINVAL, "a verification buffer is NULL");
+    if (reinterpret_cast<uintptr_t>(target_logits) % 16)
+        return fail(c, DFLARE_EINVAL, "target_logits must be 16-byte aligned");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    {
+        Trace t(c, "argmax_target", s);
+        CUDA_TRY(launch_argmax(c, target_logits, c->batch * c->cfg.block, c->tgt_tok, s));
+    }
+    Trace t(c, "verify", s);
+    CUDA_TRY(launch_verify(c, draft, c->tgt_tok, accept_len, next_token, s));
     return DFLARE_OK;
 }
 

@@ -111,7 +111,8 @@ struct dflare_ctx {
     size_t ws_floats = 0;
     uint32_t* tile_cnt = nullptr;  // split-K arrival counters
     int tile_cnt_n = 0;
-    unsigned long long* amax_slot = nullptr;  // packed (value, index) per logits row
+    unsigned long long* amax_slot = nullptr;  // packed (value, index) per logits row [max_batch*B]
+    int32_t* tgt_tok = nullptr;    // [max_batch*B] target argmax of dflare_verify_logits
     uint32_t* amax_cnt = nullptr;
     float* rope_cos = nullptr;     // [max_ctx + B][hd/2]
     float* rope_sin = nullptr;
@@ -181,7 +182,8 @@ cudaError_t launch_embed(dflare_ctx* c, const int32_t* last_token, cudaStream_t 
 cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gather_mask_rows,
                            void* out, cudaStream_t s);
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s);
-cudaError_t launch_argmax(dflare_ctx* c, int rows, int32_t* tokens, cudaStream_t s);
+cudaError_t launch_argmax(dflare_ctx* c, const float* logits, int rows, int32_t* tokens,
+                          cudaStream_t s);
 cudaError_t launch_verify(dflare_ctx* c, const int32_t* draft, const int32_t* target,
                           int32_t* accept_len, int32_t* next_token, cudaStream_t s);
 cudaError_t launch_synthetic_target(const int32_t* draft, const uint32_t* u, const int32_t* r,

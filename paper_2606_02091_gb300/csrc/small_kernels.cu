@@ -89,7 +89,9 @@ __device__ __forceinline__ uint32_t ordered_key(float v) {
 // Greedy argmax over the vocabulary (lowest id among equal maxima). Grid (chunks, rows): each
 // CTA reduces a chunk of one row with warp shuffles and publishes (key(value), ~index) through a
 // 64-bit atomicMax; the last CTA to finish turns the packed maxima into token ids and re-arms
-// the slots and the counter for the next launch.
+// the slots and the counter for the next launch. NaN entries are never chosen. A row without a
+// value above -inf publishes nothing; the last CTA then takes its first -inf entry (the lowest
+// id among equal maxima), or id 0 when every entry is NaN.
 __global__ void __launch_bounds__(256) argmax_kernel(const float* __restrict__ logits, int V,
                                                      int rows, int chunk,
                                                      unsigned long long* slot, uint32_t* cnt,
@@ -144,7 +146,14 @@ __global__ void __launch_bounds__(256) argmax_kernel(const float* __restrict__ l
         __threadfence();
         for (int r = threadIdx.x; r < rows; r += blockDim.x) {
             const unsigned long long key = atomicExch(&slot[r], 0ull);
-            tokens[r] = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+            int32_t tok = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+            if (key == 0ull) {   // no entry above -inf: a serial scan, only for such rows
+                const float* pr = logits + (size_t)r * V;
+                tok = 0;
+                for (int i = 0; i < V; ++i)
+                    if (pr[i] == -INFINITY) { tok = i; break; }
+            }
+            tokens[r] = tok;
         }
         if (threadIdx.x == 0) *cnt = 0;
     }
@@ -219,7 +228,8 @@ cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gathe
                          (const bf16*)gain, (bf16*)out, g.d, g.block, gather ? 1 : 0, g.rms_eps);
 }
 
-cudaError_t launch_argmax(dflare_ctx* c, int rows, int32_t* tokens, cudaStream_t s) {
+cudaError_t launch_argmax(dflare_ctx* c, const float* logits, int rows, int32_t* tokens,
+                          cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     const int V = c->cfg.vocab;
     // enough CTAs to fill the GPU: chunks of at least 4096 ids, a multiple of 1024
@@ -227,7 +237,7 @@ cudaError_t launch_argmax(dflare_ctx* c, int rows, int32_t* tokens, cudaStream_t
     int chunk = (V + chunks - 1) / chunks;
     chunk = std::max(4096, ((chunk + 1023) / 1024) * 1024);
     chunks = (V + chunk - 1) / chunk;
-    return launch_kernel(c->pdl, argmax_kernel, dim3(chunks, rows), dim3(256), 0, s, c->logits, V,
+    return launch_kernel(c->pdl, argmax_kernel, dim3(chunks, rows), dim3(256), 0, s, logits, V,
                          rows, chunk, c->amax_slot, c->amax_cnt, tokens);
 }
 

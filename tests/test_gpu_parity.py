@@ -259,3 +259,35 @@ def test_variant_matches_oracle(w, flags, kw):
         tok, logits, hidden = g.draft(x_t)
         _check_draft(w, tok, logits, hidden, o_res)
         assert g.lib.device_error() == 0
+
+
+@pytest.mark.parametrize("w", [TINY, SMALL_HD128, WIDE_B16], ids=lambda w: w.name)
+def test_verify_from_logits_matches_oracle(w):
+    """dflare_verify_logits against the oracle: the target's argmax taken from [batch][B][V]
+    logits, then prefix acceptance. Rows planted to agree with a random prefix of the drafts,
+    ties between two maxima in different vocabulary chunks, and rows of only -inf (lowest id);
+    integer results bit-exact, over several rounds on one context."""
+    import torch
+    s = w.shape
+    g = GpuRun(w)
+    rng = np.random.default_rng(21)
+    B, V, bsz = s.block, s.vocab, w.batch
+    for rnd in range(4):
+        draft = rng.integers(0, V, (bsz, B - 1)).astype(np.int32)
+        lg = rng.standard_normal((bsz, B, V)).astype(np.float32)
+        for b in range(bsz):
+            a = int(rng.integers(0, B))              # planted prefix length
+            for k in range(a):
+                lg[b, k, draft[b, k]] = 20.0
+            if rnd == 1 and B > 2:                    # a tie: lowest id wins
+                lo, hi = sorted(rng.choice(V, 2, replace=False))
+                lg[b, B - 1, lo] = lg[b, B - 1, hi] = 30.0
+            if rnd == 2:
+                lg[b, int(rng.integers(0, B))] = -np.inf
+        acc = torch.zeros(bsz, dtype=torch.int32, device="cuda")
+        nxt = torch.zeros(bsz, dtype=torch.int32, device="cuda")
+        g.lib.verify_logits(torch.from_numpy(draft).cuda(), torch.from_numpy(lg).cuda(), acc, nxt)
+        got = list(zip(acc.cpu().tolist(), nxt.cpu().tolist()))
+        want = [O.verify_from_logits(draft[b], lg[b]) for b in range(bsz)]
+        assert got == want, (rnd, got, want)
+    assert g.lib.device_error() == 0

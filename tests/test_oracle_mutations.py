@@ -195,3 +195,40 @@ def test_fusion_fc_transposed_weight(monkeypatch):
         return store(np.asarray(F_i, float) @ np.asarray(w_fc_i, float) + b_fc_i)
     _patch(monkeypatch, "fusion_fc", bad)
     assert _fails(TW.test_fusion_fc_brute_force_and_identity)
+
+
+def test_acceptance_ratio_inverted(monkeypatch):
+    from tests import test_oracle_sampling as TS
+    _patch(monkeypatch, "accept_prob", lambda p, q, d: min(1.0, float(q[d]) / float(p[d])))
+    assert _fails(TS.test_speculative_rule_preserves_the_target_distribution_closed_form)
+
+
+def test_residual_without_clipping(monkeypatch):
+    from tests import test_oracle_sampling as TS
+
+    def bad(p, q):
+        w = np.abs(np.asarray(p, float) - np.asarray(q, float))
+        return w / w.sum()
+    _patch(monkeypatch, "residual_dist", bad)
+    assert _fails(TS.test_speculative_rule_preserves_the_target_distribution_closed_form)
+
+
+def test_replacement_drawn_from_target_instead_of_residual(monkeypatch):
+    """A verification that redraws from p (not max(0, p - q)) after a rejection over-weights the
+    tokens the draft already proposes."""
+    from tests import test_oracle_sampling as TS
+    orig_res = D.residual_dist
+    _patch(monkeypatch, "residual_dist", lambda p, q: np.asarray(p, float))
+    assert _fails(lambda: TS.test_speculative_verify_first_token_is_target_distributed(2))
+    _patch(monkeypatch, "residual_dist", orig_res)
+
+
+def test_philox_words_swapped(monkeypatch):
+    from tests import test_oracle_sampling as TS
+    orig = D.philox4x64
+
+    def bad(counter, key, rounds=10):
+        c = orig(counter, key, rounds)
+        return [c[1], c[0], c[2], c[3]]
+    _patch(monkeypatch, "philox4x64", bad)
+    assert _fails(lambda: TS.test_uniform_stream_is_philox4x64_10(7, 2, 3, 11))

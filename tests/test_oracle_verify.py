@@ -63,3 +63,20 @@ def test_expected_accept_length(p, B):
     sd = taus.std() / np.sqrt(n)
     assert abs(taus.mean() - mean) < 4 * sd, (taus.mean(), mean, sd)
     assert taus.min() >= 1 and taus.max() <= B
+
+
+def test_verify_from_logits_equals_verify_on_planted_maxima():
+    """One planted maximum per row makes the logits route equal verify_accept on those tokens;
+    a tie between two planted maxima goes to the lower id."""
+    rng = np.random.default_rng(9)
+    B, V = 6, 40
+    for trial in range(200):
+        draft = rng.integers(0, V, B - 1)
+        g = rng.integers(0, V, B)
+        lg = rng.standard_normal((B, V))
+        lg[np.arange(B), g] = 10.0
+        assert O.verify_from_logits(draft, lg) == O.verify_accept(draft, g)
+    lg = np.zeros((B, V))
+    lg[:, 7] = lg[:, 3] = 1.0
+    assert O.verify_from_logits([3] * (B - 1), lg) == (B, 3)
+    assert O.verify_from_logits([7] * (B - 1), lg) == (1, 3)

@@ -41,3 +41,24 @@ def test_noalloc_argmax_matches_draft_block_on_two_calls():
         argmax_noalloc(dev, out)
         torch.cuda.synchronize()
         np.testing.assert_array_equal(out.cpu().numpy(), tok)
+
+
+@pytest.mark.gpu
+def test_noalloc_argmax_rows_without_a_finite_maximum():
+    """NaN entries are never chosen; a row with nothing above -inf gets its first -inf entry, a
+    row of NaN id 0; ties go to the lowest id."""
+    import torch
+    from paper_2606_02091_gb300 import argmax_noalloc
+    V = 5000
+    lg = np.random.default_rng(1).standard_normal((5, V)).astype(np.float32)
+    lg[0] = -np.inf
+    lg[1] = -np.inf
+    lg[1, :3] = np.nan
+    lg[2] = np.nan
+    lg[3, 17] = lg[3, 4096] = 50.0
+    lg[4, V - 1] = 50.0
+    lg[4, 5] = np.nan
+    dev = torch.from_numpy(lg).cuda()
+    out = torch.full((5,), -1, dtype=torch.int32, device="cuda")
+    argmax_noalloc(dev, out)
+    assert out.cpu().tolist() == [0, 3, 0, 17, V - 1]
