@@ -363,6 +363,68 @@ def fusion_variants(w, dev_w, fill_chunks, hid_step, n_step, reps=100):
     return out
 
 
+def sampled_steps(w, dev_w, fill_chunks, hid_step, x0, reps=100, temperature=1.0, seed=2024):
+    """Block steps at temperature 1 (Table 1's sampled rows): fuse the previous step's tau
+    positions, draft with dflare_draft_block_sampled, verify with dflare_verify_sampled against
+    fixed synthetic target logits ([batch][B][V] N(0, 1), resident in HBM), in a CUDA graph of one
+    step replayed `reps` times between events, on a context filled like the main run."""
+    import torch
+    from paper_2606_02091_gb300 import DFlare
+    s = w.shape
+    fill_rows = max(Ht.shape[2] for Ht, _ in fill_chunks)
+    lib = DFlare.from_shape(s, max_batch=w.batch, max_ctx=max(w.ctx_lens) + s.block * (reps + 8),
+                            max_fuse_rows=w.batch * max(fill_rows, s.block))
+    lib.set_weights(dev_w)
+    lib.reset(w.batch)
+    for Ht, nt in fill_chunks:
+        lib.fuse_context(Ht, nt)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    tgt = torch.randn((w.batch, s.block, s.vocab), generator=g, device="cuda")
+    step_ctr = torch.zeros(1, dtype=torch.int64, device="cuda")
+    acc = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
+    nxt = x0.clone()
+    draft = torch.zeros((w.batch, s.block - 1), dtype=torch.int32, device="cuda")
+
+    def step():
+        lib.fuse_context(hid_step, acc)
+        lib.draft_block_sampled(nxt, temperature, seed, step_ctr, draft)
+        lib.verify_sampled(draft, tgt, temperature, seed, step_ctr, acc, nxt)
+
+    cs = torch.cuda.Stream()
+    cs.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(cs):
+        step()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph, stream=cs):
+            step()
+    torch.cuda.synchronize()
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    lens0 = lib.ctx_lens()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    lens1 = lib.ctx_lens()
+    if lib.device_error():
+        raise RuntimeError("device error in the sampled steps")
+    out = {"ms_per_step": ms, "drafted_tokens_per_s": w.batch * (s.block - 1) / (ms / 1e3),
+           "mean_accept_len": (sum(lens1) - sum(lens0)) / (reps * w.batch),
+           "temperature": temperature, "steps": reps, "rng_steps": int(step_ctr.item()),
+           "note": "CUDA graph of one step (fuse tau positions, sampled draft, speculative-sampling "
+                   "verification); target logits are fixed N(0, 1) draws, so tau reflects an "
+                   "unrelated target, not a trained pair"}
+    del graph
+    lib.close()
+    return out
+
+
 def replica_aggregate(ms, units_per_step, steps, dist=None, device="cuda"):
     """Weak-scaling aggregate of independent replicas (one per rank, no data-path exchange):
     the job's time is the slowest rank's, its throughput every rank's units over that time.
@@ -672,6 +734,8 @@ def run_ours(args):
     if not args.no_variants:
         line["fusion_variants"] = fusion_variants(w, dev_w, fill_chunks, hid_step,
                                                   max(1, int(round(mean_tau))))
+        line["sampled"] = sampled_steps(w, dev_w, fill_chunks, hid_step,
+                                        torch.from_numpy(synth.initial_tokens(w)).cuda())
     del fill_chunks
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, dt, tau = oracle_steps(w, W, args.cpu_steps)

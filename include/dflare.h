@@ -218,6 +218,45 @@ dflare_status dflare_verify_logits(dflare_ctx* ctx, const int32_t* draft_tokens_
                                    const float* target_logits_dev, int32_t* accept_len_dev,
                                    int32_t* next_token_dev, void* stream);
 
+/*
+ * Sampled decoding at temperature T (Table 1's temperature-1 rows). The paper does not state its
+ * acceptance rule for sampling; these calls use the speculative-sampling rule of the works it
+ * builds on. Random numbers are Philox4x64-10 streams (Salmon et al., SC'11): element v of
+ * stream (purpose, step, row) is lane v mod 4 of the block at counter (1 + v/4, row, step,
+ * purpose), key (seed, 0), mapped to ((x >> 41) + 1/2) * 2^-23. Purposes: 1 draft draws (row =
+ * b*(B-1) + k-1, v = token id), 2 acceptance draws (row = b, v = k-1), 3 replacement draws
+ * (row = b, v = token id). `step_dev` is a uint64 device counter read by both calls;
+ * dflare_verify_sampled adds 1 to it when it finishes, so a captured draft-verify graph draws
+ * fresh numbers on every replay.
+ *
+ * dflare_draft_block_sampled: dflare_draft_block with d_k drawn from softmax(logits_k / T)
+ * (Gumbel-max: argmax_v l_v / T - log(-log u_v), lowest id among equal scores) instead of the
+ * argmax. temperature must be finite and > 0 (DFLARE_EINVAL otherwise).
+ */
+dflare_status dflare_draft_block_sampled(dflare_ctx* ctx, const int32_t* last_token_dev,
+                                         float temperature, uint64_t seed,
+                                         const uint64_t* step_dev, int32_t* draft_tokens_dev,
+                                         float* logits_out_dev, float* hidden_out_dev,
+                                         void* stream);
+
+/*
+ * dflare_verify_sampled: speculative-sampling verification of the block the last
+ * dflare_draft_block[_sampled] on this context drafted (its logits are kept in the context).
+ * With p_k = softmax(target_logits[b][k-1] / T) and q_k = softmax(draft logits of d_k / T),
+ * d_k is kept when r_k * q_k(d_k) < p_k(d_k) (r_k the acceptance draw); a = the number of kept
+ * drafts before the first rejection; accept_len = a + 1. next_token is drawn from
+ * max(0, p_{a+1} - q_{a+1}) when a < B-1 (from p_{a+1} if that vanishes everywhere), else from
+ * softmax(target_logits[b][B-1] / T).
+ *   draft_tokens_dev   [batch][B-1] int32 (an id outside [0, V) is rejected and sets
+ *                      DFLARE_DEVERR_TOKEN).
+ *   target_logits_dev  [batch][B][V] fp32, 16-byte aligned.
+ *   step_dev           the counter described above (incremented on the device).
+ */
+dflare_status dflare_verify_sampled(dflare_ctx* ctx, const int32_t* draft_tokens_dev,
+                                    const float* target_logits_dev, float temperature,
+                                    uint64_t seed, uint64_t* step_dev, int32_t* accept_len_dev,
+                                    int32_t* next_token_dev, void* stream);
+
 /* Copy n cached context rows [pos0, pos0+n) of draft layer `layer`, sequence `seq`, into
  * k_out_dev / v_out_dev, each [n][n_kv_heads][head_dim] T (keys already rotated). Either output
  * may be NULL. Rows past the current context hold stale data. */
@@ -235,8 +274,8 @@ dflare_status dflare_device_error(dflare_ctx* ctx, uint32_t* bits_host, void* st
  * (phase 0) and right after (phase 1) the library enqueues each of its kernel launches on
  * `stream` (name: "fuse_begin", "fuse_layers", "gemm_fusion_fc", "gemm_dflash_fc",
  * "gemm_kv_ctx", "embed", "rmsnorm", "gemm_qkv",
- * "attention", "gemm_o", "gemm_gate_up", "gemm_down", "gemm_lm_head", "argmax", "argmax_target",
- * "verify").
+ * "attention", "gemm_o", "gemm_gate_up", "gemm_down", "gemm_lm_head", "argmax", "sample",
+ * "argmax_target", "verify", "spec_stats", "spec_accept", "spec_resample").
  * A caller can record CUDA events there, also while the stream is being captured into a graph.
  * fn = NULL turns tracing off. */
 typedef void (*dflare_trace_fn)(void* user, const char* name, int phase, void* stream);

@@ -136,6 +136,34 @@ class DFlare:
                                                  _ptr(accept_len), _ptr(next_token),
                                                  _stream(stream)))
 
+    def draft_block_sampled(self, last_token, temperature, seed, step, draft_tokens,
+                            logits_out=None, hidden_out=None, stream=None):
+        """As draft_block, with tokens drawn at `temperature`; step: uint64 device counter
+        (a one-element int64 tensor)."""
+        import torch
+        _need_cuda("last_token", last_token, torch.int32)
+        _need_cuda("draft_tokens", draft_tokens, torch.int32)
+        _need_cuda("step", step, torch.int64)
+        _need_cuda("logits_out", logits_out, torch.float32)
+        _need_cuda("hidden_out", hidden_out, torch.float32)
+        self._check(self._L.dflare_draft_block_sampled(
+            self._ctx, _ptr(last_token), float(temperature), int(seed) & (2 ** 64 - 1), _ptr(step),
+            _ptr(draft_tokens), _ptr(logits_out), _ptr(hidden_out), _stream(stream)))
+
+    def verify_sampled(self, draft_tokens, target_logits, temperature, seed, step, accept_len,
+                       next_token, stream=None):
+        """Speculative-sampling verification of the last drafted block; advances step by one."""
+        import torch
+        _need_cuda("target_logits", target_logits, torch.float32)
+        _need_cuda("step", step, torch.int64)
+        for n, t in (("draft_tokens", draft_tokens), ("accept_len", accept_len),
+                     ("next_token", next_token)):
+            _need_cuda(n, t, torch.int32)
+        self._check(self._L.dflare_verify_sampled(
+            self._ctx, _ptr(draft_tokens), _ptr(target_logits), float(temperature),
+            int(seed) & (2 ** 64 - 1), _ptr(step), _ptr(accept_len), _ptr(next_token),
+            _stream(stream)))
+
     def verify_logits(self, draft_tokens, target_logits, accept_len, next_token, stream=None):
         """target_logits [batch][B][V] fp32: the target's argmax is taken on the device."""
         import torch

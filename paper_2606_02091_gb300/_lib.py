@@ -31,7 +31,8 @@ STATUS_NAMES = {0: "DFLARE_OK", 1: "DFLARE_EINVAL", 2: "DFLARE_ECAPACITY", 3: "D
 # every entry point include/dflare.h declares
 EXPORTS = ("dflare_create", "dflare_destroy", "dflare_set_weights", "dflare_reset",
            "dflare_fuse_context", "dflare_draft_block", "dflare_verify_accept",
-           "dflare_verify_logits", "dflare_read_kv",
+           "dflare_verify_logits", "dflare_draft_block_sampled", "dflare_verify_sampled",
+           "dflare_read_kv",
            "dflare_ctx_lens", "dflare_device_error", "dflare_last_error",
            "dflare_synthetic_target", "dflare_set_trace", "dflare_argmax_noalloc")
 
@@ -87,6 +88,8 @@ def load():
         "dflare_draft_block": [vp, vp, vp, vp, vp, vp],
         "dflare_verify_accept": [vp, vp, vp, vp, vp, vp],
         "dflare_verify_logits": [vp, vp, vp, vp, vp, vp],
+        "dflare_draft_block_sampled": [vp, vp, ctypes.c_float, ctypes.c_uint64, vp, vp, vp, vp, vp],
+        "dflare_verify_sampled": [vp, vp, vp, ctypes.c_float, ctypes.c_uint64, vp, vp, vp, vp],
         "dflare_read_kv": [vp, i32, i32, i32, i32, vp, vp, vp],
         "dflare_ctx_lens": [vp, vp, vp],
         "dflare_device_error": [vp, P(u32), vp],

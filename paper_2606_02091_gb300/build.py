@@ -13,7 +13,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdflare.so")
 SOURCES = ["dflare_api.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "fuse.cu",
-           "small_kernels.cu", "argmax_noalloc.cu"]
+           "small_kernels.cu", "argmax_noalloc.cu", "sampling.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 

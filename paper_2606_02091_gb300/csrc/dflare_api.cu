@@ -4,6 +4,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <string>
@@ -226,6 +227,8 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     ALLOC(c->tile_cnt, (size_t)c->tile_cnt_n * sizeof(uint32_t));
     ALLOC(c->amax_slot, rows * sizeof(unsigned long long));
     ALLOC(c->tgt_tok, rows * sizeof(int32_t));
+    ALLOC(c->spec_part, (size_t)g.max_batch * (2 * B - 1) * kSpecMaxChunks * sizeof(float2));
+    ALLOC(c->spec_a, g.max_batch * sizeof(int32_t));
     ALLOC(c->amax_cnt, sizeof(uint32_t));
     const size_t half = g.head_dim / 2, npos = (size_t)g.max_ctx + B;
     ALLOC(c->rope_cos, npos * half * sizeof(float));
@@ -420,8 +423,20 @@ dflare_status dflare_fuse_context(dflare_ctx* c, const void* hidden, const int32
     return traced_gemm(c, "gemm_kv_ctx", gd, s);
 }
 
-dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32_t* draft_tokens,
-                                 float* logits_out, float* hidden_out, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Sampling parameters of dflare_draft_block_sampled (null: greedy).
+struct Sampling {
+    float inv_t;
+    uint64_t seed;
+    const uint64_t* step;
+};
+
+dflare_status draft_block_impl(dflare_ctx* c, const int32_t* last_token, int32_t* draft_tokens,
+                               float* logits_out, float* hidden_out, void* stream,
+                               const Sampling* smp) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
     if (!c->weights_set) return fail(c, DFLARE_ESTATE, "dflare_set_weights has not been called");
     if (!last_token || !draft_tokens) return fail(c, DFLARE_EINVAL, "last_token or draft_tokens is NULL");
@@ -546,7 +561,10 @@ dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32
     h.ep.ldo = g.vocab;
     dflare_status st = traced_gemm(c, "gemm_lm_head", h, s);
     if (st != DFLARE_OK) return st;
-    {
+    if (smp) {
+        Trace t(c, "sample", s);
+        CUDA_TRY(launch_sample(c, mrows, smp->inv_t, smp->seed, smp->step, draft_tokens, s));
+    } else {
         Trace t(c, "argmax", s);
         CUDA_TRY(launch_argmax(c, c->logits, mrows, draft_tokens, s));
     }
@@ -554,6 +572,27 @@ dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32
         CUDA_TRY(cudaMemcpyAsync(logits_out, c->logits, (size_t)mrows * g.vocab * 4,
                                  cudaMemcpyDeviceToDevice, s));
     return DFLARE_OK;
+}
+
+bool bad_temperature(float t) { return !(t > 0.f) || !std::isfinite(t) || !std::isfinite(1.0f / t); }
+
+}  // namespace
+
+extern "C" {
+
+dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32_t* draft_tokens,
+                                 float* logits_out, float* hidden_out, void* stream) {
+    return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, nullptr);
+}
+
+dflare_status dflare_draft_block_sampled(dflare_ctx* c, const int32_t* last_token, float temperature,
+                                         uint64_t seed, const uint64_t* step, int32_t* draft_tokens,
+                                         float* logits_out, float* hidden_out, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (bad_temperature(temperature)) return fail(c, DFLARE_EINVAL, "temperature must be finite and > 0");
+    if (!step) return fail(c, DFLARE_EINVAL, "step is NULL");
+    const Sampling smp{1.0f / temperature, seed, step};
+    return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, &smp);
 }
 
 dflare_status dflare_verify_accept(dflare_ctx* c, const int32_t* draft, const int32_t* target,
@@ -581,6 +620,30 @@ dflare_status dflare_verify_logits(dflare_ctx* c, const int32_t* draft, const fl
     }
     Trace t(c, "verify", s);
     CUDA_TRY(launch_verify(c, draft, c->tgt_tok, accept_len, next_token, s));
+    return DFLARE_OK;
+}
+
+dflare_status dflare_verify_sampled(dflare_ctx* c, const int32_t* draft, const float* target_logits,
+                                    float temperature, uint64_t seed, uint64_t* step,
+                                    int32_t* accept_len, int32_t* next_token, void* stream) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (!target_logits || !accept_len || !next_token || !step || (!draft && c->cfg.block > 1))
+        return fail(c, DFLARE_EINVAL, "a verification buffer is NULL");
+    if (bad_temperature(temperature)) return fail(c, DFLARE_EINVAL, "temperature must be finite and > 0");
+    if (reinterpret_cast<uintptr_t>(target_logits) % 16)
+        return fail(c, DFLARE_EINVAL, "target_logits must be 16-byte aligned");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const float inv_t = 1.0f / temperature;
+    {
+        Trace t(c, "spec_stats", s);
+        CUDA_TRY(launch_spec_stats(c, target_logits, inv_t, s));
+    }
+    {
+        Trace t(c, "spec_accept", s);
+        CUDA_TRY(launch_spec_accept(c, draft, target_logits, inv_t, seed, step, s));
+    }
+    Trace t(c, "spec_resample", s);
+    CUDA_TRY(launch_spec_resample(c, target_logits, inv_t, seed, step, accept_len, next_token, s));
     return DFLARE_OK;
 }
 

@@ -11,6 +11,8 @@
 
 namespace dfl {
 
+constexpr int kSpecMaxChunks = 64;   // vocabulary chunks per row of the sampled verification
+
 // Epilogue kinds of the projection GEMMs (applied to a 128-feature x token tile in fp32).
 enum EpiKind : int {
     EPI_STORE = 0,      // out[g][tok][n] = acc (+ bias[g][n])    (storage type)
@@ -113,6 +115,9 @@ struct dflare_ctx {
     int tile_cnt_n = 0;
     unsigned long long* amax_slot = nullptr;  // packed (value, index) per logits row [max_batch*B]
     int32_t* tgt_tok = nullptr;    // [max_batch*B] target argmax of dflare_verify_logits
+    float2* spec_part = nullptr;   // [max_batch*(2B-1)][kSpecMaxChunks] softmax partials (m, s)
+    int spec_chunks = 1;           // vocabulary chunks of the current sampled verification
+    int32_t* spec_a = nullptr;     // [max_batch] first rejected draft position
     uint32_t* amax_cnt = nullptr;
     float* rope_cos = nullptr;     // [max_ctx + B][hd/2]
     float* rope_sin = nullptr;
@@ -184,6 +189,14 @@ cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gathe
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s);
 cudaError_t launch_argmax(dflare_ctx* c, const float* logits, int rows, int32_t* tokens,
                           cudaStream_t s);
+cudaError_t launch_sample(dflare_ctx* c, int rows, float inv_t, uint64_t seed, const uint64_t* step,
+                          int32_t* tokens, cudaStream_t s);
+cudaError_t launch_spec_stats(dflare_ctx* c, const float* target_logits, float inv_t, cudaStream_t s);
+cudaError_t launch_spec_accept(dflare_ctx* c, const int32_t* draft, const float* target_logits,
+                               float inv_t, uint64_t seed, const uint64_t* step, cudaStream_t s);
+cudaError_t launch_spec_resample(dflare_ctx* c, const float* target_logits, float inv_t,
+                                 uint64_t seed, uint64_t* step, int32_t* accept_len,
+                                 int32_t* next_token, cudaStream_t s);
 cudaError_t launch_verify(dflare_ctx* c, const int32_t* draft, const int32_t* target,
                           int32_t* accept_len, int32_t* next_token, cudaStream_t s);
 cudaError_t launch_synthetic_target(const int32_t* draft, const uint32_t* u, const int32_t* r,
