@@ -46,7 +46,8 @@ def parse():
     p.add_argument("--workload", default="qwen3_4b", choices=sorted(synth.PRESETS))
     p.add_argument("--e2e-steps", type=int, default=50)
     p.add_argument("--breakdown-steps", type=int, default=30)
-    p.add_argument("--cpu-steps", type=int, default=2, help="oracle steps timed for cpu_baseline")
+    p.add_argument("--cpu-seconds", type=float, default=12.0,
+                   help="CPU time budget of the oracle steps timed for cpu_baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--fill-chunk", type=int, default=2048)
     p.add_argument("--serial-launch", action="store_true",
@@ -73,8 +74,9 @@ def host_cores():
 
 # ----------------------------------------------------------------------------- CPU oracle leg
 
-def oracle_steps(w, W, n_steps):
-    """Time n_steps full oracle block steps after an untimed oracle context fill."""
+def oracle_steps(w, W, n_steps, budget_s=None):
+    """Time full oracle block steps after an untimed oracle context fill: n_steps of them, or,
+    with budget_s, as many as fit in budget_s seconds (at least 2, at most n_steps)."""
     import oracle as O
     s = w.shape
     o = O.DraftOracle(W, s, w.batch, storage="bf16" if s.dtype == "bf16" else "exact")
@@ -91,7 +93,11 @@ def oracle_steps(w, W, n_steps):
     thr = synth.accept_threshold(w.match_p)
     t0 = time.perf_counter()
     tau_sum = 0
+    done = 0
     for step in range(n_steps):
+        if budget_s is not None and step >= 2 and time.perf_counter() - t0 >= budget_s:
+            break
+        done += 1
         u, r, last = synth.target_draws(w, step)
         for b in range(w.batch):
             if taus[b]:
@@ -102,8 +108,8 @@ def oracle_steps(w, W, n_steps):
             taus[b], x_t[b] = O.verify_accept(tok, g)
             tau_sum += taus[b]
     dt = time.perf_counter() - t0
-    drafted = n_steps * w.batch * (s.block - 1)
-    return drafted / dt, dt, tau_sum / (n_steps * w.batch)
+    drafted = done * w.batch * (s.block - 1)
+    return drafted / dt, dt, tau_sum / (done * w.batch), done
 
 
 def run_reference(args):
@@ -113,10 +119,7 @@ def run_reference(args):
     w = synth.preset(args.workload)
     W = synth.weights(w)
     # bounded: at most ~150 s of oracle steps in the whole run
-    probe_v, probe_dt, _ = oracle_steps(w, W, 1)
-    budget = 150.0
-    n = max(1, min(args.steps, int(budget / max(probe_dt, 1e-3))))
-    value, dt, tau = oracle_steps(w, W, n)
+    value, dt, tau, n = oracle_steps(w, W, args.steps, budget_s=150.0)
     sample = (f"{n} of {args.steps} requested block steps of workload {w.name} (oracle fp64, "
               f"bf16 storage rounding) after an untimed oracle fill of {list(w.ctx_lens)} "
               f"positions; warmup: 1 step")
@@ -738,10 +741,10 @@ def run_ours(args):
                                         torch.from_numpy(synth.initial_tokens(w)).cuda())
     del fill_chunks
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, dt, tau = oracle_steps(w, W, args.cpu_steps)
+        v, dt, tau, n_cpu = oracle_steps(w, W, 10 ** 6, budget_s=args.cpu_seconds)
         line["cpu_baseline"] = {
             "value": v, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
-            "sample": f"{args.cpu_steps} full block steps of {w.name} (fp64, bf16 storage "
+            "sample": f"{n_cpu} full block steps of {w.name} (fp64, bf16 storage "
                       f"rounding) after an untimed oracle fill of {list(w.ctx_lens)} positions",
             "seconds": dt}
     if rank == 0:

@@ -81,6 +81,15 @@ typedef enum { DFLARE_BF16 = 0, DFLARE_F32 = 1 } dflare_dtype;
                                            may be NULL. Cannot be combined with RAW_FUSION or
                                            FUSION_FC (DFLARE_EINVAL) */
 
+#define DFLARE_FLAG_DETERMINISTIC 0x80u /* bitwise-reproducible runs: the split-K partial sums of
+                                           the residual projections (W_O, W_down) are reduced in
+                                           a fixed order by the last CTA of each tile. Without it
+                                           every split adds its partial to the fp32 residual
+                                           stream with L2 reductions, which is faster but leaves
+                                           the order of those additions, and so the last bit of
+                                           the residual, free to vary between runs (the
+                                           verification decides every emitted token either way) */
+
 /* Device error word bits (dflare_device_error) */
 #define DFLARE_DEVERR_TOKEN     0x1u    /* a token id outside [0, vocab) was read (clamped to 0) */
 #define DFLARE_DEVERR_CAPACITY  0x2u    /* ctx_len + n_new > max_ctx, or n_new outside [0, n_max]:

@@ -59,6 +59,7 @@ struct TcArgs {
     // activation addressing of the kAux instance only
     int b_kg;                  // > 0: activation group z holds contraction indices [z b_kg, (z+1) b_kg)
     int b_gsel;                // 1: activation group = weight group; 0: one activation group for all
+    int resid_red;             // EPI_RESID: each split adds its partial to resid with L2 reductions
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -439,8 +440,39 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         float* const ws = args.ws;
         uint32_t* const tile_cnt = args.tile_cnt;
         const bool resid = args.ep.kind == EPI_RESID && bn == kChunk;
+        const bool resid_red = resid && args.resid_red;
         for (int u = blockIdx.x; u < G.n_units; u += gridDim.x) {
             const Unit x = decode_unit(G, u);
+            if (resid_red) {
+                // resid += acc with fp32 reductions in L2: every split adds its own partial sum,
+                // with no workspace, no tile counter and no read of the residual (the order of
+                // the additions, and so the last bit of the sum, can vary between runs)
+                if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, err)) break;
+                tc_fence_after();
+                const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
+                float v[kChunk];
+                tmem_ld16(taddr, v);
+                tc_fence_before();
+                mbar_arrive(tempty_bar(acc));
+                const int n = x.n_tile * 128 + t, tok0 = x.tok_tile * bn;
+                const int nvalid = min(kChunk, args.ep.m_tok - tok0);
+                if (n < args.ep.n) {
+                    float* dst = args.ep.resid + (size_t)tok0 * args.ep.ld_resid + n;
+#pragma unroll
+                    for (int c = 0; c < kChunk; ++c)
+                        if (c < nvalid)
+                            asm volatile("red.global.add.f32 [%0], %1;" ::"l"(dst + (size_t)c * args.ep.ld_resid),
+                                         "f"(v[c])
+                                         : "memory");
+                }
+                if (G.n_bufs == 2) {
+                    acc ^= 1;
+                    if (acc == 0) acc_phase ^= 1u;
+                } else {
+                    acc_phase ^= 1u;
+                }
+                continue;
+            }
             // the residual rows do not depend on the accumulator: load them before waiting
             float rr[kChunk];
             if (resid) load_resid(args.ep, x.n_tile, x.tok_tile * bn, t, rr);
@@ -663,6 +695,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     // group shared by all (b_shared), or k / b_kgroup groups that the contraction runs across
     const long long a_gr = g.a_group_rows > 0 ? g.a_group_rows : g.n;
     a.b_kg = g.b_kgroup;
+    a.resid_red = (c->cfg.flags & DFLARE_FLAG_DETERMINISTIC) ? 0 : 1;
     a.b_gsel = g.b_shared ? 0 : 1;
     const int b_k = g.b_kgroup > 0 ? g.b_kgroup : g.k;
     const int b_groups = g.b_kgroup > 0 ? g.k / g.b_kgroup : (g.b_shared ? 1 : g.groups);

@@ -122,10 +122,11 @@ def test_steps_with_verification(run):
 
 def test_rope_off_block_is_mask_permutation_equivariant():
     """With block RoPE off, all mask rows have the same input, so their hidden states and logits
-    coincide (the bidirectional block has no position-dependent mask)."""
-    from paper_2606_02091_gb300 import FLAG_NO_BLOCK_ROPE
+    coincide (the bidirectional block has no position-dependent mask). Bit-identical rows need
+    reductions in a fixed order, hence the deterministic mode."""
+    from paper_2606_02091_gb300 import FLAG_DETERMINISTIC, FLAG_NO_BLOCK_ROPE
     w = SMALL_HD64
-    g = GpuRun(w, flags=FLAG_NO_BLOCK_ROPE)
+    g = GpuRun(w, flags=FLAG_NO_BLOCK_ROPE | FLAG_DETERMINISTIC)
     g.fuse(w.ctx_lens, want_fused=False)
     tok, logits, hidden = g.draft(synth.initial_tokens(w))
     o = oracle_for(w, g.W, rope_block=False)
@@ -291,3 +292,24 @@ def test_verify_from_logits_matches_oracle(w):
         want = [O.verify_from_logits(draft[b], lg[b]) for b in range(bsz)]
         assert got == want, (rnd, got, want)
     assert g.lib.device_error() == 0
+
+
+@pytest.mark.parametrize("w", [SMALL_HD128, WIDE_B16], ids=lambda w: w.name)
+def test_deterministic_mode_repeats_bit_for_bit(w):
+    """DFLARE_FLAG_DETERMINISTIC: two contexts fed the same inputs draft bit-identical hidden
+    states and logits; the default mode (split-K partials added to the residual in L2) agrees
+    with it within the tolerance."""
+    from paper_2606_02091_gb300 import FLAG_DETERMINISTIC
+    x_t = synth.initial_tokens(w)
+    runs = []
+    for flags in (FLAG_DETERMINISTIC, FLAG_DETERMINISTIC, 0):
+        g = GpuRun(w, flags=flags)
+        g.fuse(w.ctx_lens, want_fused=False)
+        runs.append(g.draft(x_t))
+        del g
+    (t1, l1, h1), (t2, l2, h2), (t3, l3, h3) = runs
+    np.testing.assert_array_equal(h1, h2)
+    np.testing.assert_array_equal(l1, l2)
+    np.testing.assert_array_equal(t1, t2)
+    assert rel_err(h3, h1) <= tolerance(w)
+    assert rel_err(l3, l1) <= tolerance(w)
