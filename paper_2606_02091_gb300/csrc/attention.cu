@@ -92,29 +92,12 @@ __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-// P.V runs on fp16 operands: P in [0, 1] keeps 11 significant bits instead of bf16's 8, and
-// the bf16 values of V convert to fp16 exactly (except magnitudes below 2^-14, which are far
-// below anything that moves an output).
-__device__ __forceinline__ void mma16816_f16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
-        "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
-    __half2 h = __floats2half2_rn(lo, hi);
+// P.V runs on bf16 operands: V as the TMA wrote it, P in [0, 1] rounded to bf16 (relative error
+// at most 2^-9, below the bf16 rounding of the attention output; the row sums l are taken from
+// the fp32 P).
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&h);
-}
-// 8 bf16 values in shared memory -> 8 fp16 values in place
-__device__ __forceinline__ void bf16x8_to_f16x8(void* p) {
-    uint4 u = *reinterpret_cast<uint4*>(p);
-    __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&u);
-    uint4 o;
-    __half2* h = reinterpret_cast<__half2*>(&o);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) h[i] = __float22half2_rn(__bfloat1622float2(b[i]));
-    *reinterpret_cast<uint4*>(p) = o;
 }
 
 constexpr int kNST = 2;                   // K/V tiles in flight per CTA (two CTAs fit on an SM)
@@ -190,6 +173,18 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = a.B * a.G;
     const uint32_t sbase = smem_addr(smem), fbar = smem_addr(full);
+    // rows [block_rows, 64) of the V stages are never written by the block tile's copy (its box
+    // has block_rows rows): zero them once, before any copy lands in the stages
+    if (a.block_rows < kKT) {
+        const int zr = kKT - a.block_rows;
+        for (int k = tid; k < kNST * (HD / 64) * zr * 8; k += blockDim.x) {
+            const int piece = k & 7, r = a.block_rows + (k >> 3) % zr, sub = (k >> 3) / zr;
+            const int st = sub / (HD / 64), h = sub % (HD / 64);
+            *reinterpret_cast<uint4*>(smem + (size_t)st * 2 * TB + TB + h * 8192 + r * 128 + piece * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
     if (tid == 0) {
         for (int i = 0; i < kNST; ++i)
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(fbar + 8u * i) : "memory");
@@ -259,22 +254,13 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
                 break;
             }
             ++consumed;
+            // keys past the tile's valid ones get P = 0; their V rows are finite (the caches and
+            // the K^d / V^d buffers are zeroed at creation and only ever hold written values),
+            // so they add nothing
             const int valid = t < n_ct ? min(kKT, L - (t0 + t) * kKT) : a.B;
-            // V to fp16 in place; rows past the tile's valid keys become zeros (their P is 0)
-            uint8_t* vt = smem + (size_t)st * 2 * TB + TB;
-            for (int k = tid; k < (int)(TB / 16); k += blockDim.x) {
-                const int r = (k & 511) >> 3;
-                if (r < valid) {
-                    bf16x8_to_f16x8(vt + (size_t)k * 16);
-                } else {
-                    *reinterpret_cast<uint4*>(vt + (size_t)k * 16) = make_uint4(0u, 0u, 0u, 0u);
-                }
-            }
-            // these generic-proxy writes come before the TMA that refills the stage later
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            if (t == 0) cp_wait<0>();
-            __syncthreads();
             if (t == 0) {
+                cp_wait<0>();
+                __syncthreads();
 #pragma unroll
                 for (int kk = 0; kk < HD / 16; ++kk) {
                     const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
@@ -339,18 +325,18 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
 #pragma unroll
             for (int kk = 0; kk < kKT / 16; ++kk) {
                 uint32_t pa[4];
-                pa[0] = pack_f16(sc[2 * kk][0], sc[2 * kk][1]);
-                pa[1] = pack_f16(sc[2 * kk][2], sc[2 * kk][3]);
-                pa[2] = pack_f16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-                pa[3] = pack_f16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+                pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+                pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+                pa[2] = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+                pa[3] = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
 #pragma unroll
                 for (int nt = 0; nt < HD / 8; nt += 2) {
                     const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                     const int c8 = nt + (lane >> 4);
                     uint32_t b0, b1, b2, b3;
                     ldsm_x4_t(sV + swz(row, c8), b0, b1, b2, b3);
-                    mma16816_f16(o[nt], pa, b0, b1);
-                    mma16816_f16(o[nt + 1], pa, b2, b3);
+                    mma16816(o[nt], pa, b0, b1);
+                    mma16816(o[nt + 1], pa, b2, b3);
                 }
             }
             __syncthreads();

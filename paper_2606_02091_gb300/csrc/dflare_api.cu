@@ -240,7 +240,10 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
         {c->ctx_len, g.max_batch * sizeof(int32_t)}, {c->app_base, g.max_batch * sizeof(int32_t)},
         {c->app_cnt, g.max_batch * sizeof(int32_t)}, {c->tile_cnt, (size_t)c->tile_cnt_n * 4},
         {c->amax_slot, rows * 8}, {c->amax_cnt, 4}, {c->err, 4},
-        {c->fused, D * (size_t)g.max_fuse_rows * d * esz}, {c->x, rows * d * 4}};
+        {c->fused, D * (size_t)g.max_fuse_rows * d * esz}, {c->x, rows * d * 4},
+        // every row the attention reads past the valid keys holds a written value or zero
+        {c->kcache, kv * esz}, {c->vcache, kv * esz}, {c->kd, rows * d_kv * esz},
+        {c->vd, rows * d_kv * esz}};
     for (auto& z : zs) {
         e = cudaMemset(z.p, 0, z.n);
         if (e != cudaSuccess) return bail(DFLARE_ECUDA, std::string("cudaMemset: ") + cudaGetErrorString(e));
