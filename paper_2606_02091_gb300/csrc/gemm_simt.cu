@@ -21,7 +21,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
     pdl_wait();
     __shared__ float sA[2][kTN][kTK + 1];
     __shared__ float sB[kTT][kTK + 1];
-    __shared__ float tile[2 * kTT * kTN];
+    __shared__ __align__(16) float tile[2 * kTT * kTN];
     const int n_tile = blockIdx.x % n_tiles, group = blockIdx.x / n_tiles;
     const int tok0 = blockIdx.y * kTT;
     const int na = A2 ? 2 : 1;

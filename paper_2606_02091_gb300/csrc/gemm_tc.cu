@@ -440,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         float* const ws = args.ws;
         uint32_t* const tile_cnt = args.tile_cnt;
         const bool resid = args.ep.kind == EPI_RESID && bn == kChunk;
-        const bool resid_red = resid && args.resid_red;
+        const bool resid_red = args.ep.kind == EPI_RESID && args.resid_red;
         for (int u = blockIdx.x; u < G.n_units; u += gridDim.x) {
             const Unit x = decode_unit(G, u);
             if (resid_red) {
@@ -450,20 +450,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
-                float v[kChunk];
-                tmem_ld16(taddr, v);
-                tc_fence_before();
-                mbar_arrive(tempty_bar(acc));
-                const int n = x.n_tile * 128 + t, tok0 = x.tok_tile * bn;
-                const int nvalid = min(kChunk, args.ep.m_tok - tok0);
-                if (n < args.ep.n) {
-                    float* dst = args.ep.resid + (size_t)tok0 * args.ep.ld_resid + n;
+                const int n = x.n_tile * 128 + t;
+                for (int c0 = 0; c0 < bn; c0 += kChunk) {
+                    float v[kChunk];
+                    tmem_ld16(taddr + (uint32_t)c0, v);
+                    if (c0 + kChunk >= bn) {
+                        tc_fence_before();
+                        mbar_arrive(tempty_bar(acc));
+                    }
+                    const int tok0 = x.tok_tile * bn + c0;
+                    const int nvalid = min(kChunk, args.ep.m_tok - tok0);
+                    if (n < args.ep.n) {
+                        float* dst = args.ep.resid + (size_t)tok0 * args.ep.ld_resid + n;
 #pragma unroll
-                    for (int c = 0; c < kChunk; ++c)
-                        if (c < nvalid)
-                            asm volatile("red.global.add.f32 [%0], %1;" ::"l"(dst + (size_t)c * args.ep.ld_resid),
-                                         "f"(v[c])
-                                         : "memory");
+                        for (int c = 0; c < kChunk; ++c)
+                            if (c < nvalid)
+                                asm volatile("red.global.add.f32 [%0], %1;" ::"l"(dst + (size_t)c * args.ep.ld_resid),
+                                             "f"(v[c])
+                                             : "memory");
+                    }
                 }
                 if (G.n_bufs == 2) {
                     acc ^= 1;
