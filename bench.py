@@ -52,6 +52,10 @@ def parse():
     p.add_argument("--fill-chunk", type=int, default=2048)
     p.add_argument("--serial-launch", action="store_true",
                    help="no programmatic dependent launch between kernels (A/B measurement)")
+    p.add_argument("--sweep", action="store_true",
+                   help="throughput sweep around the Qwen3-8B-shaped drafter (one JSON line per point)")
+    p.add_argument("--sweep-points", default="",
+                   help="comma-separated indexes into the sweep's point list (default: all)")
     p.add_argument("--no-variants", action="store_true",
                    help="skip the context-fusion comparison with the ablations and DFlash's FC")
     return p.parse_args()
@@ -428,6 +432,46 @@ def sampled_steps(w, dev_w, fill_chunks, hid_step, x0, reps=100, temperature=1.0
     return out
 
 
+def graph_breakdown(lib, cs, step, nb):
+    """Per-launch durations: a second CUDA graph of one step with CUDA events recorded by the
+    library's trace hook around every launch, replayed nb times. Returns name -> [ms, ...]."""
+    import torch
+    import paper_2606_02091_gb300 as P
+    cr = Cudart()
+    rec = []
+    pool = []
+
+    @P._lib.TRACE_FN
+    def ev_cb(user, name, phase, stream):
+        if len(pool) <= len(rec):
+            pool.append(cr.event())
+        e = pool[len(rec)]
+        cr.record(e, stream)
+        rec.append((name.decode(), phase, e))
+
+    L_ = P.load()
+    L_.dflare_set_trace(lib.raw, ev_cb, None)
+    g2 = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(cs):
+        with torch.cuda.graph(g2, stream=cs):
+            step()
+    L_.dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
+    torch.cuda.synchronize()
+    per = {}
+    for _ in range(nb):
+        g2.replay()
+        torch.cuda.synchronize()
+        open_ev = {}
+        for name, phase, e in rec:
+            if phase == 0:
+                open_ev.setdefault(name, []).append(e)
+            else:
+                st = open_ev[name].pop()
+                per.setdefault(name, []).append(cr.elapsed(st, e))
+    del g2
+    return per
+
+
 def replica_aggregate(ms, units_per_step, steps, dist=None, device="cuda"):
     """Weak-scaling aggregate of independent replicas (one per rank, no data-path exchange):
     the job's time is the slowest rank's, its throughput every rank's units over that time.
@@ -600,38 +644,9 @@ def run_ours(args):
     ms, value = replica_aggregate(ms, drafted_per_step, K, dist)
 
     # ---------------- per-kernel durations (CUDA events around every launch, graph replays)
-    cr = Cudart()
-    rec = []
-    pool = []
-
-    @P._lib.TRACE_FN
-    def ev_cb(user, name, phase, stream):
-        if len(pool) <= len(rec):
-            pool.append(cr.event())
-        e = pool[len(rec)]
-        cr.record(e, stream)
-        rec.append((name.decode(), phase, e))
-
-    L_.dflare_set_trace(lib.raw, ev_cb, None)
-    g2 = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(cs):
-        with torch.cuda.graph(g2, stream=cs):
-            step()
-    L_.dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
-    torch.cuda.synchronize()
-    per = {}
     nb = args.breakdown_steps
     t_b0 = time.perf_counter()
-    for _ in range(nb):
-        g2.replay()
-        torch.cuda.synchronize()
-        open_ev = {}
-        for name, phase, e in rec:
-            if phase == 0:
-                open_ev.setdefault(name, []).append(e)
-            else:
-                st = open_ev[name].pop()
-                per.setdefault(name, []).append(cr.elapsed(st, e))
+    per = graph_breakdown(lib, cs, step, nb)
     kernels = {}
     for name, ts in per.items():
         launches = len(ts) / nb
@@ -755,10 +770,130 @@ def run_ours(args):
     return 0
 
 
+# one-at-a-time around the centre, then two corners: b16 x B32 x L32768 x D16 (tensor- and
+# KV-heavy) and b16 x B16 (the M = 256 GEMM corner)
+SWEEP_CENTRE = dict(D=8, T=36, B=16, L=4096, batch=1, p=0.85)
+SWEEP_AXES = (("D", (2, 5, 8, 12, 16)), ("T", (4, 12, 36)), ("B", (8, 16, 32)),
+              ("L", (512, 2048, 8192, 32768)), ("batch", (1, 4, 16)), ("p", (0.6, 0.9)))
+SWEEP_CORNERS = (dict(batch=16, B=32, L=32768, D=16), dict(batch=16, B=16))
+
+
+def sweep_points():
+    pts = [dict(SWEEP_CENTRE)]
+    for k, vals in SWEEP_AXES:
+        pts += [{**SWEEP_CENTRE, k: v} for v in vals if v != SWEEP_CENTRE[k]]
+    return pts + [{**SWEEP_CENTRE, **c} for c in SWEEP_CORNERS]
+
+
+def run_sweep(args):
+    """Block steps per second over the sweep points (throughput only). Weights and target states
+    come from torch's device generator (N(0, 0.02^2) matrices, 1 + N(0, 0.02^2) gains, N(0, 1)
+    states): the content does not change the work, and the host generator would spend minutes
+    on the largest contexts. Each point fills its contexts in 2048-position chunks, then times a
+    CUDA graph of one block step (fuse tau positions, draft, synthetic target, verify)."""
+    import dataclasses
+    import torch
+    from paper_2606_02091_gb300 import DFlare, synthetic_target
+    torch.cuda.set_device(0)
+    K, Wm = args.steps, max(args.warmup, 3)
+    dmax = max(v for k, vals in SWEEP_AXES if k == "D" for v in vals)
+    top = dataclasses.replace(synth.sweep_point().shape, n_draft_layers=dmax)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(0)
+
+    def rnd(*shape, mean=0.0, std=0.02):
+        t = torch.randn(shape, generator=gen, device="cuda", dtype=torch.float32)
+        return (t * std + mean).to(torch.bfloat16)
+    Dm, d, F, V = top.n_draft_layers, top.d, top.ffn, top.vocab
+    W = {"fuse_norm": rnd(Dm, d, mean=1.0), "w_kv_ctx": rnd(Dm, 2 * top.d_kv, d),
+         "attn_norm": rnd(Dm, d, mean=1.0), "w_qkv": rnd(Dm, top.d_q + 2 * top.d_kv, d),
+         "w_o": rnd(Dm, d, top.d_q), "mlp_norm": rnd(Dm, d, mean=1.0), "w_gate": rnd(Dm, F, d),
+         "w_up": rnd(Dm, F, d), "w_down": rnd(Dm, d, F), "final_norm": rnd(d, mean=1.0),
+         "embed": rnd(V, d), "lm_head": rnd(V, d)}
+    stacked = ("fuse_norm", "w_kv_ctx", "attn_norm", "w_qkv", "w_o", "mlp_norm", "w_gate", "w_up", "w_down")
+    pts = sweep_points()
+    if args.sweep_points:
+        pts = [pts[int(i)] for i in args.sweep_points.split(",")]
+    for pt in pts:
+        w = synth.sweep_point(D=pt["D"], T=pt["T"], B=pt["B"], L=pt["L"], batch=pt["batch"], p=pt["p"])
+        s = w.shape
+        bsz, L, B, T = w.batch, pt["L"], s.block, s.n_target_layers
+        chunk = min(2048, L)
+        lib = DFlare.from_shape(s, max_batch=bsz, max_ctx=L + B * (K + Wm + 16),
+                                max_fuse_rows=bsz * max(chunk, B))
+        weights = {k: (v[:s.n_draft_layers] if k in stacked else v) for k, v in W.items()}
+        weights["fuse_logits"] = torch.randn((s.n_draft_layers, T), generator=gen, device="cuda")
+        lib.set_weights(weights)
+        lib.reset(bsz)
+        t_fill = time.perf_counter()
+        for pos0 in range(0, L, chunk):
+            H = torch.randn((T, bsz, chunk, d), generator=gen, device="cuda", dtype=torch.bfloat16)
+            n = torch.full((bsz,), min(chunk, L - pos0), dtype=torch.int32, device="cuda")
+            lib.fuse_context(H, n)
+            del H
+        torch.cuda.synchronize()
+        t_fill = time.perf_counter() - t_fill
+        hid = torch.randn((T, bsz, B, d), generator=gen, device="cuda", dtype=torch.bfloat16)
+        u, r, last = synth.target_draws(w, 0, 1024)
+        u_d, r_d, last_d = (torch.from_numpy(x).cuda() for x in (u.view(np.int32), r, last))
+        step_ctr = torch.zeros(1, dtype=torch.int32, device="cuda")
+        acc = torch.zeros(bsz, dtype=torch.int32, device="cuda")
+        nxt = torch.from_numpy(synth.initial_tokens(w)).cuda()
+        draft = torch.zeros((bsz, B - 1), dtype=torch.int32, device="cuda")
+        tgt = torch.zeros((bsz, B), dtype=torch.int32, device="cuda")
+        thr = synth.accept_threshold(w.match_p)
+
+        def step():
+            lib.fuse_context(hid, acc)
+            lib.draft_block(nxt, draft)
+            synthetic_target(draft, u_d, r_d, last_d, step_ctr, thr, bsz, B, tgt)
+            lib.verify_accept(draft, tgt, acc, nxt)
+
+        cs = torch.cuda.Stream()
+        cs.wait_stream(torch.cuda.current_stream())
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cs):
+            step()
+            torch.cuda.synchronize()
+            with torch.cuda.graph(graph, stream=cs):
+                step()
+        torch.cuda.synchronize()
+        for _ in range(Wm):
+            graph.replay()
+        torch.cuda.synchronize()
+        lens0 = lib.ctx_lens()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(K):
+            graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / K
+        tau = (sum(lib.ctx_lens()) - sum(lens0)) / (K * bsz)
+        if lib.device_error():
+            raise RuntimeError(f"device error at sweep point {pt}")
+        kern = {}
+        if args.breakdown_steps > 0:
+            per = graph_breakdown(lib, cs, step, args.breakdown_steps)
+            kern = {n: round(1e3 * float(np.sum(ts)) / args.breakdown_steps, 1) for n, ts in per.items()}
+        e = 2
+        wbytes = e * (s.n_draft_layers * (d * (s.d_q + 2 * s.d_kv) + s.d_q * d + 3 * d * s.ffn + 2 * s.d_kv * d)
+                      + V * d)
+        print(json.dumps({"sweep": pt, "ms_per_step": ms, "drafted_tokens_per_s": bsz * (B - 1) / (ms / 1e3),
+                          "mean_accept_len": tau, "accepted_tokens_per_s": bsz * tau / (ms / 1e3),
+                          "weight_gbs": wbytes / (ms / 1e3) / 1e9, "fill_s": t_fill,
+                          "us_per_step_events": kern}), flush=True)
+        del graph
+        lib.close()
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     return run_ours(args)
 
 

@@ -637,20 +637,18 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     a.k_blocks = (g.k + kBK - 1) / kBK;
     const int tiles = g.groups * a.n_tiles * a.tok_tiles;
     const int sms = c->num_sms;
-    // split-K choice: minimise waves * k-blocks per unit (+1 for the reduction), within the
-    // workspace and counter capacity
+    // split-K choice: the most splits that still run as one wave (tiles * splits <= SMs), within
+    // the workspace and counter capacity. Measured: a second wave of split units is slower than
+    // fewer, longer units even when it shortens every unit (d 4096 gate/up: 3 splits over 288
+    // units 97 us, 1 split over 96 units 42 us), so no split count that spills into a second
+    // wave is taken.
     int best = 1;
-    long long best_cost = (long long)((tiles + sms - 1) / sms) * a.k_blocks;
-    for (int sp = 2; sp <= 16 && sp <= a.k_blocks / 2; ++sp) {
+    for (int sp = 2; sp <= 16 && sp <= a.k_blocks / 2 && tiles * sp <= sms; ++sp) {
         const int kbp = (a.k_blocks + sp - 1) / sp;
         const int spn = (a.k_blocks + kbp - 1) / kbp;
         const size_t need = (size_t)tiles * spn * a.n_a * a.bn * 128;
         if (need > c->ws_floats || tiles > c->tile_cnt_n) break;
-        const long long cost = (long long)((tiles * spn + sms - 1) / sms) * kbp + 1;
-        if (cost < best_cost) {
-            best_cost = cost;
-            best = spn;
-        }
+        best = spn;
     }
     // Shared-memory budget: up to 227 KB (one CTA per SM; measured faster than two smaller CTAs
     // per SM, with or without programmatic dependent launch). Stage size: four 64-wide k-blocks
