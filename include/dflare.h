@@ -187,7 +187,8 @@ dflare_status dflare_fuse_context(dflare_ctx* ctx, const void* target_hidden_dev
  * Draft one block per sequence (Sec. 3.2, drafting phase, with Eq. 4's keys/values).
  *   last_token_dev    [batch] int32: the target decode token x_t of each sequence, at position
  *                     ctx_len[b]; the B-1 mask positions follow at ctx_len[b]+1 ..
- *   draft_tokens_dev  [batch][B-1] int32 out: greedy argmax at each mask position (ties -> lowest id).
+ *   draft_tokens_dev  [batch][B-1] int32 out: greedy argmax at each mask position (ties -> lowest id);
+ *                     may be NULL when B = 1 (no mask positions, nothing is drafted).
  *   logits_out_dev    optional [batch][B-1][V] fp32 out: the LM-head logits at the mask positions.
  *   hidden_out_dev    optional [D+1][batch][B][d] fp32 out: the block rows after the embedding and
  *                     after every draft layer (the residual stream, kept in fp32).
@@ -303,6 +304,7 @@ const char* dflare_last_error(const dflare_ctx* ctx);
  *   g[b][B-1] = last[s][b];
  * then *step_dev += 1. Tables: u [n_steps][batch][B-1] uint32, r [n_steps][batch][B-1] int32 in
  * [0, V-1), last [n_steps][batch] int32. threshold = floor(p * 2^32) for match probability p.
+ * With B = 1 the draft, u and r tables are empty and may be NULL.
  */
 dflare_status dflare_synthetic_target(const int32_t* draft_tokens_dev, const uint32_t* u_dev,
                                       const int32_t* r_dev, const int32_t* last_dev, int n_steps,

@@ -442,7 +442,9 @@ dflare_status draft_block_impl(dflare_ctx* c, const int32_t* last_token, int32_t
                                const Sampling* smp) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
     if (!c->weights_set) return fail(c, DFLARE_ESTATE, "dflare_set_weights has not been called");
-    if (!last_token || !draft_tokens) return fail(c, DFLARE_EINVAL, "last_token or draft_tokens is NULL");
+    // with B = 1 the block has no mask rows: nothing is drafted and draft_tokens may be NULL
+    if (!last_token || (!draft_tokens && c->cfg.block > 1))
+        return fail(c, DFLARE_EINVAL, "last_token or draft_tokens is NULL");
     const dflare_config& g = c->cfg;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const size_t esz = c->esz, d = g.d, B = g.block, F = g.ffn;
@@ -706,7 +708,8 @@ dflare_status dflare_synthetic_target(const int32_t* draft, const uint32_t* u, c
                                       uint32_t threshold, int batch, int block, int32_t* target,
                                       void* stream) {
     dflare_ctx* c = nullptr;
-    if (!u || !r || !last || !step || !target || (!draft && block > 1))
+    // with B = 1 there are no drafts: draft_tokens, u and r are empty and may be NULL
+    if (!last || !step || !target || ((!draft || !u || !r) && block > 1))
         return fail(nullptr, DFLARE_EINVAL, "a synthetic-target buffer is NULL");
     if (n_steps < 1 || batch < 1 || block < 1 || block > 32)
         return fail(nullptr, DFLARE_EINVAL, "n_steps, batch or block out of range");

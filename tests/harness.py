@@ -35,6 +35,29 @@ BLOCK32 = synth.Workload(
     synth.Shape(d=256, n_draft_layers=2, n_target_layers=3, n_q_heads=8, n_kv_heads=2,
                 head_dim=128, ffn=512, vocab=1500, block=32),
     (90, 17), 0.8, seed=14)
+# degenerate and less common shapes: more draft layers than the fusion kernels hold at once
+# (D 10), 128 query rows per KV head (G 8: two 64-row query tiles), a single fused target layer
+# with block 1 (no mask rows: nothing is drafted), and block 2
+D10 = synth.Workload(
+    "d10_bf16",
+    synth.Shape(d=256, n_draft_layers=10, n_target_layers=2, n_q_heads=4, n_kv_heads=2,
+                head_dim=64, ffn=256, vocab=700, block=4),
+    (33, 70), 0.8, seed=15)
+G8 = synth.Workload(
+    "g8_bf16_hd64",
+    synth.Shape(d=512, n_draft_layers=2, n_target_layers=3, n_q_heads=16, n_kv_heads=2,
+                head_dim=64, ffn=512, vocab=900, block=16),
+    (150, 45), 0.75, seed=16)
+BLOCK1 = synth.Workload(
+    "block1_t1_bf16",
+    synth.Shape(d=256, n_draft_layers=2, n_target_layers=1, n_q_heads=4, n_kv_heads=2,
+                head_dim=64, ffn=256, vocab=300, block=1),
+    (20, 1), 0.8, seed=17)
+BLOCK2 = synth.Workload(
+    "block2_bf16",
+    synth.Shape(d=256, n_draft_layers=2, n_target_layers=2, n_q_heads=4, n_kv_heads=2,
+                head_dim=128, ffn=256, vocab=300, block=2),
+    (64, 129), 0.8, seed=18)
 TINY = synth.preset("tiny_f32")
 
 

@@ -8,12 +8,12 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import (BLOCK32, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16, GpuRun, f64, oracle_for,
-                           rel_err, tolerance)
+from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16,
+                           GpuRun, f64, oracle_for, rel_err, tolerance)
 
 pytestmark = pytest.mark.gpu
 GAP = 1e-2
-WORKLOADS = [TINY, SMALL_HD128, SMALL_HD64]
+WORKLOADS = [TINY, SMALL_HD128, SMALL_HD64, D10, G8, BLOCK1, BLOCK2]
 
 
 @pytest.fixture(scope="module", params=WORKLOADS, ids=lambda w: w.name)
