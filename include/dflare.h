@@ -20,7 +20,12 @@
  *   borrowed: the caller owns them and keeps them valid until the stream has executed the call.
  * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Every call is
  *   stream-ordered and asynchronous unless it says otherwise; none allocates memory except
- *   dflare_create.
+ *   dflare_create (and the CUDA graphs below).
+ * - dflare_fuse_context, dflare_draft_block and dflare_draft_block_sampled replay repeated calls
+ *   as CUDA graphs: the second call with the same operands (context batch, buffer pointers,
+ *   sampling parameters) on a non-legacy stream that is not being captured is captured and
+ *   launched, later ones are replayed (host cost of a few microseconds). Results are those of the
+ *   direct launches. dflare_set_weights discards the graphs.
  * - Errors: argument checks happen on the host before anything is enqueued and return a status
  *   at once. Errors found by kernels (a token id out of range, a context that would overflow)
  *   set bits of a device error word read by dflare_device_error. Asynchronous CUDA errors are

@@ -610,6 +610,13 @@ int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int
     return sp;
 }
 
+int attention_launch_splits(const dflare_ctx* c) {
+    const dflare_config& g = c->cfg;
+    if (g.dtype == DFLARE_F32) return attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
+    const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
+    return attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc);
+}
+
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
     const dflare_config& g = c->cfg;
     AttnArgs a{};

@@ -152,6 +152,170 @@ const uint8_t* at(const void* base, size_t elems, size_t esz) {
     return static_cast<const uint8_t*>(base) + elems * esz;
 }
 
+// Repeated calls with the same operands run as one CUDA graph: the first call of a new operand
+// set runs its launches directly, the second is captured (thread-local capture on the caller's
+// stream) and launched, later ones replay the graph. The kernels' parameters depend only on the
+// operands in the key and on state that is fixed for the context (the weights: set_weights drops
+// the graphs); everything that varies from step to step (context lengths, accepted counts, step
+// counters) is read by the kernels from device memory. Calls made while the stream is being
+// captured, with a trace hook set, or on the legacy default stream run directly.
+void drop_slot(GraphSlot& sl) {
+    if (sl.exec) cudaGraphExecDestroy(sl.exec);
+    sl = GraphSlot{};
+}
+void drop_graph(CallGraph& cg) {
+    for (GraphSlot& sl : cg.slot) drop_slot(sl);
+}
+template <class F>
+dflare_status graphed(dflare_ctx* c, CallGraph& cg, const uint64_t* key, int nk, cudaStream_t s, F&& body) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (!s || c->trace_fn || cudaStreamIsCapturing(s, &cs) != cudaSuccess ||
+        cs != cudaStreamCaptureStatusNone) {
+        cudaGetLastError();
+        return body();
+    }
+    const size_t kb = (size_t)nk * sizeof(uint64_t);
+    GraphSlot* sl = nullptr;
+    for (GraphSlot& x : cg.slot)
+        if (x.seen && memcmp(x.key, key, kb) == 0) sl = &x;
+    if (!sl) {   // a new operand set: run it directly and remember it (evicting the oldest)
+        sl = &cg.slot[0];
+        for (GraphSlot& x : cg.slot)
+            if (x.used < sl->used) sl = &x;
+        drop_slot(*sl);
+        memcpy(sl->key, key, kb);
+        sl->seen = true;
+        sl->used = ++cg.clock;
+        return body();
+    }
+    sl->used = ++cg.clock;
+    if (sl->exec) {
+        if (cudaGraphLaunch(sl->exec, s) == cudaSuccess) return DFLARE_OK;
+        cudaGetLastError();
+        drop_slot(*sl);
+        return body();
+    }
+    // the second call with these operands: capture it
+    if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+        cudaGetLastError();
+        return body();
+    }
+    const dflare_status st = body();
+    cudaGraph_t graph = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(s, &graph);
+    if (st != DFLARE_OK || e != cudaSuccess || !graph) {
+        if (graph) cudaGraphDestroy(graph);
+        cudaGetLastError();
+        drop_slot(*sl);
+        return st != DFLARE_OK ? st : body();   // nothing ran while capturing: run it now
+    }
+    cudaGraphExec_t exec = nullptr;
+    const cudaError_t ei = cudaGraphInstantiate(&exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ei != cudaSuccess || cudaGraphLaunch(exec, s) != cudaSuccess) {
+        if (exec) cudaGraphExecDestroy(exec);
+        cudaGetLastError();
+        drop_slot(*sl);
+        return body();
+    }
+    sl->exec = exec;
+    return DFLARE_OK;
+}
+
+dflare_status fuse_context_launches(dflare_ctx* c, const void* hidden, const int32_t* n_new,
+                                    int n_max, void* fused_out, cudaStream_t s) {
+    const dflare_config& g = c->cfg;
+    const int m_tok = c->batch * n_max;
+    const size_t d_q = (size_t)g.n_q_heads * g.head_dim, d_kv = (size_t)g.n_kv_heads * g.head_dim;
+    {
+        Trace t(c, "fuse_begin", s);
+        CUDA_TRY(launch_fuse_begin(c, n_new, n_max, s));
+    }
+    // ctx_src: what the context K/V projection reads, [groups][ctx_rows][d]
+    const void* ctx_src = c->fused;
+    long long ctx_rows = g.max_fuse_rows;
+    int ctx_shared = 0;
+    if (g.flags & DFLARE_FLAG_DFLASH_FC) {
+        // Eq. 1: c_t = W_fc [h^(1); ...; h^(T)] + b_fc as one GEMM whose contraction runs over
+        // the T stacked target layers of target_hidden; one c for every draft layer
+        GemmDesc fc{};
+        fc.a = c->w.dflash_fc_w;
+        fc.b = hidden;
+        fc.groups = 1;
+        fc.n = g.d;
+        fc.k = g.n_target_layers * g.d;
+        fc.m_tok = m_tok;
+        fc.b_group_rows = m_tok;
+        fc.b_kgroup = g.d;
+        fc.ep = epi_base(c);
+        fc.ep.kind = EPI_STORE;
+        fc.ep.m_tok = m_tok;
+        fc.ep.n = g.d;
+        fc.ep.out = fused_out ? fused_out : c->fused;
+        fc.ep.ldo = g.d;
+        fc.ep.bias = c->w.dflash_fc_b;
+        dflare_status st = traced_gemm(c, "gemm_dflash_fc", fc, s);
+        if (st != DFLARE_OK) return st;
+        ctx_src = fc.ep.out;
+        ctx_rows = m_tok;
+        ctx_shared = 1;
+    } else {
+        const bool fc_after = g.flags & DFLARE_FLAG_FUSION_FC;
+        {
+            Trace t(c, "fuse_layers", s);
+            CUDA_TRY(launch_fuse_layers(c, hidden, n_max, fc_after ? nullptr : fused_out, s));
+        }
+        if (fc_after) {
+            // "+FC": F'^(i) = F^(i) W_fc^(i)T + b_fc^(i), one d x d GEMM per draft layer
+            GemmDesc fc{};
+            fc.a = c->w.fusion_fc_w;
+            fc.b = c->fused;
+            fc.groups = g.n_draft_layers;
+            fc.n = g.d;
+            fc.k = g.d;
+            fc.m_tok = m_tok;
+            fc.b_group_rows = g.max_fuse_rows;
+            fc.ep = epi_base(c);
+            fc.ep.kind = EPI_STORE;
+            fc.ep.m_tok = m_tok;
+            fc.ep.n = g.d;
+            fc.ep.out = fused_out ? fused_out : c->fused_fc;
+            fc.ep.ldo = g.d;
+            fc.ep.out_gstride = (fused_out ? (long long)m_tok : g.max_fuse_rows) * g.d;
+            fc.ep.bias = c->w.fusion_fc_b;
+            dflare_status st = traced_gemm(c, "gemm_fusion_fc", fc, s);
+            if (st != DFLARE_OK) return st;
+            ctx_src = fc.ep.out;
+            ctx_rows = fused_out ? (long long)m_tok : g.max_fuse_rows;
+        }
+    }
+    GemmDesc gd{};
+    if (g.flags & (DFLARE_FLAG_SHARED_KV | DFLARE_FLAG_DFLASH_FC)) {
+        // W_K^d / W_V^d: rows [d_q, d_q + 2 d_kv) of each layer's w_qkv
+        gd.a = at(c->w.w_qkv, d_q * g.d, c->esz);
+        gd.a_group_rows = (long long)(d_q + 2 * d_kv);
+    } else {
+        gd.a = c->w.w_kv_ctx;
+    }
+    gd.b = ctx_src;
+    gd.b_shared = ctx_shared;
+    gd.groups = g.n_draft_layers;
+    gd.n = (int)(2 * d_kv);
+    gd.k = g.d;
+    gd.m_tok = m_tok;
+    gd.b_group_rows = ctx_rows;
+    gd.ep = epi_base(c);
+    gd.ep.kind = EPI_KV_APPEND;
+    gd.ep.m_tok = gd.m_tok;
+    gd.ep.n = gd.n;
+    gd.ep.kcache = c->kcache;
+    gd.ep.vcache = c->vcache;
+    gd.ep.app_base = c->app_base;
+    gd.ep.app_cnt = c->app_cnt;
+    gd.ep.n_max = n_max;
+    return traced_gemm(c, "gemm_kv_ctx", gd, s);
+}
+
 }  // namespace
 
 namespace dfl {
@@ -275,6 +439,8 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
 dflare_status dflare_destroy(dflare_ctx* c) {
     if (!c) return DFLARE_OK;
     cudaDeviceSynchronize();
+    drop_graph(c->draft_graph);
+    drop_graph(c->fuse_graph);
     free_all(c);
     delete c;
     return DFLARE_OK;
@@ -304,6 +470,8 @@ dflare_status dflare_set_weights(dflare_ctx* c, const dflare_weights* w, void* s
             return fail(c, DFLARE_EINVAL, std::string("weight ") + n.name + " is not 16-byte aligned");
     }
     c->w = *w;
+    drop_graph(c->draft_graph);   // captured launches hold the previous weights' tensor maps
+    drop_graph(c->fuse_graph);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (!dflash) CUDA_TRY(launch_fusion_alpha(c, s));
     c->weights_set = true;
@@ -332,98 +500,14 @@ dflare_status dflare_fuse_context(dflare_ctx* c, const void* hidden, const int32
     if (n_max > c->cfg.max_ctx) return fail(c, DFLARE_ECAPACITY, "n_max exceeds max_ctx");
     if (reinterpret_cast<uintptr_t>(hidden) % 16 || reinterpret_cast<uintptr_t>(fused_out) % 16)
         return fail(c, DFLARE_EINVAL, "target_hidden and fused_out must be 16-byte aligned");
-    const dflare_config& g = c->cfg;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const int m_tok = c->batch * n_max;
-    const size_t d_q = (size_t)g.n_q_heads * g.head_dim, d_kv = (size_t)g.n_kv_heads * g.head_dim;
-    {
-        Trace t(c, "fuse_begin", s);
-        CUDA_TRY(launch_fuse_begin(c, n_new, n_max, s));
-    }
-    // ctx_src: what the context K/V projection reads, [groups][ctx_rows][d]
-    const void* ctx_src = c->fused;
-    long long ctx_rows = g.max_fuse_rows;
-    int ctx_shared = 0;
-    if (g.flags & DFLARE_FLAG_DFLASH_FC) {
-        // Eq. 1: c_t = W_fc [h^(1); ...; h^(T)] + b_fc as one GEMM whose contraction runs over
-        // the T stacked target layers of target_hidden; one c for every draft layer
-        GemmDesc fc{};
-        fc.a = c->w.dflash_fc_w;
-        fc.b = hidden;
-        fc.groups = 1;
-        fc.n = g.d;
-        fc.k = g.n_target_layers * g.d;
-        fc.m_tok = m_tok;
-        fc.b_group_rows = m_tok;
-        fc.b_kgroup = g.d;
-        fc.ep = epi_base(c);
-        fc.ep.kind = EPI_STORE;
-        fc.ep.m_tok = m_tok;
-        fc.ep.n = g.d;
-        fc.ep.out = fused_out ? fused_out : c->fused;
-        fc.ep.ldo = g.d;
-        fc.ep.bias = c->w.dflash_fc_b;
-        dflare_status st = traced_gemm(c, "gemm_dflash_fc", fc, s);
-        if (st != DFLARE_OK) return st;
-        ctx_src = fc.ep.out;
-        ctx_rows = m_tok;
-        ctx_shared = 1;
-    } else {
-        const bool fc_after = g.flags & DFLARE_FLAG_FUSION_FC;
-        {
-            Trace t(c, "fuse_layers", s);
-            CUDA_TRY(launch_fuse_layers(c, hidden, n_max, fc_after ? nullptr : fused_out, s));
-        }
-        if (fc_after) {
-            // "+FC": F'^(i) = F^(i) W_fc^(i)T + b_fc^(i), one d x d GEMM per draft layer
-            GemmDesc fc{};
-            fc.a = c->w.fusion_fc_w;
-            fc.b = c->fused;
-            fc.groups = g.n_draft_layers;
-            fc.n = g.d;
-            fc.k = g.d;
-            fc.m_tok = m_tok;
-            fc.b_group_rows = g.max_fuse_rows;
-            fc.ep = epi_base(c);
-            fc.ep.kind = EPI_STORE;
-            fc.ep.m_tok = m_tok;
-            fc.ep.n = g.d;
-            fc.ep.out = fused_out ? fused_out : c->fused_fc;
-            fc.ep.ldo = g.d;
-            fc.ep.out_gstride = (fused_out ? (long long)m_tok : g.max_fuse_rows) * g.d;
-            fc.ep.bias = c->w.fusion_fc_b;
-            dflare_status st = traced_gemm(c, "gemm_fusion_fc", fc, s);
-            if (st != DFLARE_OK) return st;
-            ctx_src = fc.ep.out;
-            ctx_rows = fused_out ? (long long)m_tok : g.max_fuse_rows;
-        }
-    }
-    GemmDesc gd{};
-    if (g.flags & (DFLARE_FLAG_SHARED_KV | DFLARE_FLAG_DFLASH_FC)) {
-        // W_K^d / W_V^d: rows [d_q, d_q + 2 d_kv) of each layer's w_qkv
-        gd.a = at(c->w.w_qkv, d_q * g.d, c->esz);
-        gd.a_group_rows = (long long)(d_q + 2 * d_kv);
-    } else {
-        gd.a = c->w.w_kv_ctx;
-    }
-    gd.b = ctx_src;
-    gd.b_shared = ctx_shared;
-    gd.groups = g.n_draft_layers;
-    gd.n = (int)(2 * d_kv);
-    gd.k = g.d;
-    gd.m_tok = m_tok;
-    gd.b_group_rows = ctx_rows;
-    gd.ep = epi_base(c);
-    gd.ep.kind = EPI_KV_APPEND;
-    gd.ep.m_tok = gd.m_tok;
-    gd.ep.n = gd.n;
-    gd.ep.kcache = c->kcache;
-    gd.ep.vcache = c->vcache;
-    gd.ep.app_base = c->app_base;
-    gd.ep.app_cnt = c->app_cnt;
-    gd.ep.n_max = n_max;
-    c->ctx_ub = std::min(c->cfg.max_ctx, c->ctx_ub + n_max);
-    return traced_gemm(c, "gemm_kv_ctx", gd, s);
+    const uint64_t key[] = {(uint64_t)c->batch, (uint64_t)(uintptr_t)hidden, (uint64_t)(uintptr_t)n_new,
+                            (uint64_t)n_max, (uint64_t)(uintptr_t)fused_out};
+    const dflare_status st = graphed(c, c->fuse_graph, key, 5, s, [&] {
+        return fuse_context_launches(c, hidden, n_new, n_max, fused_out, s);
+    });
+    if (st == DFLARE_OK) c->ctx_ub = std::min(c->cfg.max_ctx, c->ctx_ub + n_max);
+    return st;
 }
 
 }  // extern "C"
@@ -587,7 +671,13 @@ extern "C" {
 
 dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32_t* draft_tokens,
                                  float* logits_out, float* hidden_out, void* stream) {
-    return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, nullptr);
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    const uint64_t key[] = {(uint64_t)c->batch, (uint64_t)(uintptr_t)last_token,
+                            (uint64_t)(uintptr_t)draft_tokens, (uint64_t)(uintptr_t)logits_out,
+                            (uint64_t)(uintptr_t)hidden_out, (uint64_t)attention_launch_splits(c), 0, 0};
+    return graphed(c, c->draft_graph, key, 8, static_cast<cudaStream_t>(stream), [&] {
+        return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, nullptr);
+    });
 }
 
 dflare_status dflare_draft_block_sampled(dflare_ctx* c, const int32_t* last_token, float temperature,
@@ -597,7 +687,15 @@ dflare_status dflare_draft_block_sampled(dflare_ctx* c, const int32_t* last_toke
     if (bad_temperature(temperature)) return fail(c, DFLARE_EINVAL, "temperature must be finite and > 0");
     if (!step) return fail(c, DFLARE_EINVAL, "step is NULL");
     const Sampling smp{1.0f / temperature, seed, step};
-    return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, &smp);
+    uint32_t tbits;
+    memcpy(&tbits, &smp.inv_t, 4);
+    const uint64_t key[] = {(uint64_t)c->batch, (uint64_t)(uintptr_t)last_token,
+                            (uint64_t)(uintptr_t)draft_tokens, (uint64_t)(uintptr_t)logits_out,
+                            (uint64_t)(uintptr_t)hidden_out, (uint64_t)attention_launch_splits(c),
+                            seed, ((uint64_t)tbits << 32) ^ (uint64_t)(uintptr_t)step ^ (1ull << 63)};
+    return graphed(c, c->draft_graph, key, 8, static_cast<cudaStream_t>(stream), [&] {
+        return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, &smp);
+    });
 }
 
 dflare_status dflare_verify_accept(dflare_ctx* c, const int32_t* draft, const int32_t* target,

@@ -76,6 +76,21 @@ struct GemmDesc {
 
 }  // namespace dfl
 
+// Calls of the library replayed as CUDA graphs (see graphed() in dflare_api.cu): a few operand
+// sets per call type, least recently used first out (a caller that double-buffers its inputs
+// alternates between two).
+struct GraphSlot {
+    uint64_t key[8] = {};
+    bool seen = false;
+    cudaGraphExec_t exec = nullptr;
+    uint64_t used = 0;
+};
+struct CallGraph {
+    static constexpr int kSlots = 4;
+    GraphSlot slot[kSlots];
+    uint64_t clock = 0;
+};
+
 struct dflare_ctx {
     dflare_config cfg;
     int device = 0;
@@ -122,6 +137,7 @@ struct dflare_ctx {
     float* rope_cos = nullptr;     // [max_ctx + B][hd/2]
     float* rope_sin = nullptr;
     uint32_t* err = nullptr;       // device error word
+    CallGraph draft_graph, fuse_graph;   // graphs of repeated dflare_draft_block / _fuse_context calls
     dflare_trace_fn trace_fn = nullptr;
     void* trace_user = nullptr;
     std::string msg;
@@ -174,6 +190,9 @@ void noalloc_set_error(const std::string& message);
 
 // launchers (each returns the first CUDA error it meets)
 cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std::string* why);
+// the split count the next attention launch takes (the only launch parameter that depends on the
+// host-side context-length bound)
+int attention_launch_splits(const dflare_ctx* c);
 // bf16 tensor map with a 128-byte swizzle and zero fill outside the tensor (dims innermost first;
 // strides_bytes for dims 1..rank-1); false when the driver rejects it.
 bool encode_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,

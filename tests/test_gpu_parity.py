@@ -313,3 +313,68 @@ def test_deterministic_mode_repeats_bit_for_bit(w):
     np.testing.assert_array_equal(t1, t2)
     assert rel_err(h3, h1) <= tolerance(w)
     assert rel_err(l3, l1) <= tolerance(w)
+
+
+def test_repeated_calls_replay_as_graphs():
+    """Calls repeated with the same operands run as CUDA graphs (the second is captured, later ones
+    replay it). Two deterministic contexts take the same five steps on a side stream: one reusing
+    its buffers every step (replayed graphs), one with fresh buffers every call (direct launches).
+    Hidden states, logits, tokens, caches and context lengths agree bit for bit, and a change of
+    batch or buffers afterwards runs the new operands, not the old graph."""
+    import torch
+    from paper_2606_02091_gb300 import FLAG_DETERMINISTIC
+    w = SMALL_HD128
+    s = w.shape
+    bsz, B = w.batch, s.block
+    runs = []
+    for reuse in (True, False):
+        g = GpuRun(w, flags=FLAG_DETERMINISTIC)
+        st = torch.cuda.Stream()
+        dt = torch.bfloat16
+        with torch.cuda.stream(st):
+            g.fuse(w.ctx_lens, want_fused=False)
+            lens = list(w.ctx_lens)
+            mk = lambda: (torch.zeros((s.n_target_layers, bsz, B, s.d), dtype=dt, device="cuda"),
+                          torch.zeros(bsz, dtype=torch.int32, device="cuda"),
+                          torch.tensor(synth.initial_tokens(w), device="cuda"),
+                          torch.zeros((bsz, B - 1), dtype=torch.int32, device="cuda"),
+                          torch.zeros((bsz, B - 1, s.vocab), dtype=torch.float32, device="cuda"),
+                          torch.zeros((s.n_draft_layers + 1, bsz, B, s.d), dtype=torch.float32, device="cuda"))
+            bufs = mk()
+            out = []
+            for step in range(5):
+                if not reuse:
+                    fresh = mk()
+                    fresh[2].copy_(bufs[2])
+                    bufs = fresh
+                hid, n_new, last, toks, logits, hidden = bufs
+                n = [3 + (step + b) % 4 for b in range(bsz)]
+                from tests.harness import fill_hidden
+                hid.copy_(torch.from_numpy(fill_hidden(w, [B] * bsz, lens)).view(dt))
+                n_new.copy_(torch.tensor(n, dtype=torch.int32))
+                g.lib.fuse_context(hid, n_new, stream=st)
+                lens = [L + k for L, k in zip(lens, n)]
+                g.lib.draft_block(last, toks, logits, hidden, stream=st)
+                out.append((toks.clone(), logits.clone(), hidden.clone()))
+                last.copy_(toks[:, 0])
+        torch.cuda.synchronize()
+        kv = [g.lib.read_kv(i, b, 0, lens[b]) for i in range(s.n_draft_layers) for b in range(bsz)]
+        runs.append((out, kv, g.lib.ctx_lens(), lens))
+        assert g.lib.device_error() == 0
+        if reuse:   # a different batch after replays: direct launches for the new operands
+            from tests.harness import fill_hidden, to_device
+            w1 = w.with_(ctx_lens=w.ctx_lens[:1])
+            g.lib.reset(1)
+            g.lib.fuse_context(to_device(fill_hidden(w1, [w.ctx_lens[0]])),
+                               torch.tensor([w.ctx_lens[0]], dtype=torch.int32, device="cuda"))
+            t1, l1, h1 = g.draft(synth.initial_tokens(w)[:1])
+            o = oracle_for(w1, g.W)
+            o.fuse_context(0, synth.hidden_states(w, 0, 0, w.ctx_lens[0]))
+            _, ol, oh = o.draft_block(0, int(synth.initial_tokens(w)[0]))
+            assert rel_err(l1[0], ol) <= tolerance(w)
+    (oa, kva, la, lens_a), (ob, kvb, lb, lens_b) = runs
+    assert la == lb == lens_a == lens_b
+    for (ta, lga, ha), (tb, lgb, hb) in zip(oa, ob):
+        assert torch.equal(ta, tb) and torch.equal(lga, lgb) and torch.equal(ha, hb)
+    for (ka, va), (kb, vb) in zip(kva, kvb):
+        assert torch.equal(ka, kb) and torch.equal(va, vb)
