@@ -169,7 +169,7 @@ void drop_graph(CallGraph& cg) {
 template <class F>
 dflare_status graphed(dflare_ctx* c, CallGraph& cg, const uint64_t* key, int nk, cudaStream_t s, F&& body) {
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-    if (!s || c->trace_fn || cudaStreamIsCapturing(s, &cs) != cudaSuccess ||
+    if (!s || c->trace_fn || nk > GraphSlot::kKeyLen || cudaStreamIsCapturing(s, &cs) != cudaSuccess ||
         cs != cudaStreamCaptureStatusNone) {
         cudaGetLastError();
         return body();
@@ -674,8 +674,8 @@ dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
     const uint64_t key[] = {(uint64_t)c->batch, (uint64_t)(uintptr_t)last_token,
                             (uint64_t)(uintptr_t)draft_tokens, (uint64_t)(uintptr_t)logits_out,
-                            (uint64_t)(uintptr_t)hidden_out, (uint64_t)attention_launch_splits(c), 0, 0};
-    return graphed(c, c->draft_graph, key, 8, static_cast<cudaStream_t>(stream), [&] {
+                            (uint64_t)(uintptr_t)hidden_out, (uint64_t)attention_launch_splits(c), 0, 0, 0, 0};
+    return graphed(c, c->draft_graph, key, 10, static_cast<cudaStream_t>(stream), [&] {
         return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, nullptr);
     });
 }
@@ -692,8 +692,8 @@ dflare_status dflare_draft_block_sampled(dflare_ctx* c, const int32_t* last_toke
     const uint64_t key[] = {(uint64_t)c->batch, (uint64_t)(uintptr_t)last_token,
                             (uint64_t)(uintptr_t)draft_tokens, (uint64_t)(uintptr_t)logits_out,
                             (uint64_t)(uintptr_t)hidden_out, (uint64_t)attention_launch_splits(c),
-                            seed, ((uint64_t)tbits << 32) ^ (uint64_t)(uintptr_t)step ^ (1ull << 63)};
-    return graphed(c, c->draft_graph, key, 8, static_cast<cudaStream_t>(stream), [&] {
+                            1, seed, (uint64_t)tbits, (uint64_t)(uintptr_t)step};
+    return graphed(c, c->draft_graph, key, 10, static_cast<cudaStream_t>(stream), [&] {
         return draft_block_impl(c, last_token, draft_tokens, logits_out, hidden_out, stream, &smp);
     });
 }

@@ -80,7 +80,8 @@ struct GemmDesc {
 // sets per call type, least recently used first out (a caller that double-buffers its inputs
 // alternates between two).
 struct GraphSlot {
-    uint64_t key[8] = {};
+    static constexpr int kKeyLen = 10;
+    uint64_t key[kKeyLen] = {};
     bool seen = false;
     cudaGraphExec_t exec = nullptr;
     uint64_t used = 0;
