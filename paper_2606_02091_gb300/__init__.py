@@ -27,7 +27,9 @@ def _stream(stream=None):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def _need_cuda(name, t, dtype=None):
+def _need_cuda(name, t, dtype=None, numel=None):
+    """A contiguous CUDA tensor of `dtype` holding at least `numel` elements (None: unchecked).
+    The C ABI takes bare pointers, so an undersized buffer is caught here, on the host."""
     if t is None:
         return
     if not t.is_cuda:
@@ -36,6 +38,8 @@ def _need_cuda(name, t, dtype=None):
         raise ValueError(f"{name} must be contiguous")
     if dtype is not None and t.dtype != dtype:
         raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements, needs at least {numel}")
 
 
 class DFlare:
@@ -84,6 +88,14 @@ class DFlare:
     def _check(self, status):
         return _lib.check(status, self._ctx)
 
+    def _tdtype(self):
+        import torch
+        return torch.bfloat16 if self.dtype == "bf16" else torch.float32
+
+    def _rows(self):
+        """(batch, B, mask rows per sequence B - 1)"""
+        return self.batch, self.cfg.block, self.cfg.block - 1
+
     @property
     def raw(self):
         """The dflare_ctx* handle (for direct C-ABI calls)."""
@@ -111,27 +123,45 @@ class DFlare:
     def fuse_context(self, hidden, n_new, fused_out=None, stream=None):
         """hidden [T][batch][n_max][d]; n_new int32 [batch] (device)."""
         import torch
-        _need_cuda("hidden", hidden)
-        _need_cuda("n_new", n_new, torch.int32)
-        _need_cuda("fused_out", fused_out)
+        c = self.cfg
+        if hidden.dim() != 4 or hidden.shape[0] != c.n_target_layers or hidden.shape[1] != self.batch \
+                or hidden.shape[3] != c.d:
+            raise ValueError(f"hidden must be [T={c.n_target_layers}][batch={self.batch}][n_max][d={c.d}], "
+                             f"got {list(hidden.shape)}")
         n_max = hidden.shape[2]
+        _need_cuda("hidden", hidden, self._tdtype())
+        _need_cuda("n_new", n_new, torch.int32, self.batch)
+        slots = 1 if c.flags & FLAG_DFLASH_FC else c.n_draft_layers   # DFlash: one shared c_t
+        _need_cuda("fused_out", fused_out, self._tdtype(), slots * self.batch * n_max * c.d)
         self._check(self._L.dflare_fuse_context(self._ctx, _ptr(hidden), _ptr(n_new), n_max,
                                                 _ptr(fused_out), _stream(stream)))
 
     def draft_block(self, last_token, draft_tokens, logits_out=None, hidden_out=None, stream=None):
-        import torch
-        _need_cuda("last_token", last_token, torch.int32)
-        _need_cuda("draft_tokens", draft_tokens, torch.int32)
-        _need_cuda("logits_out", logits_out, torch.float32)
-        _need_cuda("hidden_out", hidden_out, torch.float32)
+        self._check_draft_args(last_token, draft_tokens, logits_out, hidden_out)
         self._check(self._L.dflare_draft_block(self._ctx, _ptr(last_token), _ptr(draft_tokens),
                                                _ptr(logits_out), _ptr(hidden_out), _stream(stream)))
 
+    def _check_draft_args(self, last_token, draft_tokens, logits_out, hidden_out):
+        import torch
+        b, B, m = self._rows()
+        c = self.cfg
+        _need_cuda("last_token", last_token, torch.int32, b)
+        _need_cuda("draft_tokens", draft_tokens, torch.int32, b * m)
+        _need_cuda("logits_out", logits_out, torch.float32, b * m * c.vocab)
+        _need_cuda("hidden_out", hidden_out, torch.float32, (c.n_draft_layers + 1) * b * B * c.d)
+
+    def _check_verify_args(self, draft_tokens, accept_len, next_token):
+        import torch
+        b, _, m = self._rows()
+        _need_cuda("draft_tokens", draft_tokens, torch.int32, b * m)
+        _need_cuda("accept_len", accept_len, torch.int32, b)
+        _need_cuda("next_token", next_token, torch.int32, b)
+
     def verify_accept(self, draft_tokens, target_argmax, accept_len, next_token, stream=None):
         import torch
-        for n, t in (("draft_tokens", draft_tokens), ("target_argmax", target_argmax),
-                     ("accept_len", accept_len), ("next_token", next_token)):
-            _need_cuda(n, t, torch.int32)
+        b, B, _ = self._rows()
+        self._check_verify_args(draft_tokens, accept_len, next_token)
+        _need_cuda("target_argmax", target_argmax, torch.int32, b * B)
         self._check(self._L.dflare_verify_accept(self._ctx, _ptr(draft_tokens), _ptr(target_argmax),
                                                  _ptr(accept_len), _ptr(next_token),
                                                  _stream(stream)))
@@ -141,11 +171,8 @@ class DFlare:
         """As draft_block, with tokens drawn at `temperature`; step: uint64 device counter
         (a one-element int64 tensor)."""
         import torch
-        _need_cuda("last_token", last_token, torch.int32)
-        _need_cuda("draft_tokens", draft_tokens, torch.int32)
-        _need_cuda("step", step, torch.int64)
-        _need_cuda("logits_out", logits_out, torch.float32)
-        _need_cuda("hidden_out", hidden_out, torch.float32)
+        self._check_draft_args(last_token, draft_tokens, logits_out, hidden_out)
+        _need_cuda("step", step, torch.int64, 1)
         self._check(self._L.dflare_draft_block_sampled(
             self._ctx, _ptr(last_token), float(temperature), int(seed) & (2 ** 64 - 1), _ptr(step),
             _ptr(draft_tokens), _ptr(logits_out), _ptr(hidden_out), _stream(stream)))
@@ -154,11 +181,10 @@ class DFlare:
                        next_token, stream=None):
         """Speculative-sampling verification of the last drafted block; advances step by one."""
         import torch
-        _need_cuda("target_logits", target_logits, torch.float32)
-        _need_cuda("step", step, torch.int64)
-        for n, t in (("draft_tokens", draft_tokens), ("accept_len", accept_len),
-                     ("next_token", next_token)):
-            _need_cuda(n, t, torch.int32)
+        b, B, _ = self._rows()
+        self._check_verify_args(draft_tokens, accept_len, next_token)
+        _need_cuda("target_logits", target_logits, torch.float32, b * B * self.cfg.vocab)
+        _need_cuda("step", step, torch.int64, 1)
         self._check(self._L.dflare_verify_sampled(
             self._ctx, _ptr(draft_tokens), _ptr(target_logits), float(temperature),
             int(seed) & (2 ** 64 - 1), _ptr(step), _ptr(accept_len), _ptr(next_token),
@@ -167,10 +193,9 @@ class DFlare:
     def verify_logits(self, draft_tokens, target_logits, accept_len, next_token, stream=None):
         """target_logits [batch][B][V] fp32: the target's argmax is taken on the device."""
         import torch
-        _need_cuda("target_logits", target_logits, torch.float32)
-        for n, t in (("draft_tokens", draft_tokens), ("accept_len", accept_len),
-                     ("next_token", next_token)):
-            _need_cuda(n, t, torch.int32)
+        b, B, _ = self._rows()
+        self._check_verify_args(draft_tokens, accept_len, next_token)
+        _need_cuda("target_logits", target_logits, torch.float32, b * B * self.cfg.vocab)
         self._check(self._L.dflare_verify_logits(self._ctx, _ptr(draft_tokens), _ptr(target_logits),
                                                  _ptr(accept_len), _ptr(next_token),
                                                  _stream(stream)))
@@ -201,10 +226,10 @@ def argmax_noalloc(logits, tokens_out, stream=None):
     """Greedy argmax of [rows][vocab] fp32 device logits into int32 tokens_out without any device
     allocation (see dflare_argmax_noalloc: fixed scratch, at most NOALLOC_MAX_ROWS rows)."""
     import torch
+    vocab = logits.shape[-1]
+    rows = logits.numel() // vocab if vocab else 0
     _need_cuda("logits", logits, torch.float32)
-    _need_cuda("tokens_out", tokens_out, torch.int32)
-    rows, vocab = logits.shape[0], logits.shape[-1]
-    rows = logits.numel() // vocab
+    _need_cuda("tokens_out", tokens_out, torch.int32, rows)
     _lib.check(load().dflare_argmax_noalloc(_ptr(logits), rows, vocab, _ptr(tokens_out),
                                             _stream(stream)))
 

@@ -102,3 +102,73 @@ def test_valid_config_without_gpu_fails_loudly(lib):
     st = lib.dflare_create(ctypes.byref(_cfg()), ctypes.byref(ctx))
     assert st == 3                                       # DFLARE_ECUDA
     assert not ctx
+
+
+class _FakeCuda:
+    """Stands in for a CUDA tensor on a machine without one: only what the binding inspects."""
+
+    def __init__(self, numel, dtype, shape=None):
+        self._n, self.dtype = numel, dtype
+        self.shape = tuple(shape) if shape is not None else (numel,)
+        self.is_cuda = True
+
+    def is_contiguous(self):
+        return True
+
+    def numel(self):
+        return self._n
+
+    def dim(self):
+        return len(self.shape)
+
+    def data_ptr(self):
+        raise AssertionError("an undersized buffer reached the C call")
+
+
+class _NoLib:
+    def __getattr__(self, name):
+        raise AssertionError(f"an undersized buffer reached the C call ({name})")
+
+
+def _bare_binding(block=4, vocab=11, d=8, D=2, T=3, batch=2, flags=0):
+    from paper_2606_02091_gb300 import DFlare, _lib
+    o = object.__new__(DFlare)   # no dflare_create: the checks run before any library call
+    o.cfg = _lib.Config(d, D, T, 2, 1, 4, 16, vocab, block, batch, 64, 64, vocab - 1, 1e-6, 1e6,
+                        _lib.DFLARE_F32, flags)
+    o.dtype, o.batch, o._ctx, o._L = "f32", batch, None, _NoLib()
+    return o
+
+
+def test_binding_rejects_undersized_buffers_on_the_host():
+    import torch
+    o = _bare_binding()
+    i32, f32 = torch.int32, torch.float32
+    ok_last, ok_toks = _FakeCuda(2, i32), _FakeCuda(2 * 3, i32)
+    with pytest.raises(ValueError, match="draft_tokens"):
+        o.draft_block(ok_last, _FakeCuda(5, i32))
+    with pytest.raises(ValueError, match="last_token"):
+        o.draft_block(_FakeCuda(1, i32), ok_toks)
+    with pytest.raises(ValueError, match="logits_out"):
+        o.draft_block(ok_last, ok_toks, logits_out=_FakeCuda(2 * 3 * 11 - 1, f32))
+    with pytest.raises(ValueError, match="hidden_out"):
+        o.draft_block(ok_last, ok_toks, hidden_out=_FakeCuda(3 * 2 * 4 * 8 - 1, f32))
+    with pytest.raises(ValueError, match="target_argmax"):
+        o.verify_accept(ok_toks, _FakeCuda(7, i32), ok_last, ok_last)
+    with pytest.raises(ValueError, match="target_logits"):
+        o.verify_logits(ok_toks, _FakeCuda(2 * 4 * 11 - 1, f32), ok_last, ok_last)
+    with pytest.raises(ValueError, match="must be torch.int32"):
+        o.verify_accept(ok_toks, _FakeCuda(8, torch.int64), ok_last, ok_last)
+    with pytest.raises(ValueError, match="step"):
+        o.draft_block_sampled(ok_last, 1.0, 0, _FakeCuda(0, torch.int64), ok_toks)
+    hid = _FakeCuda(3 * 2 * 5 * 8, f32, (3, 2, 5, 8))
+    with pytest.raises(ValueError, match="fused_out"):
+        o.fuse_context(hid, _FakeCuda(2, i32), _FakeCuda(2 * 2 * 5 * 8 - 1, f32))
+    with pytest.raises(ValueError, match="hidden must be"):
+        o.fuse_context(_FakeCuda(3 * 2 * 5 * 8, f32, (3, 1, 10, 8)), _FakeCuda(2, i32))
+    with pytest.raises(ValueError, match="must be torch.float32"):
+        o.fuse_context(_FakeCuda(3 * 2 * 5 * 8, torch.bfloat16, (3, 2, 5, 8)), _FakeCuda(2, i32))
+    # DFlash writes one shared context slot, so one slot is enough there
+    from paper_2606_02091_gb300 import FLAG_DFLASH_FC
+    od = _bare_binding(flags=FLAG_DFLASH_FC)
+    with pytest.raises(AssertionError, match="reached the C call"):
+        od.fuse_context(hid, _FakeCuda(2, i32), _FakeCuda(2 * 5 * 8, f32))
