@@ -674,6 +674,15 @@ def run_ours(args):
     for k in kernels.values():
         if k["gbs"]:
             k["frac_of_hbm"] = k["gbs"] / hbm
+    # the whole block step against HBM: every kernel's algorithmic bytes over the graph-timed
+    # step (no events between launches)
+    s_bytes = sum(k["algorithmic_bytes"] * k["launches_per_step"] for k in kernels.values())
+    s_gbs = s_bytes / (ms / K * 1e-3) / 1e9
+    step_roofline = {"bytes_per_step": s_bytes, "ms_per_step": ms / K, "achieved": s_gbs,
+                     "peak": hbm, "unit": "GB/s", "frac": s_gbs / hbm,
+                     "lower_bound_ms": s_bytes / (hbm * 1e9) * 1e3,
+                     "note": "algorithmic bytes of every kernel of a step (weights, context K/V, "
+                             "target states, logits) / the CUDA-graph step time"}
 
     # ---------------- end to end through the public calls with host buffers
     pin_h = hid_host.pin_memory()
@@ -756,6 +765,7 @@ def run_ours(args):
         "mean_accept_len": mean_tau,
         "accepted_tokens_per_s": world * w.batch * mean_tau * K / (ms / 1e3),
         "roofline": roofline,
+        "step_roofline": step_roofline,
         "kernels": kernels,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "ms_per_step": 1e3 * max(e2e_ms / 1e3, wall) / E,
