@@ -153,7 +153,9 @@ __device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* m, int
 // (sequence, head, query tile) form a thread-block cluster. The keys are cut into tiles of 64:
 // ceil(L / 64) context tiles, then one tile of the block's own B keys (K^d, V^d); the splits take
 // contiguous runs of tiles whose counts differ by at most one. One thread streams the tiles with TMA into a ring of kNST swizzled stages;
-// every thread waits on the stage's mbarrier. Each CTA runs online softmax over its keys and
+// every thread waits on the stage's mbarrier, and each warp signals a stage's second mbarrier when
+// it has read the tile, which is what the streaming thread waits for before refilling the stage (no
+// CTA-wide barrier per tile). Each CTA runs online softmax over its keys and
 // pushes its partial (O / l in fp16, running max, running sum) row by row into the shared memory
 // of the CTA that merges that row (DSMEM stores); after one cluster barrier every CTA merges its
 // slice of the 64 rows from its own shared memory and writes the bf16 result. No partials go
@@ -172,14 +174,15 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     // [p * RP + lr], O / l in fp16 and (running max in log2 units, running sum)
     __half* rO = reinterpret_cast<__half*>(Qs + kQT * LD);     // [kQT][HD]
     float* rML = reinterpret_cast<float*>(rO + kQT * HD);        // [kQT][2]
-    uint64_t* full = reinterpret_cast<uint64_t*>(rML + 2 * kQT);
+    uint64_t* full = reinterpret_cast<uint64_t*>(rML + 2 * kQT);   // [kNST] tile landed
+    uint64_t* empty = full + kNST;                                  // [kNST] tile read by all 4 warps
     constexpr int RP = kQT / S;                                  // merged rows per CTA
     cg::cluster_group cluster = cg::this_cluster();
     const int s = (int)cluster.block_rank();
     const int g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = a.B * a.G;
-    const uint32_t sbase = smem_addr(smem), fbar = smem_addr(full);
+    const uint32_t sbase = smem_addr(smem), fbar = smem_addr(full), ebar = smem_addr(empty);
     // rows [block_rows, 64) of the V stages are never written by the block tile's copy (its box
     // has block_rows rows): zero them once, before any copy lands in the stages
     if (a.block_rows < kKT) {
@@ -193,8 +196,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     if (tid == 0) {
-        for (int i = 0; i < kNST; ++i)
+        for (int i = 0; i < kNST; ++i) {
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(fbar + 8u * i) : "memory");
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 4;" ::"r"(ebar + 8u * i) : "memory");
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.kc)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.vc)) : "memory");
@@ -230,6 +235,14 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
         }
     };
     int issued = 0, consumed = 0;
+    bool prod_ok = true;   // thread 0: every wait for an emptied stage ended in time
+    // thread 0 refills the stage of tile `issued` once all four warps have read the tile that
+    // used it before (tile issued - kNST)
+    auto refill = [&]() {
+        if (issued >= kNST)
+            prod_ok = tile_wait(ebar + 8u * (issued % kNST), (uint32_t)(issued / kNST - 1) & 1u);
+        if (prod_ok) issue(issued++);
+    };
     if (tid == 0)
         for (; issued < min(kNST - 1, n_tiles); ++issued) issue(issued);
 
@@ -251,12 +264,24 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
         }
         cp_commit();
+        // the query tile is complete in shared memory before the loop (the only CTA barrier on
+        // this path before the loop ends; the first K/V tile is already in flight)
+        cp_wait<0>();
+        __syncthreads();
         uint32_t qa[HD / 16][4];
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+            const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
+            ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
+        }
         for (int t = 0; t < n_tiles; ++t) {
             const int st = t % kNST;
-            if (tid == 0 && issued < n_tiles) issue(issued++);   // the stage freed at the end of t-1
+            if (tid == 0 && prod_ok && issued < n_tiles) refill();   // tile t + kNST - 1
             const bool landed = tile_wait(fbar + 8u * st, (uint32_t)(t / kNST) & 1u);
-            if (__syncthreads_or(!landed)) {   // one decision for the whole CTA
+            // each warp decides for itself (no CTA barrier inside the loop); a warp that gives
+            // up stops reading tiles and arriving on the empty barriers, so thread 0's next wait
+            // for an emptied stage runs out as well
+            if (__any_sync(0xffffffffu, !landed || (tid == 0 && !prod_ok))) {
                 timed_out = true;
                 break;
             }
@@ -265,15 +290,6 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             // the K^d / V^d buffers are zeroed at creation and only ever hold written values),
             // so they add nothing
             const int valid = t < n_ct ? min(kKT, L - (t0 + t) * kKT) : a.B;
-            if (t == 0) {
-                cp_wait<0>();
-                __syncthreads();
-#pragma unroll
-                for (int kk = 0; kk < HD / 16; ++kk) {
-                    const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
-                    ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
-                }
-            }
             const uint32_t sK = sbase + (uint32_t)st * 2 * TB, sV = sK + TB;
             // S = Q K^T for 16 rows x 64 keys
             // (k outer, keys inner: eight independent accumulators between dependent MMAs)
@@ -346,7 +362,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
                     mma16816(o[nt + 1], pa, b2, b3);
                 }
             }
-            __syncthreads();
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ebar + 8u * st) : "memory");
         }
         cp_wait<0>();
 #pragma unroll
@@ -355,12 +372,12 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             l1 += __shfl_xor_sync(0xffffffffu, l1, off);
         }
     }
-    if (timed_out) {
-        if (tid == 0) atomicOr(a.err, DFLARE_DEVERR_TIMEOUT);
-        // copies still in flight land before this shared memory is reused or released
-        if (tid == 0)
-            for (int t = consumed; t < issued; ++t) tile_wait(fbar + 8u * (t % kNST), (uint32_t)(t / kNST) & 1u);
-    }
+    if (timed_out && lane == 0) atomicOr(a.err, DFLARE_DEVERR_TIMEOUT);
+    // copies still in flight (only after a timeout) land before this shared memory is reused or
+    // released; then every warp is done with the K/V stages, which the push below reuses
+    if (tid == 0)
+        for (int t = consumed; t < issued; ++t) tile_wait(fbar + 8u * (t % kNST), (uint32_t)(t / kNST) & 1u);
+    __syncthreads();
     asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
     // push the partial: query row r belongs to the merge slice of CTA r / RP, which keeps it at
     // [s * RP + r % RP]; O is normalised by l first (|O / l| <= max |V|, safe in fp16). The rows
@@ -518,7 +535,7 @@ __global__ void attn_combine_kernel(const AttnArgs a, T* __restrict__ out) {
 template <int HD>
 size_t mma_smem_bytes() {   // alignment pad, K/V stages, padded Q tile, pushed partials, barriers
     return 1024 + (size_t)kNST * 2 * HD * 128 + (size_t)kQT * (HD + 8) * sizeof(bf16) +
-           (size_t)kQT * HD * sizeof(__half) + (size_t)kQT * 2 * sizeof(float) + 8 * kNST;
+           (size_t)kQT * HD * sizeof(__half) + (size_t)kQT * 2 * sizeof(float) + 2 * 8 * kNST;
 }
 
 template <int HD, int S>
