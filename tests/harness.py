@@ -35,6 +35,13 @@ BLOCK32 = synth.Workload(
     synth.Shape(d=256, n_draft_layers=2, n_target_layers=3, n_q_heads=8, n_kv_heads=2,
                 head_dim=128, ffn=512, vocab=1500, block=32),
     (90, 17), 0.8, seed=14)
+# more token rows than one GEMM token tile holds: batch 9 x block 32 = 288 block rows (a 256-row
+# tile and a ragged 32-row one in every draft projection) and 279 LM-head rows
+MULTI_TILE = synth.Workload(
+    "multi_tile_bf16_b9_B32",
+    synth.Shape(d=256, n_draft_layers=2, n_target_layers=2, n_q_heads=4, n_kv_heads=2,
+                head_dim=64, ffn=384, vocab=800, block=32),
+    tuple(5 + (23 * b) % 67 for b in range(9)), 0.8, seed=19)
 # degenerate and less common shapes: more draft layers than the fusion kernels hold at once
 # (D 10), 128 query rows per KV head (G 8: two 64-row query tiles), a single fused target layer
 # with block 1 (no mask rows: nothing is drafted), and block 2

@@ -8,7 +8,7 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16,
+from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, MULTI_TILE, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16,
                            GpuRun, f64, oracle_for, rel_err, tolerance)
 
 pytestmark = pytest.mark.gpu
@@ -198,10 +198,11 @@ def test_simt_gemm_agrees_with_tcgen05_gemm():
     assert rel_err(la, lb) <= tolerance(w)
 
 
-@pytest.mark.parametrize("w", [WIDE_B16, BLOCK32], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [WIDE_B16, BLOCK32, MULTI_TILE], ids=lambda w: w.name)
 def test_wide_token_tiles_match_oracle(w):
-    """256 token rows per projection (batch 16, the widest tcgen05 token tile) and block 32: fused
-    context, cached K/V and the draft block against the oracle."""
+    """256 token rows per projection (batch 16, the widest tcgen05 token tile), block 32, and 288
+    rows (two token tiles, the second ragged): fused context, cached K/V and the draft block
+    against the oracle."""
     g = GpuRun(w)
     o = oracle_for(w, g.W)
     fused = f64(g.fuse(w.ctx_lens))
