@@ -29,6 +29,7 @@ constexpr uint64_t kPhiloxM0 = 0xD2E7470EE14C6C93ull, kPhiloxM1 = 0xCA5A82639512
 constexpr uint64_t kWeyl0 = 0x9E3779B97F4A7C15ull, kWeyl1 = 0xBB67AE8584CAA73Bull;
 constexpr uint64_t kRngDraft = 1, kRngAccept = 2, kRngResidual = 3;
 constexpr int kNone = 0x7fffffff;
+constexpr int kU = 4;   // groups of four logits a thread loads at once in the vocabulary scans
 
 __device__ __forceinline__ float unit_from_bits(uint64_t x) {
     return ((float)(x >> 41) + 0.5f) * 0x1p-23f;
@@ -137,16 +138,26 @@ __global__ void __launch_bounds__(256) sample_kernel(const float* __restrict__ l
     const bool vec = (V & 3) == 0;
     float bv = -INFINITY;
     int bi = kNone;
-    for (int i = c0 + threadIdx.x * 4; i < c1; i += blockDim.x * 4) {
-        float x[4], u[4];
-        load4(p, i, c1, vec, x);
-        philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)row, step, kRngDraft, seed, u);
+    // kU groups of four logits per thread and iteration, all loads issued before the first
+    // Philox block (ids ascend within a thread, so ">" keeps the lowest id of equal scores)
+    const int stride = blockDim.x * 4;
+    for (int base = c0 + threadIdx.x * 4; base < c1; base += stride * kU) {
+        float x[kU][4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float sc = x[e] * inv_t + gumbel(u[e]);
-            if (sc > bv) {
-                bv = sc;
-                bi = i + e;
+        for (int g = 0; g < kU; ++g) load4(p, base + g * stride, c1, vec, x[g]);
+#pragma unroll
+        for (int g = 0; g < kU; ++g) {
+            const int i = base + g * stride;
+            if (i >= c1) break;
+            float u[4];
+            philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)row, step, kRngDraft, seed, u);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float sc = x[g][e] * inv_t + gumbel(u[e]);
+                if (sc > bv) {
+                    bv = sc;
+                    bi = i + e;
+                }
             }
         }
     }
@@ -180,13 +191,32 @@ __global__ void __launch_bounds__(256) spec_stats_kernel(const float* __restrict
     const float* p = r < n_target_rows ? target + (size_t)r * V
                                        : draft + (size_t)(r - n_target_rows) * V;
     float m = -INFINITY, s = 0.f;
-    for (int i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-        const float x = p[i] * inv_t;
-        if (x > m) {
-            s = s * expf(m - x) + 1.f;
-            m = x;
-        } else if (x > -INFINITY) {
-            s += expf(x - m);
+    // kU groups of four logits per thread and iteration, loaded before they are used; the
+    // group's maximum updates the running maximum once, then its terms are added
+    const bool vec = (V & 3) == 0;
+    const int stride = blockDim.x * 4;
+    for (int base = c0 + threadIdx.x * 4; base < c1; base += stride * kU) {
+        float x[kU][4];
+#pragma unroll
+        for (int g = 0; g < kU; ++g) load4(p, base + g * stride, c1, vec, x[g]);
+        float gm = -INFINITY;
+#pragma unroll
+        for (int g = 0; g < kU; ++g)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                x[g][e] *= inv_t;   // NaN past the chunk: fmaxf ignores it, the test below skips it
+                gm = fmaxf(gm, x[g][e]);
+            }
+        if (gm > m) {
+            s = m > -INFINITY ? s * expf(m - gm) : 0.f;
+            m = gm;
+        }
+        if (m > -INFINITY) {
+#pragma unroll
+            for (int g = 0; g < kU; ++g)
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (x[g][e] > -INFINITY) s += expf(x[g][e] - m);
         }
     }
     __shared__ float sm[8], ss[8];
@@ -218,6 +248,7 @@ __global__ void __launch_bounds__(256) spec_stats_kernel(const float* __restrict
 // (max, normaliser) of one row from its chunk partials
 __device__ __forceinline__ float2 row_stats(const float2* part, int row, int chunks) {
     float m = -INFINITY, s = 0.f;
+#pragma unroll 8
     for (int c = 0; c < chunks; ++c) {
         const float2 q = part[(size_t)row * chunks + c];
         const float M = fmaxf(m, q.x);
@@ -286,20 +317,30 @@ __global__ void __launch_bounds__(256) spec_resample_kernel(
     const bool vec = (V & 3) == 0;
     float bv = -INFINITY;
     int bi = kNone;
-    for (int i = c0 + threadIdx.x * 4; i < c1; i += blockDim.x * 4) {
-        float xt[4], xq[4], u[4];
-        load4(lt, i, c1, vec, xt);
-        if (resid) load4(lq, i, c1, vec, xq);
-        philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)b, step, kRngResidual, seed, u);
+    const int stride = blockDim.x * 4;
+    for (int base = c0 + threadIdx.x * 4; base < c1; base += stride * kU) {
+        float xt[kU][4], xq[kU][4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            float w = expf(xt[e] * inv_t - st.x) / st.y;
-            if (resid) w -= expf(xq[e] * inv_t - sq.x) / sq.y;
-            if (w > 0.f) {
-                const float sc = logf(w) + gumbel(u[e]);
-                if (sc > bv) {
-                    bv = sc;
-                    bi = i + e;
+        for (int g = 0; g < kU; ++g) {
+            load4(lt, base + g * stride, c1, vec, xt[g]);
+            if (resid) load4(lq, base + g * stride, c1, vec, xq[g]);
+        }
+#pragma unroll
+        for (int g = 0; g < kU; ++g) {
+            const int i = base + g * stride;
+            if (i >= c1) break;
+            float u[4];
+            philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)b, step, kRngResidual, seed, u);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                float w = expf(xt[g][e] * inv_t - st.x) / st.y;
+                if (resid) w -= expf(xq[g][e] * inv_t - sq.x) / sq.y;
+                if (w > 0.f) {
+                    const float sc = logf(w) + gumbel(u[e]);
+                    if (sc > bv) {
+                        bv = sc;
+                        bi = i + e;
+                    }
                 }
             }
         }
@@ -341,9 +382,10 @@ __global__ void __launch_bounds__(256) spec_resample_kernel(
     }
 }
 
-// chunk size (a multiple of 4, at least 1024) and count for `rows` rows of V entries
-void chunking(int V, int rows, int sms, int max_chunks, int* chunk, int* chunks) {
-    int n = std::max(1, (2 * sms + rows - 1) / rows);
+// chunk size (a multiple of 4, at least 1024) and count for `rows` rows of V entries, about
+// per_sm CTAs per SM (the scans that end in one packed atomicMax per CTA use two)
+void chunking(int V, int rows, int sms, int max_chunks, int per_sm, int* chunk, int* chunks) {
+    int n = std::max(1, (per_sm * sms + rows - 1) / rows);
     n = std::min(n, max_chunks);
     int c = (V + n - 1) / n;
     c = std::max(1024, ((c + 3) / 4) * 4);
@@ -357,7 +399,7 @@ cudaError_t launch_sample(dflare_ctx* c, int rows, float inv_t, uint64_t seed, c
                           int32_t* tokens, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     int chunk, chunks;
-    chunking(c->cfg.vocab, rows, c->num_sms, 1 << 20, &chunk, &chunks);
+    chunking(c->cfg.vocab, rows, c->num_sms, 1 << 20, 2, &chunk, &chunks);
     return launch_kernel(c->pdl, sample_kernel, dim3(chunks, rows), dim3(256), 0, s, c->logits,
                          c->cfg.vocab, rows, chunk, inv_t, seed, step, c->amax_slot, c->amax_cnt,
                          tokens);
@@ -367,7 +409,7 @@ cudaError_t launch_spec_stats(dflare_ctx* c, const float* target_logits, float i
     const int B = c->cfg.block, V = c->cfg.vocab;
     const int rows = c->batch * B + c->batch * (B - 1);
     int chunk, chunks;
-    chunking(V, rows, c->num_sms, kSpecMaxChunks, &chunk, &chunks);
+    chunking(V, rows, c->num_sms, kSpecMaxChunks, 4, &chunk, &chunks);
     c->spec_chunks = chunks;
     return launch_kernel(c->pdl, spec_stats_kernel, dim3(chunks, rows), dim3(256), 0, s,
                          target_logits, (const float*)c->logits, V, c->batch * B, chunk, inv_t,
@@ -386,7 +428,7 @@ cudaError_t launch_spec_resample(dflare_ctx* c, const float* target_logits, floa
                                  uint64_t seed, uint64_t* step, int32_t* accept_len,
                                  int32_t* next_token, cudaStream_t s) {
     int chunk, chunks;
-    chunking(c->cfg.vocab, c->batch, c->num_sms, 1 << 20, &chunk, &chunks);
+    chunking(c->cfg.vocab, c->batch, c->num_sms, 1 << 20, 2, &chunk, &chunks);
     return launch_kernel(c->pdl, spec_resample_kernel, dim3(chunks, c->batch), dim3(256), 0, s,
                          target_logits, (const float*)c->logits, c->cfg.vocab, c->cfg.block,
                          c->batch, chunk, c->spec_chunks, inv_t, seed, step,

@@ -107,12 +107,27 @@ __global__ void __launch_bounds__(256) argmax_kernel(const float* __restrict__ l
     float bv = -INFINITY;
     int bi = 0x7fffffff;
     if ((V & 3) == 0) {
-        for (int i = c0 + threadIdx.x * 4; i < c1; i += blockDim.x * 4) {
-            const float4 q = *reinterpret_cast<const float4*>(p + i);
-            if (q.x > bv) { bv = q.x; bi = i; }
-            if (q.y > bv) { bv = q.y; bi = i + 1; }
-            if (q.z > bv) { bv = q.z; bi = i + 2; }
-            if (q.w > bv) { bv = q.w; bi = i + 3; }
+        // four 16-byte loads in flight per thread (a scan with one load per iteration waits a
+        // full memory round trip per 16 bytes); ids ascend within a thread, so ">" keeps the
+        // lowest id of equal maxima; a load past the chunk reads as -inf, never chosen
+        constexpr int U = 4;
+        const int stride = blockDim.x * 4;
+        for (int base = c0 + threadIdx.x * 4; base < c1; base += stride * U) {
+            float4 q[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int i = base + u * stride;
+                q[u] = i < c1 ? *reinterpret_cast<const float4*>(p + i)
+                              : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int i = base + u * stride;
+                if (q[u].x > bv) { bv = q[u].x; bi = i; }
+                if (q[u].y > bv) { bv = q[u].y; bi = i + 1; }
+                if (q[u].z > bv) { bv = q[u].z; bi = i + 2; }
+                if (q[u].w > bv) { bv = q[u].w; bi = i + 3; }
+            }
         }
     } else {
         for (int i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
