@@ -621,16 +621,25 @@ int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub)
 }
 
 // Tensor-core path: the splits of one (sequence, head, query tile) are one cluster of 1, 2, 4, 8
-// or 16 CTAs: as many as needed for about two CTAs per SM, at most one per 64-key tile.
+// or 16 CTAs, at most one per 64-key tile: the most that still run as one wave at two CTAs per
+// SM, unless that leaves a CTA more than 12 tiles; then as many as give about two CTAs per SM in
+// all. Measured: with a few tiles per CTA the fixed cost of a CTA (launch, first tile, partial
+// push, cluster barrier, merge: ~6 us) dominates and one wave wins (Qwen3-8B-shaped batch 4,
+// 32 (sequence, head) pairs at L <= 4096: 8 splits, 1.256 ms per step, against 16 splits in two
+// waves, 1.327 ms); with long runs per CTA two waves of shorter CTAs overlap the next kernel
+// better (GPT-OSS-shaped batch 2, L 8192: 16 splits 1.046 ms, 8 splits 1.048 ms).
 int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int len_ub,
                              int max_cluster) {
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + kQT - 1) / kQT;
     const int base = batch * g.n_kv_heads * q_tiles;
-    const int want = (2 * num_sms + base - 1) / base;
     const int tiles = (len_ub + g.block + kKT - 1) / kKT;
     int sp = 1;
-    while (sp < max_cluster && sp < want && 2 * sp <= tiles) sp *= 2;
+    while (sp < max_cluster && 2 * sp <= tiles && base * 2 * sp <= 2 * num_sms) sp *= 2;
+    if ((tiles + sp - 1) / sp > 12) {
+        const int want = (2 * num_sms + base - 1) / base;
+        while (sp < max_cluster && sp < want && 2 * sp <= tiles) sp *= 2;
+    }
     return sp;
 }
 
