@@ -34,6 +34,9 @@
  * - Storage types: bf16 (default) or fp32 (dflare_config.dtype). "T" below is that type. Integer
  *   arrays are int32, row-major.
  * - One context serves one stream at a time; calls on one context must not overlap.
+ * - Devices: a context lives on the device that was current at dflare_create. Every call on it
+ *   makes that device current while it runs and restores the caller's device before returning,
+ *   so one thread may drive contexts on several GPUs; `stream` must belong to that device.
  */
 #ifndef DFLARE_H
 #define DFLARE_H

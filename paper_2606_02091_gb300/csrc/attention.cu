@@ -540,17 +540,17 @@ size_t mma_smem_bytes() {   // alignment pad, K/V stages, padded Q tile, pushed 
 
 template <int HD, int S>
 cudaError_t launch_mma(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
+    static PerDeviceOnce configured;
+    cudaError_t e = configured([] {
+        cudaError_t r = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)mma_smem_bytes<HD>());
-        if (e == cudaSuccess && S > 8)
-            e = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
+        if (r == cudaSuccess && S > 8)
+            r = cudaFuncSetAttribute(attn_mma_kernel<HD, S>,
                                      cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+        return r;
+    });
+    if (e != cudaSuccess) return e;
     return launch_cluster(c->pdl, S, attn_mma_kernel<HD, S>, dim3(S, a.hkv * a.q_tiles, c->batch),
                           dim3(128), mma_smem_bytes<HD>(), s, maps, a, static_cast<bf16*>(c->attn));
 }
@@ -570,9 +570,15 @@ cudaError_t run_mma(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cuda
 // of that size fit, else 8).
 template <int HD>
 int max_attention_cluster() {
-    static int cached = 0;
-    if (cached) return cached;
-    cached = 8;
+    static std::atomic<int> cache[64];   // per device (modulo 64): 0 = not yet queried
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 8;
+    }
+    std::atomic<int>& slot = cache[dev & 63];
+    if (const int known = slot.load(std::memory_order_acquire)) return known;
+    int cached = 8;
     if (cudaFuncSetAttribute(attn_mma_kernel<HD, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)mma_smem_bytes<HD>()) == cudaSuccess &&
         cudaFuncSetAttribute(attn_mma_kernel<HD, 16>, cudaFuncAttributeNonPortableClusterSizeAllowed,
@@ -593,6 +599,7 @@ int max_attention_cluster() {
             cached = 16;
     }
     cudaGetLastError();
+    slot.store(cached, std::memory_order_release);
     return cached;
 }
 

@@ -438,6 +438,7 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
 
 dflare_status dflare_destroy(dflare_ctx* c) {
     if (!c) return DFLARE_OK;
+    DeviceGuard dg(c->device);
     cudaDeviceSynchronize();
     drop_graph(c->draft_graph);
     drop_graph(c->fuse_graph);
@@ -448,6 +449,7 @@ dflare_status dflare_destroy(dflare_ctx* c) {
 
 dflare_status dflare_set_weights(dflare_ctx* c, const dflare_weights* w, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!w) return fail(c, DFLARE_EINVAL, "weights is NULL");
     const unsigned fl = c->cfg.flags;
     const bool dflash = fl & DFLARE_FLAG_DFLASH_FC;
@@ -480,6 +482,7 @@ dflare_status dflare_set_weights(dflare_ctx* c, const dflare_weights* w, void* s
 
 dflare_status dflare_reset(dflare_ctx* c, int batch, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (batch < 1 || batch > c->cfg.max_batch)
         return fail(c, DFLARE_ECAPACITY, "batch outside [1, max_batch]");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -492,6 +495,7 @@ dflare_status dflare_reset(dflare_ctx* c, int batch, void* stream) {
 dflare_status dflare_fuse_context(dflare_ctx* c, const void* hidden, const int32_t* n_new,
                                   int n_max, void* fused_out, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!c->weights_set) return fail(c, DFLARE_ESTATE, "dflare_set_weights has not been called");
     if (!hidden || !n_new) return fail(c, DFLARE_EINVAL, "target_hidden or n_new is NULL");
     if (n_max < 1) return fail(c, DFLARE_EINVAL, "n_max must be >= 1");
@@ -672,6 +676,7 @@ extern "C" {
 dflare_status dflare_draft_block(dflare_ctx* c, const int32_t* last_token, int32_t* draft_tokens,
                                  float* logits_out, float* hidden_out, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     const uint64_t key[] = {(uint64_t)c->batch, (uint64_t)(uintptr_t)last_token,
                             (uint64_t)(uintptr_t)draft_tokens, (uint64_t)(uintptr_t)logits_out,
                             (uint64_t)(uintptr_t)hidden_out, (uint64_t)attention_launch_splits(c), 0, 0, 0, 0};
@@ -684,6 +689,7 @@ dflare_status dflare_draft_block_sampled(dflare_ctx* c, const int32_t* last_toke
                                          uint64_t seed, const uint64_t* step, int32_t* draft_tokens,
                                          float* logits_out, float* hidden_out, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (bad_temperature(temperature)) return fail(c, DFLARE_EINVAL, "temperature must be finite and > 0");
     if (!step) return fail(c, DFLARE_EINVAL, "step is NULL");
     const Sampling smp{1.0f / temperature, seed, step};
@@ -701,6 +707,7 @@ dflare_status dflare_draft_block_sampled(dflare_ctx* c, const int32_t* last_toke
 dflare_status dflare_verify_accept(dflare_ctx* c, const int32_t* draft, const int32_t* target,
                                    int32_t* accept_len, int32_t* next_token, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!target || !accept_len || !next_token || (!draft && c->cfg.block > 1))
         return fail(c, DFLARE_EINVAL, "a verification buffer is NULL");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -712,6 +719,7 @@ dflare_status dflare_verify_accept(dflare_ctx* c, const int32_t* draft, const in
 dflare_status dflare_verify_logits(dflare_ctx* c, const int32_t* draft, const float* target_logits,
                                    int32_t* accept_len, int32_t* next_token, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!target_logits || !accept_len || !next_token || (!draft && c->cfg.block > 1))
         return fail(c, DFLARE_EINVAL, "a verification buffer is NULL");
     if (reinterpret_cast<uintptr_t>(target_logits) % 16)
@@ -730,6 +738,7 @@ dflare_status dflare_verify_sampled(dflare_ctx* c, const int32_t* draft, const f
                                     float temperature, uint64_t seed, uint64_t* step,
                                     int32_t* accept_len, int32_t* next_token, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!target_logits || !accept_len || !next_token || !step || (!draft && c->cfg.block > 1))
         return fail(c, DFLARE_EINVAL, "a verification buffer is NULL");
     if (bad_temperature(temperature)) return fail(c, DFLARE_EINVAL, "temperature must be finite and > 0");
@@ -753,6 +762,7 @@ dflare_status dflare_verify_sampled(dflare_ctx* c, const int32_t* draft, const f
 dflare_status dflare_read_kv(dflare_ctx* c, int layer, int seq, int pos0, int n, void* k_out,
                              void* v_out, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     const dflare_config& g = c->cfg;
     if (layer < 0 || layer >= g.n_draft_layers || seq < 0 || seq >= g.max_batch || pos0 < 0 || n < 0 ||
         (long long)pos0 + n > g.max_ctx)
@@ -775,6 +785,7 @@ dflare_status dflare_read_kv(dflare_ctx* c, int layer, int seq, int pos0, int n,
 
 dflare_status dflare_ctx_lens(dflare_ctx* c, int32_t* host, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!host) return fail(c, DFLARE_EINVAL, "ctx_len_host is NULL");
     CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
     CUDA_TRY(cudaMemcpy(host, c->ctx_len, c->batch * sizeof(int32_t), cudaMemcpyDeviceToHost));
@@ -783,6 +794,7 @@ dflare_status dflare_ctx_lens(dflare_ctx* c, int32_t* host, void* stream) {
 
 dflare_status dflare_device_error(dflare_ctx* c, uint32_t* bits, void* stream) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    DeviceGuard dg(c->device);
     if (!bits) return fail(c, DFLARE_EINVAL, "bits_host is NULL");
     CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
     CUDA_TRY(cudaMemcpy(bits, c->err, sizeof(uint32_t), cudaMemcpyDeviceToHost));

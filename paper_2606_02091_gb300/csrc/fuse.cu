@@ -371,15 +371,16 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
                   : g.n_draft_layers == 5 ? fuse_rows_kernel<T, 5> : fuse_rows_kernel<T, 8>;
         const int threads = rthreads;
         const size_t rsmem = rsmem_need;
-        static bool rconf = false;
-        if (!rconf) {
+        static PerDeviceOnce rconf;
+        const cudaError_t re = rconf([] {
             for (auto k : {fuse_rows_kernel<T, 4>, fuse_rows_kernel<T, 5>, fuse_rows_kernel<T, 8>}) {
                 cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                      220 * 1024);
                 if (e != cudaSuccess) return e;
             }
-            rconf = true;
-        }
+            return cudaSuccess;
+        });
+        if (re != cudaSuccess) return re;
         // persistent: as many CTAs as fit at once (two per SM at d = 2560), at most one per position
         int per_sm = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rk, threads, rsmem) != cudaSuccess || per_sm < 1)
@@ -391,16 +392,17 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
                              (long long)g.max_fuse_rows, g.rms_eps, c->err);
     }
     auto kern = g.n_draft_layers <= 4 ? fuse_layers_kernel<T, 4> : fuse_layers_kernel<T, 8>;
-    static bool configured = false;
-    if (!configured) {
+    static PerDeviceOnce configured;
+    const cudaError_t ce = configured([] {
         for (auto k : {fuse_layers_kernel<T, 4>, fuse_layers_kernel<T, 8>}) {
             cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  (int)((64 + 16) * kFuseCH * sizeof(T) +
                                                        (kFuseGroups - 1) * 8 * 8 * 64 * 4));
             if (e != cudaSuccess) return e;
         }
-        configured = true;
-    }
+        return cudaSuccess;
+    });
+    if (ce != cudaSuccess) return ce;
     return launch_cluster(c->pdl, C, kern, dim3(C, n_max, c->batch), dim3(256), smem, s, H,
                           (const float*)c->alpha, gain, F, Fo, (const int32_t*)c->app_cnt,
                           g.n_draft_layers, g.n_target_layers, c->batch, n_max, g.d,

@@ -716,13 +716,12 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         return cudaErrorInvalidValue;
     }
     const bool aux = g.b_kgroup > 0 || g.b_shared || g.ep.bias || g.ep.out_gstride;
-    static int configured[2] = {0, 0};
-    if (!configured[aux]) {
-        cudaError_t e = cudaFuncSetAttribute(aux ? gemm_tc_kernel<true> : gemm_tc_kernel<false>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
-        if (e != cudaSuccess) return e;
-        configured[aux] = 1;
-    }
+    static PerDeviceOnce configured[2];
+    const cudaError_t ce = configured[aux]([aux] {
+        return cudaFuncSetAttribute(aux ? gemm_tc_kernel<true> : gemm_tc_kernel<false>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+    });
+    if (ce != cudaSuccess) return ce;
     const int grid = std::min(a.n_units, sms);
     return launch_kernel(c->pdl, aux ? gemm_tc_kernel<true> : gemm_tc_kernel<false>, dim3(grid),
                          dim3(kThreads), smem, s, a);

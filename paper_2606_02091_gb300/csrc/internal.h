@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <string>
 #include <vector>
 
@@ -79,6 +80,38 @@ struct GemmDesc {
 // Calls of the library replayed as CUDA graphs (see graphed() in dflare_api.cu): a few operand
 // sets per call type, least recently used first out (a caller that double-buffers its inputs
 // alternates between two).
+// Makes the context's device current for the duration of an API call and restores the caller's
+// device afterwards (a process may drive contexts on several GPUs from one thread).
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        int cur = -1;
+        if (cudaGetDevice(&cur) == cudaSuccess && cur != dev && cudaSetDevice(dev) == cudaSuccess) prev = cur;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+    DeviceGuard(const DeviceGuard&) = delete;
+    DeviceGuard& operator=(const DeviceGuard&) = delete;
+};
+
+// cudaFuncSetAttribute acts on the current device only: a launcher runs its configuration once per
+// device (devices are told apart modulo 64).
+struct PerDeviceOnce {
+    std::atomic<uint64_t> mask{0};
+    template <class F>
+    cudaError_t operator()(F&& configure) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return e;
+        const uint64_t bit = 1ull << (dev & 63);
+        if (mask.load(std::memory_order_acquire) & bit) return cudaSuccess;
+        e = configure();
+        if (e == cudaSuccess) mask.fetch_or(bit, std::memory_order_acq_rel);
+        return e;
+    }
+};
+
 struct GraphSlot {
     static constexpr int kKeyLen = 10;
     uint64_t key[kKeyLen] = {};
