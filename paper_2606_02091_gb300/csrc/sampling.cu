@@ -399,7 +399,7 @@ cudaError_t launch_sample(dflare_ctx* c, int rows, float inv_t, uint64_t seed, c
                           int32_t* tokens, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     int chunk, chunks;
-    chunking(c->cfg.vocab, rows, c->num_sms, 1 << 20, 2, &chunk, &chunks);
+    chunking(c->cfg.vocab, rows, c->num_sms, 1 << 20, 4, &chunk, &chunks);
     return launch_kernel(c->pdl, sample_kernel, dim3(chunks, rows), dim3(256), 0, s, c->logits,
                          c->cfg.vocab, rows, chunk, inv_t, seed, step, c->amax_slot, c->amax_cnt,
                          tokens);
