@@ -24,7 +24,7 @@ and notation (arxiv 2606.02091):
   by the speculative-sampling rejection rule (the rule is not stated in the paper; see the
   sampling section below).
 
-Where the paper is silent the oracle takes these readings (each is also listed in the design doc):
+Where the paper is silent the oracle takes these readings:
 pre-norm residual blocks (RMSNorm -> attention -> residual; RMSNorm -> SwiGLU MLP -> residual)
 and a final RMSNorm before the LM head; RMSNorm y = g * x / sqrt(mean(x^2) + eps) with one gain
 vector per norm; no biases and no QK-norm; rotate-half RoPE on queries and keys, context row r

@@ -122,7 +122,7 @@ def fill_hidden(w: synth.Workload, lens, pos0=None):
     return H
 
 
-class GpuRun:
+class GpuSide:
     """The library on one workload: weights uploaded, sequences reset."""
 
     def __init__(self, w: synth.Workload, flags: int = 0, max_ctx: int | None = None,

@@ -8,7 +8,7 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import GpuRun, f64, oracle_for, rel_err, tolerance
+from tests.harness import GpuSide, f64, oracle_for, rel_err, tolerance
 
 pytestmark = pytest.mark.gpu
 GAP = 1e-2
@@ -16,7 +16,7 @@ GAP = 1e-2
 
 def test_qwen3_4b_full_step():
     w = synth.preset("qwen3_4b")
-    g = GpuRun(w, max_ctx=4096, max_fuse_rows=2048)
+    g = GpuSide(w, max_ctx=4096, max_fuse_rows=2048)
     fused = g.fuse(w.ctx_lens)
     x_t = synth.initial_tokens(w)
     tok, logits, hidden = g.draft(x_t)
@@ -44,7 +44,7 @@ def test_sampled_rows_full_size(name):
     w = synth.preset(name)
     s = w.shape
     chunk = 1024
-    g = GpuRun(w, max_ctx=max(w.ctx_lens) + 64, max_fuse_rows=w.batch * chunk)
+    g = GpuSide(w, max_ctx=max(w.ctx_lens) + 64, max_fuse_rows=w.batch * chunk)
     import torch
     last_fused = None
     for pos0 in range(0, max(w.ctx_lens), chunk):

@@ -9,7 +9,7 @@ import pytest
 import oracle as O
 import synth
 from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, MULTI_TILE, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16,
-                           GpuRun, f64, oracle_for, rel_err, tolerance)
+                           GpuSide, f64, oracle_for, rel_err, tolerance)
 
 pytestmark = pytest.mark.gpu
 GAP = 1e-2
@@ -19,7 +19,7 @@ WORKLOADS = [TINY, SMALL_HD128, SMALL_HD64, D10, G8, BLOCK1, BLOCK2]
 @pytest.fixture(scope="module", params=WORKLOADS, ids=lambda w: w.name)
 def run(request):
     w = request.param
-    g = GpuRun(w)
+    g = GpuSide(w)
     o = oracle_for(w, g.W)
     fused = g.fuse(w.ctx_lens)
     F = [o.fuse_context(b, synth.hidden_states(w, b, 0, n)) for b, n in enumerate(w.ctx_lens)]
@@ -126,7 +126,7 @@ def test_rope_off_block_is_mask_permutation_equivariant():
     reductions in a fixed order, hence the deterministic mode."""
     from paper_2606_02091_gb300 import FLAG_DETERMINISTIC, FLAG_NO_BLOCK_ROPE
     w = SMALL_HD64
-    g = GpuRun(w, flags=FLAG_NO_BLOCK_ROPE | FLAG_DETERMINISTIC)
+    g = GpuSide(w, flags=FLAG_NO_BLOCK_ROPE | FLAG_DETERMINISTIC)
     g.fuse(w.ctx_lens, want_fused=False)
     tok, logits, hidden = g.draft(synth.initial_tokens(w))
     o = oracle_for(w, g.W, rope_block=False)
@@ -145,7 +145,7 @@ def test_raw_fusion_ablation():
     """-Softmax (Table 2): alpha = W^fuse as is."""
     from paper_2606_02091_gb300 import FLAG_RAW_FUSION
     w = TINY
-    g = GpuRun(w, flags=FLAG_RAW_FUSION)
+    g = GpuSide(w, flags=FLAG_RAW_FUSION)
     fused = f64(g.fuse(w.ctx_lens))
     o = oracle_for(w, g.W, softmax_fusion=False)
     F = o.fuse_context(0, synth.hidden_states(w, 0, 0, w.ctx_lens[0]))
@@ -157,7 +157,7 @@ def test_empty_and_capacity_edges():
     import torch
     from paper_2606_02091_gb300 import DEVERR_CAPACITY
     w = SMALL_HD64
-    g = GpuRun(w, max_ctx=310)
+    g = GpuSide(w, max_ctx=310)
     g.fuse([0, 0], want_fused=False)
     assert g.lib.ctx_lens() == [0, 0]
     # an empty context still drafts (the block attends only to itself)
@@ -178,7 +178,7 @@ def test_empty_and_capacity_edges():
 def test_bad_token_is_flagged():
     from paper_2606_02091_gb300 import DEVERR_TOKEN
     w = SMALL_HD64
-    g = GpuRun(w)
+    g = GpuSide(w)
     g.fuse(w.ctx_lens, want_fused=False)
     g.draft([w.shape.vocab + 5, -1])
     assert g.lib.device_error() & DEVERR_TOKEN
@@ -188,7 +188,7 @@ def test_simt_gemm_agrees_with_tcgen05_gemm():
     """The two GEMM implementations give the same path within the bf16 tolerance."""
     from paper_2606_02091_gb300 import FLAG_SIMT_GEMM
     w = SMALL_HD128
-    a, b = GpuRun(w), GpuRun(w, flags=FLAG_SIMT_GEMM, weights=None)
+    a, b = GpuSide(w), GpuSide(w, flags=FLAG_SIMT_GEMM, weights=None)
     a.fuse(w.ctx_lens, want_fused=False)
     b.fuse(w.ctx_lens, want_fused=False)
     x_t = synth.initial_tokens(w)
@@ -203,7 +203,7 @@ def test_wide_token_tiles_match_oracle(w):
     """256 token rows per projection (batch 16, the widest tcgen05 token tile), block 32, and 288
     rows (two token tiles, the second ragged): fused context, cached K/V and the draft block
     against the oracle."""
-    g = GpuRun(w)
+    g = GpuSide(w)
     o = oracle_for(w, g.W)
     fused = f64(g.fuse(w.ctx_lens))
     for b, n in enumerate(w.ctx_lens):
@@ -244,7 +244,7 @@ def test_variant_matches_oracle(w, flags, kw):
     o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
     tol = tolerance(w)
     for want_fused in (True, False):
-        g = GpuRun(w, flags=flag, weights=W)
+        g = GpuSide(w, flags=flag, weights=W)
         fused = g.fuse(w.ctx_lens, want_fused=want_fused)
         assert g.lib.ctx_lens() == list(w.ctx_lens)
         if fused is not None:
@@ -271,7 +271,7 @@ def test_verify_from_logits_matches_oracle(w):
     integer results bit-exact, over several rounds on one context."""
     import torch
     s = w.shape
-    g = GpuRun(w)
+    g = GpuSide(w)
     rng = np.random.default_rng(21)
     B, V, bsz = s.block, s.vocab, w.batch
     for rnd in range(4):
@@ -304,7 +304,7 @@ def test_deterministic_mode_repeats_bit_for_bit(w):
     x_t = synth.initial_tokens(w)
     runs = []
     for flags in (FLAG_DETERMINISTIC, FLAG_DETERMINISTIC, 0):
-        g = GpuRun(w, flags=flags)
+        g = GpuSide(w, flags=flags)
         g.fuse(w.ctx_lens, want_fused=False)
         runs.append(g.draft(x_t))
         del g
@@ -329,7 +329,7 @@ def test_repeated_calls_replay_as_graphs():
     bsz, B = w.batch, s.block
     runs = []
     for reuse in (True, False):
-        g = GpuRun(w, flags=FLAG_DETERMINISTIC)
+        g = GpuSide(w, flags=FLAG_DETERMINISTIC)
         st = torch.cuda.Stream()
         dt = torch.bfloat16
         with torch.cuda.stream(st):

@@ -12,7 +12,7 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import SMALL_HD128, TINY, WIDE_B16, GpuRun
+from tests.harness import SMALL_HD128, TINY, WIDE_B16, GpuSide
 
 pytestmark = pytest.mark.gpu
 MARGIN = 1e-4
@@ -36,7 +36,7 @@ def _draw_ok(gpu_tok, log_w, u):
 
 def _sampled_run(w, T, seed, step0):
     import torch
-    g = GpuRun(w)
+    g = GpuSide(w)
     g.fuse(w.ctx_lens, want_fused=False)
     s = w.shape
     bsz = w.batch

@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 import synth
-from tests.harness import SMALL_HD128, GpuRun
+from tests.harness import SMALL_HD128, GpuSide
 
 
 def test_noalloc_rejects_more_rows_than_its_scratch():
@@ -29,7 +29,7 @@ def test_noalloc_argmax_matches_draft_block_on_two_calls():
     import torch
     from paper_2606_02091_gb300 import argmax_noalloc
     w = SMALL_HD128
-    g = GpuRun(w)
+    g = GpuSide(w)
     g.fuse(w.ctx_lens, want_fused=False)
     x_t = synth.initial_tokens(w)
     tok1, logits1, _ = g.draft(x_t)
