@@ -240,8 +240,9 @@ dflare_status dflare_verify_logits(dflare_ctx* ctx, const int32_t* draft_tokens_
  * Sampled decoding at temperature T (Table 1's temperature-1 rows). The paper does not state its
  * acceptance rule for sampling; these calls use the speculative-sampling rule of the works it
  * builds on. Random numbers are Philox4x64-10 streams (Salmon et al., SC'11): element v of
- * stream (purpose, step, row) is lane v mod 4 of the block at counter (1 + v/4, row, step,
- * purpose), key (seed, 0), mapped to ((x >> 41) + 1/2) * 2^-23. Purposes: 1 draft draws (row =
+ * stream (purpose, step, row) comes from word x = word (v/2) mod 4 of the block at counter
+ * (1 + v/8, row, step, purpose), key (seed, 0): ((x >> 41) + 1/2) * 2^-23 for even v,
+ * (((x >> 9) & 0x7FFFFF) + 1/2) * 2^-23 for odd v. Purposes: 1 draft draws (row =
  * b*(B-1) + k-1, v = token id), 2 acceptance draws (row = b, v = k-1), 3 replacement draws
  * (row = b, v = token id). `step_dev` is a uint64 device counter read by both calls;
  * dflare_verify_sampled adds 1 to it when it finishes, so a captured draft-verify graph draws

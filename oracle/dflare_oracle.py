@@ -298,10 +298,11 @@ def synthetic_target(draft, u, r, last, threshold: int):
 # target's distribution after the last block row. Draws use the Gumbel-max form
 # argmax_v (log w_v + G_v), G_v = -log(-log u_v), which samples v with probability w_v / sum w.
 #
-# Random numbers: the uniforms of stream (purpose, step, row) are lanes of Philox4x64-10
-# (Salmon, Moraes, Dror, Shaw, SC'11): element v is lane v mod 4 of the block at counter
-# (1 + v div 4, row, step, purpose) under key (seed, 0), mapped to ((x >> 41) + 1/2) 2^-23, a
-# value in (0, 1) that fp32 represents exactly.
+# Random numbers: the uniforms of stream (purpose, step, row) are cut from Philox4x64-10 words
+# (Salmon, Moraes, Dror, Shaw, SC'11): element v comes from word (v div 2) mod 4 of the block at
+# counter (1 + v div 8, row, step, purpose) under key (seed, 0), bits 63..41 for even v and
+# bits 31..9 for odd v, as (23-bit integer + 1/2) 2^-23, a value in (0, 1) that fp32 represents
+# exactly.
 
 RNG_DRAFT, RNG_ACCEPT, RNG_RESIDUAL = 1, 2, 3
 _M64 = (1 << 64) - 1
@@ -328,13 +329,21 @@ def philox4x64(counter, key, rounds: int = 10):
 def uniforms(seed: int, purpose: int, step: int, row: int, n: int):
     """u_0 .. u_{n-1} of stream (purpose, step, row), float64 values in (0, 1).
 
-    numpy's Philox bit generator computes the same Philox4x64-10 blocks; it advances the counter
-    before its first block, so it starts from word 0 = 0 to produce block 1 first.
+    Output word w of the stream is word w mod 4 of the Philox4x64-10 block at counter
+    (1 + w div 4, row, step, purpose) under key (seed, 0); it gives two uniforms, u_{2w} from its
+    bits 63..41 and u_{2w+1} from its bits 31..9, each as (23-bit integer + 1/2) 2^-23.
+    numpy's Philox bit generator computes the same blocks; it advances the counter before its
+    first block, so it starts from word 0 = 0 to produce block 1 first.
     """
     u64 = lambda *v: np.array([int(x) & _M64 for x in v], dtype=np.uint64)
     g = np.random.Philox(counter=u64(0, row, step, purpose), key=u64(seed, 0))
-    x = g.random_raw(int(n)) if n else np.zeros(0, np.uint64)
-    return ((x >> np.uint64(41)).astype(F64) + 0.5) * 2.0 ** -23
+    nw = (int(n) + 1) // 2
+    x = g.random_raw(nw) if nw else np.zeros(0, np.uint64)
+    hi = (x >> np.uint64(41)).astype(F64)
+    lo = ((x >> np.uint64(9)) & np.uint64(0x7FFFFF)).astype(F64)
+    bits = np.empty(2 * nw, F64)
+    bits[0::2], bits[1::2] = hi, lo
+    return (bits[:int(n)] + 0.5) * 2.0 ** -23
 
 
 def softmax_t(logits, temperature: float):

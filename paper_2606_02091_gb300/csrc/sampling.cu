@@ -10,10 +10,12 @@
 // draft is kept the extra token is drawn from the target's distribution after the last block row.
 //
 // Random numbers: Philox4x64-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy
-// as 1, 2, 3", SC'11), written here from that definition. Element v of stream (purpose, step,
-// row) is lane v mod 4 of the block at counter (1 + v / 4, row, step, purpose) under key
-// (seed, 0), mapped to ((x >> 41) + 1/2) 2^-23, a value in (0, 1) that fp32 holds exactly. The
-// step is read from a device counter that the verification advances, so a captured graph of a
+// as 1, 2, 3", SC'11), written here from that definition. Output word w of stream (purpose,
+// step, row) is word w mod 4 of the block at counter (1 + w / 4, row, step, purpose) under key
+// (seed, 0); it gives element 2w from its bits 63..41 and element 2w + 1 from its bits 31..9,
+// each as (23-bit integer + 1/2) 2^-23, a value in (0, 1) that fp32 holds exactly. One block
+// thus serves eight elements (the Philox rounds are the drafting kernel's main cost). The step
+// is read from a device counter that the verification advances, so a captured graph of a
 // draft-verify step draws fresh numbers on every replay.
 #include <math.h>
 
@@ -30,12 +32,16 @@ constexpr uint64_t kWeyl0 = 0x9E3779B97F4A7C15ull, kWeyl1 = 0xBB67AE8584CAA73Bul
 constexpr uint64_t kRngDraft = 1, kRngAccept = 2, kRngResidual = 3;
 constexpr int kNone = 0x7fffffff;
 constexpr int kU = 4;   // groups of four logits a thread loads at once in the vocabulary scans
+constexpr int kDrawU = 2;   // groups of eight logits (one Philox block each) per thread and iteration
 
-__device__ __forceinline__ float unit_from_bits(uint64_t x) {
+__device__ __forceinline__ float unit_from_bits(uint64_t x) {   // bits 63..41
     return ((float)(x >> 41) + 0.5f) * 0x1p-23f;
 }
+__device__ __forceinline__ float unit_from_low_bits(uint64_t x) {   // bits 31..9
+    return ((float)((uint32_t)(x >> 9) & 0x7FFFFFu) + 0.5f) * 0x1p-23f;
+}
 
-// The four uniforms of block `blk` of stream (purpose, step, row).
+// The eight uniforms of block `blk` of stream (purpose, step, row): elements 8 (blk - 1) .. + 7.
 __device__ __forceinline__ void philox_uniforms(uint64_t blk, uint64_t row, uint64_t step,
                                                 uint64_t purpose, uint64_t seed, float* u) {
     uint64_t c0 = blk, c1 = row, c2 = step, c3 = purpose, k0 = seed, k1 = 0;
@@ -53,9 +59,13 @@ __device__ __forceinline__ void philox_uniforms(uint64_t blk, uint64_t row, uint
         c3 = lo0;
     }
     u[0] = unit_from_bits(c0);
-    u[1] = unit_from_bits(c1);
-    u[2] = unit_from_bits(c2);
-    u[3] = unit_from_bits(c3);
+    u[1] = unit_from_low_bits(c0);
+    u[2] = unit_from_bits(c1);
+    u[3] = unit_from_low_bits(c1);
+    u[4] = unit_from_bits(c2);
+    u[5] = unit_from_low_bits(c2);
+    u[6] = unit_from_bits(c3);
+    u[7] = unit_from_low_bits(c3);
 }
 
 __device__ __forceinline__ float gumbel(float u) { return -logf(-logf(u)); }
@@ -122,7 +132,7 @@ __device__ __forceinline__ void load4(const float* p, int i, int c1, bool vec, f
 }
 
 // ---------------------------------------------------------------------------------- drafting
-// Grid (chunks, rows), chunk a multiple of 4: every thread takes groups of four logits and the
+// Grid (chunks, rows), chunk a multiple of 8: every thread takes groups of eight logits and the
 // one Philox block that covers them.
 __global__ void __launch_bounds__(256) sample_kernel(const float* __restrict__ logits, int V, int rows,
                                                      int chunk, float inv_t, uint64_t seed,
@@ -138,21 +148,25 @@ __global__ void __launch_bounds__(256) sample_kernel(const float* __restrict__ l
     const bool vec = (V & 3) == 0;
     float bv = -INFINITY;
     int bi = kNone;
-    // kU groups of four logits per thread and iteration, all loads issued before the first
-    // Philox block (ids ascend within a thread, so ">" keeps the lowest id of equal scores)
-    const int stride = blockDim.x * 4;
-    for (int base = c0 + threadIdx.x * 4; base < c1; base += stride * kU) {
-        float x[kU][4];
+    // kDrawU groups of eight logits (one Philox block each) per thread and iteration, all loads
+    // issued before the first block (ids ascend within a thread, so ">" keeps the lowest id of
+    // equal scores)
+    const int stride = blockDim.x * 8;
+    for (int base = c0 + threadIdx.x * 8; base < c1; base += stride * kDrawU) {
+        float x[kDrawU][8];
 #pragma unroll
-        for (int g = 0; g < kU; ++g) load4(p, base + g * stride, c1, vec, x[g]);
+        for (int g = 0; g < kDrawU; ++g) {
+            load4(p, base + g * stride, c1, vec, x[g]);
+            load4(p, base + g * stride + 4, c1, vec, x[g] + 4);
+        }
 #pragma unroll
-        for (int g = 0; g < kU; ++g) {
+        for (int g = 0; g < kDrawU; ++g) {
             const int i = base + g * stride;
             if (i >= c1) break;
-            float u[4];
-            philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)row, step, kRngDraft, seed, u);
+            float u[8];
+            philox_uniforms(1 + (uint64_t)(i >> 3), (uint64_t)row, step, kRngDraft, seed, u);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
+            for (int e = 0; e < 8; ++e) {
                 const float sc = x[g][e] * inv_t + gumbel(u[e]);
                 if (sc > bv) {
                     bv = sc;
@@ -284,9 +298,9 @@ __global__ void __launch_bounds__(32) spec_accept_kernel(const float* __restrict
             const float2 sq = row_stats(part, batch * B + dr, chunks);
             const float p = expf(target[(size_t)tr * V + d] * inv_t - st.x) / st.y;
             const float q = expf(draft_logits[(size_t)dr * V + d] * inv_t - sq.x) / sq.y;
-            float u[4];
-            philox_uniforms(1 + (uint64_t)(j >> 2), (uint64_t)b, step, kRngAccept, seed, u);
-            rej = !(u[j & 3] * q < p);
+            float u[8];
+            philox_uniforms(1 + (uint64_t)(j >> 3), (uint64_t)b, step, kRngAccept, seed, u);
+            rej = !(u[j & 7] * q < p);
         }
     }
     const unsigned mask = __ballot_sync(0xffffffffu, rej);
@@ -317,22 +331,26 @@ __global__ void __launch_bounds__(256) spec_resample_kernel(
     const bool vec = (V & 3) == 0;
     float bv = -INFINITY;
     int bi = kNone;
-    const int stride = blockDim.x * 4;
-    for (int base = c0 + threadIdx.x * 4; base < c1; base += stride * kU) {
-        float xt[kU][4], xq[kU][4];
+    const int stride = blockDim.x * 8;
+    for (int base = c0 + threadIdx.x * 8; base < c1; base += stride * kDrawU) {
+        float xt[kDrawU][8], xq[kDrawU][8];
 #pragma unroll
-        for (int g = 0; g < kU; ++g) {
+        for (int g = 0; g < kDrawU; ++g) {
             load4(lt, base + g * stride, c1, vec, xt[g]);
-            if (resid) load4(lq, base + g * stride, c1, vec, xq[g]);
+            load4(lt, base + g * stride + 4, c1, vec, xt[g] + 4);
+            if (resid) {
+                load4(lq, base + g * stride, c1, vec, xq[g]);
+                load4(lq, base + g * stride + 4, c1, vec, xq[g] + 4);
+            }
         }
 #pragma unroll
-        for (int g = 0; g < kU; ++g) {
+        for (int g = 0; g < kDrawU; ++g) {
             const int i = base + g * stride;
             if (i >= c1) break;
-            float u[4];
-            philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)b, step, kRngResidual, seed, u);
+            float u[8];
+            philox_uniforms(1 + (uint64_t)(i >> 3), (uint64_t)b, step, kRngResidual, seed, u);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
+            for (int e = 0; e < 8; ++e) {
                 float w = expf(xt[g][e] * inv_t - st.x) / st.y;
                 if (resid) w -= expf(xq[g][e] * inv_t - sq.x) / sq.y;
                 if (w > 0.f) {
@@ -359,11 +377,11 @@ __global__ void __launch_bounds__(256) spec_resample_kernel(
                 float best = -INFINITY;
                 tok = 0;
                 for (int i = 0; i < V; ++i) {
-                    float u[4];
-                    philox_uniforms(1 + (uint64_t)(i >> 2), (uint64_t)s, step, kRngResidual, seed, u);
+                    float u[8];
+                    philox_uniforms(1 + (uint64_t)(i >> 3), (uint64_t)s, step, kRngResidual, seed, u);
                     const float w = expf(l[i] * inv_t - t2.x) / t2.y;
                     if (w > 0.f) {
-                        const float sc = logf(w) + gumbel(u[i & 3]);
+                        const float sc = logf(w) + gumbel(u[i & 7]);
                         if (sc > best) {
                             best = sc;
                             tok = i;
@@ -382,13 +400,13 @@ __global__ void __launch_bounds__(256) spec_resample_kernel(
     }
 }
 
-// chunk size (a multiple of 4, at least 1024) and count for `rows` rows of V entries, about
+// chunk size (a multiple of 8, at least 1024) and count for `rows` rows of V entries, about
 // per_sm CTAs per SM (the scans that end in one packed atomicMax per CTA use two)
 void chunking(int V, int rows, int sms, int max_chunks, int per_sm, int* chunk, int* chunks) {
     int n = std::max(1, (per_sm * sms + rows - 1) / rows);
     n = std::min(n, max_chunks);
     int c = (V + n - 1) / n;
-    c = std::max(1024, ((c + 3) / 4) * 4);
+    c = std::max(1024, ((c + 7) / 8) * 8);   // a multiple of 8: no Philox block straddles chunks
     *chunk = c;
     *chunks = (V + c - 1) / c;
 }

@@ -25,13 +25,15 @@ def _chi2(counts, probs):
 
 @pytest.mark.parametrize("seed,purpose,step,row", [(0, 1, 0, 0), (7, 2, 3, 11), (2 ** 63 + 5, 3, 2 ** 40, 2 ** 33)])
 def test_uniform_stream_is_philox4x64_10(seed, purpose, step, row):
-    """uniforms() (numpy's Philox) and philox4x64() (written from the definition) agree, lane by
-    lane, on the counter layout (1 + v div 4, row, step, purpose), key (seed, 0)."""
+    """uniforms() (numpy's Philox) and philox4x64() (written from the definition) agree on the
+    stream layout: element v comes from word (v div 2) mod 4 of the block at counter
+    (1 + v div 8, row, step, purpose), key (seed, 0), bits 63..41 for even v, 31..9 for odd v."""
     n = 23
     u = O.uniforms(seed, purpose, step, row, n)
     for v in range(n):
-        x = O.philox4x64([1 + v // 4, row, step, purpose], [seed, 0])[v % 4]
-        assert u[v] == ((x >> 41) + 0.5) * 2.0 ** -23
+        x = O.philox4x64([1 + v // 8, row, step, purpose], [seed, 0])[(v // 2) % 4]
+        bits = x >> 41 if v % 2 == 0 else (x >> 9) & 0x7FFFFF
+        assert u[v] == (bits + 0.5) * 2.0 ** -23
 
 
 def test_philox_rounds_and_key_schedule_matter():
@@ -50,6 +52,11 @@ def test_uniforms_are_exact_fp32_values_in_open_unit_interval():
     # mean 1/2 and variance 1/12 within 5 standard errors
     assert abs(u.mean() - 0.5) < 5 * np.sqrt(1 / 12 / u.size)
     assert abs(u.var() - 1 / 12) < 5 * np.sqrt(1 / 180 / u.size)
+    # the two uniforms cut from one 64-bit word (its high and low bits) are uncorrelated
+    hi, lo = u[0::2], u[1::2]
+    assert abs(np.corrcoef(hi, lo)[0, 1]) < 5 / np.sqrt(hi.size)
+    for half in (hi, lo):
+        assert abs(half.mean() - 0.5) < 5 * np.sqrt(1 / 12 / half.size)
 
 
 def test_gumbel_draw_frequencies_follow_the_weights():
