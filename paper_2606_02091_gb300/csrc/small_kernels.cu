@@ -247,8 +247,9 @@ cudaError_t launch_argmax(dflare_ctx* c, const float* logits, int rows, int32_t*
                           cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     const int V = c->cfg.vocab;
-    // enough CTAs to fill the GPU: chunks of at least 4096 ids, a multiple of 1024
-    int chunks = std::max(1, (2 * c->num_sms + rows - 1) / rows);
+    // about four CTAs per SM (measured against two: 0.5207 -> 0.5195 ms per Qwen3-4B-shaped step;
+    // one: 0.5225 ms): chunks of at least 4096 ids, a multiple of 1024
+    int chunks = std::max(1, (4 * c->num_sms + rows - 1) / rows);
     int chunk = (V + chunks - 1) / chunks;
     chunk = std::max(4096, ((chunk + 1023) / 1024) * 1024);
     chunks = (V + chunk - 1) / chunk;
