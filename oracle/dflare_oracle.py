@@ -106,12 +106,13 @@ def fuse_context(hidden, alpha, fuse_gain, eps: float, store=exact):
     """
     hidden = np.asarray(hidden, F64)
     D, T = alpha.shape
+    # s^(i) = sum_j alpha[i, j] h^(j) for every i at once: the [D][T] weights times the T target
+    # states taken as a [T][n d] matrix
+    rest = hidden.shape[1:]
+    s = (np.asarray(alpha, F64) @ hidden.reshape(T, int(np.prod(rest)))).reshape((D,) + rest)
     out = np.empty((D,) + hidden.shape[1:], F64)
     for i in range(D):
-        s = np.zeros(hidden.shape[1:], F64)
-        for j in range(T):
-            s += alpha[i, j] * hidden[j]
-        out[i] = store(rms_norm(s, fuse_gain[i], eps))
+        out[i] = store(rms_norm(s[i], fuse_gain[i], eps))
     return out
 
 
