@@ -336,8 +336,12 @@ dflare_status dflare_synthetic_target(const int32_t* draft_tokens_dev, const uin
  * DFLARE_NOALLOC_MAX_ROWS rows, held by every GPU that loads the library until the process
  * exits); it calls no cudaMalloc, cudaFree or allocating library routine.
  * - rows > DFLARE_NOALLOC_MAX_ROWS returns DFLARE_ECAPACITY (message in dflare_last_error(NULL)).
- * - The first call on a device looks up the scratch array's device address with that device
- *   current; make that first call before capturing a stream into a CUDA graph.
+ * - A call made outside stream capture looks up the scratch array's device address (and the
+ *   SM count) with the calling thread's current device; a call made while `stream` is being
+ *   captured uses the values of the last call outside capture on that device. So make the first
+ *   call on a device before capturing a stream into a CUDA graph (a first call inside a capture
+ *   returns DFLARE_ECUDA), and after cudaDeviceReset make one call outside capture before
+ *   capturing again: the reset invalidates the address held for capture.
  * - Every call on a device shares the same scratch array, which keeps the last call's contents;
  *   each call clears the part it uses on `stream` before its kernel. Calls that overlap on the
  *   GPU (on different streams, or from several host threads) race on the scratch and give wrong

@@ -7,6 +7,8 @@
 // e.g. a target model's verification logits.
 #include <math.h>
 
+#include <algorithm>
+#include <cstdint>
 #include <mutex>
 #include <string>
 
@@ -24,26 +26,36 @@ namespace {
 struct Scratch {
     unsigned long long* slot = nullptr;
     unsigned int* count = nullptr;
+    int num_sms = 0;
 };
 
-// Device addresses of the two arrays, looked up once per device with that device current
-// (in host code the symbols only name host-side stand-ins).
+// Device addresses of the two arrays (in host code the symbols only name host-side stand-ins)
+// and the SM count, per device. A call made outside stream capture looks them up again with the
+// device current (cheap), so a context rebuilt after cudaDeviceReset gets the new addresses; a
+// call made during capture uses the values of the last call outside capture on that device.
 std::mutex g_mu;
 Scratch g_scratch[64];
 
-cudaError_t scratch_for_current_device(Scratch* out) {
+cudaError_t scratch_for_current_device(cudaStream_t stream, Scratch* out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    e = cudaStreamIsCapturing(stream, &cs);
+    if (e != cudaSuccess) return e;
     std::lock_guard<std::mutex> lk(g_mu);
-    if (!g_scratch[dev].slot) {
+    if (cs == cudaStreamCaptureStatusNone) {
         Scratch s;
         e = cudaGetSymbolAddress(reinterpret_cast<void**>(&s.slot), g_noalloc_slot);
         if (e != cudaSuccess) return e;
         e = cudaGetSymbolAddress(reinterpret_cast<void**>(&s.count), g_noalloc_count);
         if (e != cudaSuccess) return e;
+        e = cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
         g_scratch[dev] = s;
+    } else if (!g_scratch[dev].slot) {
+        return cudaErrorStreamCaptureUnsupported;   // first call on this device inside a capture
     }
     *out = g_scratch[dev];
     return cudaSuccess;
@@ -55,12 +67,17 @@ __device__ __forceinline__ uint32_t order_key(float v) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+__device__ __forceinline__ void take(float q, int i, float& bv, int& bi) {
+    if (q > bv) { bv = q; bi = i; }   // NaN never compares greater; equal values keep the lower id
+}
+
 // Grid (chunks, rows): each CTA reduces one vocabulary chunk of one row (lowest index among
 // equal maxima) and folds (ordered value, ~index) into the row's slot with a 64-bit atomicMax;
-// the last CTA to arrive writes the token ids. NaN entries are never chosen; a row with no value
-// above -inf gets its first -inf entry (id 0 when every entry is NaN).
+// the last CTA to arrive writes the token ids. With vec4 (rows 16-byte aligned, chunk a multiple
+// of 4) every thread keeps four 16-byte loads in flight. NaN entries are never chosen; a row
+// with no value above -inf gets its first -inf entry (id 0 when every entry is NaN).
 __global__ void __launch_bounds__(256) argmax_noalloc_kernel(const float* __restrict__ logits,
-                                                             int V, int rows, int chunk,
+                                                             int V, int rows, int chunk, int vec4,
                                                              unsigned long long* slot,
                                                              unsigned int* count,
                                                              int32_t* __restrict__ tokens) {
@@ -72,9 +89,27 @@ __global__ void __launch_bounds__(256) argmax_noalloc_kernel(const float* __rest
     const float* p = logits + (size_t)row * V;
     float bv = -INFINITY;
     int bi = 0x7fffffff;
-    for (int i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-        const float q = p[i];
-        if (q > bv) { bv = q; bi = i; }
+    if (vec4) {
+        const float4* p4 = reinterpret_cast<const float4*>(p);
+        const int q0 = c0 >> 2, q1 = c1 >> 2;   // whole float4 groups; V % 4 == 0 here
+        for (int q = q0 + threadIdx.x; q < q1; q += 4 * blockDim.x) {
+            float4 f[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int qq = q + j * blockDim.x;
+                f[j] = qq < q1 ? __ldg(p4 + qq) : make_float4(NAN, NAN, NAN, NAN);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int i = 4 * (q + j * blockDim.x);
+                take(f[j].x, i, bv, bi);
+                take(f[j].y, i + 1, bv, bi);
+                take(f[j].z, i + 2, bv, bi);
+                take(f[j].w, i + 3, bv, bi);
+            }
+        }
+    } else {
+        for (int i = c0 + threadIdx.x; i < c1; i += blockDim.x) take(p[i], i, bv, bi);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -129,16 +164,22 @@ extern "C" dflare_status dflare_argmax_noalloc(const float* logits_dev, int rows
         return DFLARE_ECAPACITY;
     }
     dfl::Scratch sc;
-    cudaError_t e = dfl::scratch_for_current_device(&sc);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = dfl::scratch_for_current_device(s, &sc);
     if (e == cudaSuccess) e = cudaMemsetAsync(sc.slot, 0, (size_t)rows * sizeof(unsigned long long), s);
     if (e == cudaSuccess) e = cudaMemsetAsync(sc.count, 0, sizeof(unsigned int), s);
     if (e == cudaSuccess) {
-        int chunks = (vocab + 8191) / 8192;
-        if (chunks < 1) chunks = 1;
-        const int chunk = (vocab + chunks - 1) / chunks;
+        // about four CTAs of 256 threads per SM over all rows, at least 1024 logits per CTA
+        const int target = 4 * (sc.num_sms > 0 ? sc.num_sms : 1);
+        int chunks = (target + rows - 1) / rows;
+        chunks = std::max(1, std::min(chunks, (vocab + 1023) / 1024));
+        const bool vec4 = vocab % 4 == 0 && (reinterpret_cast<uintptr_t>(logits_dev) & 15u) == 0;
+        int chunk = (vocab + chunks - 1) / chunks;
+        if (vec4) chunk = (chunk + 3) & ~3;
+        chunks = (vocab + chunk - 1) / chunk;
         dfl::argmax_noalloc_kernel<<<dim3(chunks, rows), 256, 0, s>>>(logits_dev, vocab, rows, chunk,
-                                                                       sc.slot, sc.count, tokens_dev);
+                                                                       vec4 ? 1 : 0, sc.slot, sc.count,
+                                                                       tokens_dev);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) {

@@ -5,6 +5,8 @@ compiled into the library. The GPU test checks it against the tokens dflare_draf
 from the same logits, on two calls in a row (the second call reuses the scratch the first one
 left behind)."""
 import ctypes
+import os
+import re
 
 import numpy as np
 import pytest
@@ -22,6 +24,13 @@ def test_noalloc_rejects_more_rows_than_its_scratch():
     assert st == _lib.DFLARE_ECAPACITY
     assert b"DFLARE_NOALLOC_MAX_ROWS" in lib.dflare_last_error(None)
     assert lib.dflare_argmax_noalloc(None, 1, 10, fake, None) == _lib.DFLARE_EINVAL
+
+
+def test_noalloc_source_calls_no_allocator():
+    """The entry point's translation unit calls no CUDA allocation or free routine."""
+    src = open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                            "paper_2606_02091_gb300", "csrc", "argmax_noalloc.cu")).read()
+    assert not re.search(r"\bcu(da)?(Mem)?(Malloc|Free|Alloc)\w*\s*\(", src)
 
 
 @pytest.mark.gpu
@@ -62,3 +71,54 @@ def test_noalloc_argmax_rows_without_a_finite_maximum():
     out = torch.full((5,), -1, dtype=torch.int32, device="cuda")
     argmax_noalloc(dev, out)
     assert out.cpu().tolist() == [0, 3, 0, 17, V - 1]
+
+
+@pytest.mark.gpu
+def test_noalloc_argmax_across_vocabulary_chunks_allocates_nothing():
+    """A 151936-token vocabulary (many CTAs per row, merged through the packed 64-bit atomicMax):
+    equal maxima in different chunks (lowest id), a maximum only in the last, partial chunk, rows
+    of -inf with NaN in one chunk, random rows; two calls in a row on different logits. After a
+    warm-up call, repeated calls change neither torch's allocated bytes nor the device's free
+    memory."""
+    import torch
+    from paper_2606_02091_gb300 import argmax_noalloc
+    V = 151936
+    rng = np.random.default_rng(7)
+
+    def case(seed):
+        lg = np.random.default_rng(seed).standard_normal((8, V)).astype(np.float32)
+        want = [int(np.argmax(r)) for r in lg]
+        lg[0, 100] = lg[0, 140000] = 60.0
+        want[0] = 100
+        lg[1, V - 3] = 60.0
+        want[1] = V - 3
+        lg[2] = -np.inf
+        lg[2, 50000:51000] = np.nan
+        want[2] = 0
+        lg[3] = -np.inf
+        lg[3, :10] = np.nan
+        lg[3, 90000:90100] = np.nan
+        want[3] = 10
+        top = int(rng.integers(1, V))
+        lg[4, [top, 7, V - 1]] = 70.0
+        want[4] = min(top, 7)
+        lg[5, 3] = np.nan
+        lg[5, 151935] = 80.0
+        want[5] = 151935
+        return lg, want
+
+    out = torch.full((8,), -1, dtype=torch.int32, device="cuda")
+    for seed in (1, 2):
+        lg, want = case(seed)
+        dev = torch.from_numpy(lg).cuda()
+        argmax_noalloc(dev, out)
+        assert out.cpu().tolist() == want, seed
+    torch.cuda.synchronize()
+    alloc0 = torch.cuda.memory_allocated()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(20):
+        argmax_noalloc(dev, out)
+    torch.cuda.synchronize()
+    assert torch.cuda.memory_allocated() == alloc0
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert out.cpu().tolist() == want
