@@ -183,172 +183,204 @@ __global__ void __launch_bounds__(256) fuse_layers_kernel(
     }
 }
 
-// Many positions (context fill): a persistent grid of CTAs of d/8 threads walks the positions (no
-// cluster). The T target rows of each position (d contiguous elements each) stream through shared
-// memory as 1-D bulk copies issued by one thread, kRB rows per stage, kNS - 1 stages in flight; the
-// stage sequence runs on across positions, so the next position's first rows load while the
-// current one is reduced and stored. Completion is tracked by an mbarrier per stage (bounded
-// waits). Thread t forms the D (<= DMAX) draft-layer sums of features [8t, 8t + 8) in registers,
-// and the CTA reduces the D sums of squares in one pass (warp shuffles, then the warps' partials
-// in order).
-constexpr int kRB = 8;   // target rows per stage
-constexpr int kNS = 2;   // stages (kNS - 1 in flight while one is summed)
+// Many positions (context fill): a persistent grid of one CTA per SM walks the positions (no
+// cluster). Warp-specialised: the last warp's first thread streams the T target rows of each
+// position (d contiguous elements each) through a ring of `ns` shared-memory stages of kRB rows as
+// 1-D bulk copies, the stage sequence running on across positions; the other warps (one thread
+// per 8 features) consume the stages. Each stage has a "full" mbarrier (the copies landed) and an
+// "empty" one that every consumer warp arrives on once it has read the stage, which is what the
+// producer waits for before refilling it: no CTA barrier per stage, and up to ns - 1 stages in
+// flight while one is summed. Thread t forms the D (<= DMAX) draft-layer sums of features
+// [8t, 8t + 8) in registers; at the end of a position the consumer warps reduce the D sums of
+// squares (warp shuffles, then the warps' partials in order) behind a named barrier. Every wait
+// is bounded; a CTA that times out sets DFLARE_DEVERR_TIMEOUT and stops.
+constexpr int kRB = 4;          // target rows per stage
+constexpr int kMaxNS = 16;      // most stages in the ring
+constexpr uint64_t kFillWaitNs = 2000000000ull;
+
+__device__ __forceinline__ bool fill_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+    const uint64_t t0 = globaltimer_ns();
+    for (int it = 0;; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if ((it & 63) == 63) {
+            if (*abort_flag) return false;
+            if (globaltimer_ns() - t0 > kFillWaitNs) {
+                *abort_flag = 1;
+                return false;
+            }
+        }
+    }
+}
+
 template <class T, int DMAX>
-__global__ void __launch_bounds__(512) fuse_rows_kernel(
+__global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
     const T* __restrict__ H, const float* __restrict__ alpha, const T* __restrict__ gain,
     T* __restrict__ F, T* __restrict__ F_out, const int32_t* __restrict__ app_cnt, int D, int Tn,
-    int batch, int n_max, int d, long long f_layer_rows, float eps, uint32_t* err) {
+    int batch, int n_max, int d, long long f_layer_rows, float eps, int ns, uint32_t* err) {
     pdl_trigger();
-    extern __shared__ __align__(128) uint8_t stage_mem[];   // [kNS][kRB][d]
-    __shared__ float s_alpha[16 * 64];
+    extern __shared__ __align__(128) uint8_t stage_mem[];   // [ns][kRB][d]
+    __shared__ __align__(16) float s_alpha[64 * DMAX];       // [j][i] (Tn <= 64)
     __shared__ float red[16][DMAX];
     __shared__ float inv_s[DMAX];
-    __shared__ __align__(8) uint64_t bar[kNS];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
-    const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(&bar[0]);
+    __shared__ __align__(8) uint64_t full_bar[kMaxNS], empty_bar[kMaxNS];
+    __shared__ int abort_flag;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int n_cw = (int)(blockDim.x >> 5) - 1;   // consumer warps; the last warp produces
+    const int n_ct = n_cw * 32;
+    const uint32_t fb0 = (uint32_t)__cvta_generic_to_shared(&full_bar[0]);
+    const uint32_t eb0 = (uint32_t)__cvta_generic_to_shared(&empty_bar[0]);
     const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(stage_mem);
     if (tid == 0) {
-        for (int i = 0; i < kNS; ++i)
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar0 + 8u * i) : "memory");
+        for (int i = 0; i < ns; ++i) {
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(fb0 + 8u * i) : "memory");
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(eb0 + 8u * i), "r"(n_cw) : "memory");
+        }
+        abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     pdl_wait();
-    for (int k = tid; k < D * Tn; k += blockDim.x) s_alpha[k] = alpha[k];
+    for (int k = tid; k < D * Tn; k += blockDim.x) {
+        const int i = k / Tn, j = k % Tn;
+        s_alpha[j * DMAX + i] = alpha[k];
+    }
+    for (int k = tid; k < Tn * DMAX; k += blockDim.x)
+        if (k % DMAX >= D) s_alpha[k] = 0.f;
     __syncthreads();
-    const int e0 = tid * 8;
-    const bool act = e0 < d;
+    volatile int* abrt = &abort_flag;
     const int n_pos = batch * n_max;
     const size_t lstride = (size_t)n_pos * d;
     const uint32_t row_bytes = (uint32_t)(d * sizeof(T));
-    const T* stg = reinterpret_cast<const T*>(stage_mem);
     const int nst = (Tn + kRB - 1) / kRB;   // stages per position
     // this CTA's positions pid = blockIdx.x + k * gridDim.x that have rows to append
+    auto valid = [&](int pid) { return pid % n_max < app_cnt[pid / n_max]; };
     auto next_pos = [&](int pid) {
         for (pid += gridDim.x; pid < n_pos; pid += gridDim.x)
-            if (pid % n_max < app_cnt[pid / n_max]) return pid;
+            if (valid(pid)) return pid;
         return n_pos;
     };
     int first = (int)blockIdx.x;
-    if (first < n_pos && !(first % n_max < app_cnt[first / n_max])) first = next_pos(first);
-    // stage stream: (position, stage within the position); g counts stages (buffer g % kNS)
-    int ipos = first, ik = 0, g_issue = 0;
-    auto issue_next = [&]() {   // thread 0 only
-        if (ipos >= n_pos) return;
-        const int st = g_issue % kNS, j0 = ik * kRB, nr = min(kRB, Tn - j0);
-        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar0 + 8u * st),
-                     "r"((uint32_t)nr * row_bytes)
-                     : "memory");
-        for (int u = 0; u < nr; ++u)
-            asm volatile(
-                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                    sbase + (uint32_t)(st * kRB + u) * row_bytes),
-                "l"(H + (size_t)(j0 + u) * lstride + (size_t)ipos * d), "r"(row_bytes), "r"(bar0 + 8u * st)
-                : "memory");
-        ++g_issue;
-        if (++ik == nst) {
-            ik = 0;
-            ipos = next_pos(ipos);
-        }
-    };
-    if (tid == 0)
-        for (int i = 0; i < kNS - 1; ++i) issue_next();
-    int g = 0;   // stages consumed
-    bool ok = true;
-    for (int pid = first; pid < n_pos && ok; pid = next_pos(pid)) {
-        const int b = pid / n_max, r = pid % n_max;
-        float acc[DMAX][8];
-#pragma unroll
-        for (int i = 0; i < DMAX; ++i)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
-        for (int k = 0; k < nst; ++k, ++g) {
-            const int st = g % kNS;
-            if (tid == 0) issue_next();   // stage g + kNS - 1, into the buffer freed after g - 1
-            bool landed = false;
-            {
-                const uint64_t t0 = globaltimer_ns();
-                while (true) {
-                    uint32_t done;
-                    asm volatile(
-                        "{\n\t.reg .pred p;\n\t"
-                        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-                        "selp.u32 %0, 1, 0, p;\n\t}"
-                        : "=r"(done)
-                        : "r"(bar0 + 8u * st), "r"((uint32_t)((g / kNS) & 1))
-                        : "memory");
-                    if (done) { landed = true; break; }
-                    if (globaltimer_ns() - t0 > 2000000000ull) break;
-                }
-            }
-            if (__syncthreads_or(!landed)) {
-                if (tid == 0) {
-                    atomicOr(err, DFLARE_DEVERR_TIMEOUT);
-                    // copies still in flight land before the CTA exits (again bounded)
-                    for (int q = g; q < g_issue; ++q) {
-                        const uint64_t t1 = globaltimer_ns();
-                        uint32_t done = 0;
-                        while (!done && globaltimer_ns() - t1 < 2000000000ull)
-                            asm volatile(
-                                "{\n\t.reg .pred p;\n\t"
-                                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-                                "selp.u32 %0, 1, 0, p;\n\t}"
-                                : "=r"(done)
-                                : "r"(bar0 + 8u * (q % kNS)), "r"((uint32_t)((q / kNS) & 1))
-                                : "memory");
+    if (first < n_pos && !valid(first)) first = next_pos(first);
+
+    if (warp == n_cw) {
+        // ---------------- producer: one thread streams every stage of every position in turn
+        if (lane == 0) {
+            int g = 0;
+            bool ok = true;
+            for (int pid = first; pid < n_pos && ok; pid = next_pos(pid)) {
+                for (int k = 0; k < nst; ++k, ++g) {
+                    const int st = g % ns, use = g / ns;
+                    if (use > 0 && !fill_wait(eb0 + 8u * st, (uint32_t)((use - 1) & 1), abrt)) {
+                        ok = false;
+                        break;
                     }
+                    const int j0 = k * kRB, nr = min(kRB, Tn - j0);
+                    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb0 + 8u * st),
+                                 "r"((uint32_t)nr * row_bytes)
+                                 : "memory");
+                    for (int u = 0; u < nr; ++u)
+                        asm volatile(
+                            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                                sbase + (uint32_t)(st * kRB + u) * row_bytes),
+                            "l"(H + (size_t)(j0 + u) * lstride + (size_t)pid * d), "r"(row_bytes),
+                            "r"(fb0 + 8u * st)
+                            : "memory");
                 }
-                ok = false;
-                break;
             }
-            if (act) {
+            // after a timeout: every issued copy lands before the CTA exits (bounded again)
+            if (!ok || *abrt) {
+                volatile int never = 0;
+                for (int q = max(0, g - ns); q < g; ++q)
+                    fill_wait(fb0 + 8u * (q % ns), (uint32_t)((q / ns) & 1), &never);
+                atomicOr(err, DFLARE_DEVERR_TIMEOUT);
+            }
+        }
+    } else {
+        // ---------------- consumers: thread t owns features [8t, 8t + 8)
+        const int e0 = tid * 8;
+        const bool act = e0 < d;
+        const T* stg = reinterpret_cast<const T*>(stage_mem);
+        int g = 0;
+        bool ok = true;
+        for (int pid = first; pid < n_pos && ok; pid = next_pos(pid)) {
+            const int b = pid / n_max, r = pid % n_max;
+            float acc[DMAX][8];
 #pragma unroll
-                for (int u = 0; u < kRB; ++u) {
-                    const int j = k * kRB + u;
-                    if (j >= Tn) break;
-                    float h[8];
-                    load8(stg + (size_t)(st * kRB + u) * d + e0, h);
+            for (int i = 0; i < DMAX; ++i)
 #pragma unroll
-                    for (int i = 0; i < DMAX; ++i) {
-                        if (i < D) {
-                            const float a = s_alpha[i * Tn + j];
+                for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
+            for (int k = 0; k < nst; ++k, ++g) {
+                const int st = g % ns;
+                if (!fill_wait(fb0 + 8u * st, (uint32_t)((g / ns) & 1), abrt)) {
+                    ok = false;
+                    break;
+                }
+                if (act) {
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a, h[e], acc[i][e]);
+                    for (int u = 0; u < kRB; ++u) {
+                        const int j = k * kRB + u;
+                        if (j >= Tn) break;
+                        float h[8], a[DMAX];
+                        load8(stg + (size_t)(st * kRB + u) * d + e0, h);
+#pragma unroll
+                        for (int i = 0; i < DMAX; i += 4) {
+                            const float4 a4 = *reinterpret_cast<const float4*>(&s_alpha[j * DMAX + i]);
+                            a[i] = a4.x;
+                            a[i + 1] = a4.y;
+                            a[i + 2] = a4.z;
+                            a[i + 3] = a4.w;
                         }
+#pragma unroll
+                        for (int i = 0; i < DMAX; ++i)
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a[i], h[e], acc[i][e]);
                     }
                 }
+                __syncwarp();
+                if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(eb0 + 8u * st) : "memory");
             }
-            __syncthreads();   // stage st is read before it is refilled
-        }
-        if (!ok) break;
-#pragma unroll
-        for (int i = 0; i < DMAX; ++i) {
-            float v = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) v = fmaf(acc[i][e], acc[i][e], v);
-            v = warp_sum(v);
-            if (lane == 0) red[warp][i] = v;
-        }
-        __syncthreads();
-        if (tid < D) {
-            float tot = 0.f;
-            for (int w = 0; w < nw; ++w) tot += red[w][tid];
-            inv_s[tid] = inv_rms(tot, d, eps);
-        }
-        __syncthreads();
-        if (act) {
+            // the consumer warps leave the position loop together: a warp whose wait ran out sets
+            // the abort flag, which every other consumer sees at the barrier below
+            asm volatile("bar.sync 1, %0;" ::"r"(n_ct) : "memory");
+            if (!ok || *abrt) break;
 #pragma unroll
             for (int i = 0; i < DMAX; ++i) {
-                if (i >= D) break;
-                float gg[8], o[8];
-                load8(gain + (size_t)i * d + e0, gg);
-                const float inv = inv_s[i];
+                float v = 0.f;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) o[e] = gg[e] * (acc[i][e] * inv);
-                store8(F + ((size_t)i * f_layer_rows + pid) * d + e0, o);
-                if (F_out) store8(F_out + (((size_t)i * batch + b) * n_max + r) * d + e0, o);
+                for (int e = 0; e < 8; ++e) v = fmaf(acc[i][e], acc[i][e], v);
+                v = warp_sum(v);
+                if (lane == 0) red[warp][i] = v;
+            }
+            asm volatile("bar.sync 1, %0;" ::"r"(n_ct) : "memory");
+            if (tid < D) {
+                float tot = 0.f;
+                for (int w = 0; w < n_cw; ++w) tot += red[w][tid];
+                inv_s[tid] = inv_rms(tot, d, eps);
+            }
+            asm volatile("bar.sync 1, %0;" ::"r"(n_ct) : "memory");
+            if (act) {
+#pragma unroll
+                for (int i = 0; i < DMAX; ++i) {
+                    if (i >= D) break;
+                    float gg[8], o[8];
+                    load8(gain + (size_t)i * d + e0, gg);
+                    const float inv = inv_s[i];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) o[e] = gg[e] * (acc[i][e] * inv);
+                    store8(F + ((size_t)i * f_layer_rows + pid) * d + e0, o);
+                    if (F_out) store8(F_out + (((size_t)i * batch + b) * n_max + r) * d + e0, o);
+                }
             }
         }
     }
+    __syncthreads();
 }
 
 template <class T>
@@ -362,26 +394,26 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
     const T* gain = static_cast<const T*>(c->w.fuse_norm);
     T* F = static_cast<T*>(c->fused);
     T* Fo = static_cast<T*>(fused_out);
-    const int rthreads = ((g.d / 8 + 31) / 32) * 32;
-    const size_t rsmem_need = (size_t)kNS * kRB * g.d * sizeof(T);
-    if ((long long)c->batch * n_max >= 2LL * c->num_sms && rsmem_need <= 220 * 1024 &&
-        g.n_draft_layers <= 8) {
-        // enough positions to fill the GPU: one CTA per position
-        auto rk = g.n_draft_layers <= 4 ? fuse_rows_kernel<T, 4>
-                  : g.n_draft_layers == 5 ? fuse_rows_kernel<T, 5> : fuse_rows_kernel<T, 8>;
-        const int threads = rthreads;
-        const size_t rsmem = rsmem_need;
+    // context fill: one warp-specialised CTA per SM (d / 8 consumer threads and a producer warp),
+    // a ring of as many kRB-row stages as fit in about 200 KB (at most kMaxNS)
+    const int cthreads = ((g.d / 8 + 31) / 32) * 32;
+    const size_t stage_bytes = (size_t)kRB * g.d * sizeof(T);
+    const int ns = (int)std::min<size_t>(kMaxNS, (200 * 1024) / stage_bytes);
+    if ((long long)c->batch * n_max >= 2LL * c->num_sms && ns >= 3 && cthreads <= 512 &&
+        g.n_draft_layers <= 8 && g.n_target_layers <= 64) {
+        auto rk = g.n_draft_layers <= 4 ? fuse_rows_kernel<T, 4> : fuse_rows_kernel<T, 8>;
+        const int threads = cthreads + 32;
+        const size_t rsmem = (size_t)ns * stage_bytes;
         static PerDeviceOnce rconf;
         const cudaError_t re = rconf([] {
-            for (auto k : {fuse_rows_kernel<T, 4>, fuse_rows_kernel<T, 5>, fuse_rows_kernel<T, 8>}) {
+            for (auto k : {fuse_rows_kernel<T, 4>, fuse_rows_kernel<T, 8>}) {
                 cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                     220 * 1024);
+                                                     200 * 1024);
                 if (e != cudaSuccess) return e;
             }
             return cudaSuccess;
         });
         if (re != cudaSuccess) return re;
-        // persistent: as many CTAs as fit at once (two per SM at d = 2560), at most one per position
         int per_sm = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rk, threads, rsmem) != cudaSuccess || per_sm < 1)
             per_sm = 1;
@@ -389,7 +421,7 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
         return launch_kernel(c->pdl, rk, dim3(grid), dim3(threads), rsmem, s, H,
                              (const float*)c->alpha, gain, F, Fo, (const int32_t*)c->app_cnt,
                              g.n_draft_layers, g.n_target_layers, c->batch, n_max, g.d,
-                             (long long)g.max_fuse_rows, g.rms_eps, c->err);
+                             (long long)g.max_fuse_rows, g.rms_eps, ns, c->err);
     }
     auto kern = g.n_draft_layers <= 4 ? fuse_layers_kernel<T, 4> : fuse_layers_kernel<T, 8>;
     static PerDeviceOnce configured;
