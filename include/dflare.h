@@ -300,6 +300,19 @@ dflare_status dflare_device_error(dflare_ctx* ctx, uint32_t* bits_host, void* st
 typedef void (*dflare_trace_fn)(void* user, const char* name, int phase, void* stream);
 dflare_status dflare_set_trace(dflare_ctx* ctx, dflare_trace_fn fn, void* user);
 
+/* Optional device-side timing of the projection GEMM launches (the tcgen05 kernel behind every
+ * "gemm_*" trace name). stamps_dev: caller-owned device array of 3 * slots uint64, laid out as
+ * [0, slots) first-CTA entry times, [slots, 2 slots) times at which the first CTA's activation
+ * dependency on the previous kernel was met, [2 slots, 3 slots) last-CTA exit times, all in
+ * %globaltimer nanoseconds. After this call, GEMM launch number k (counted from this call, k <
+ * slots) folds its CTAs' times into slot k with atomicMin (entry, dependency) and atomicMax
+ * (exit); later launches are not timed. The caller sets the first two ranges to all-ones and the
+ * third to zero before the launches it reads, and may capture the launches into a CUDA graph
+ * (the slot numbers are fixed at capture). Adds two global atomics per CTA while enabled.
+ * stamps_dev = NULL (or slots = 0) turns timing off. Calls made with timing on launch directly
+ * (they are not replayed from the library's own graphs). */
+dflare_status dflare_set_timing(dflare_ctx* ctx, unsigned long long* stamps_dev, int slots);
+
 /* Message of the last failing call on ctx (or of the last failing dflare_create when ctx is
  * NULL). Never NULL; valid until the next call on the same context. */
 const char* dflare_last_error(const dflare_ctx* ctx);

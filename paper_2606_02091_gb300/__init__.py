@@ -214,6 +214,16 @@ class DFlare:
         self._check(self._L.dflare_ctx_lens(self._ctx, arr, _stream(stream)))
         return list(arr)
 
+    def set_timing(self, stamps=None, slots: int = 0):
+        """Device-side timing of the next `slots` GEMM launches into the int64 device tensor
+        `stamps` (3 * slots entries: entry, dependency met, exit; see dflare_set_timing); with no
+        arguments timing is turned off."""
+        import torch
+        if stamps is not None:
+            _need_cuda("stamps", stamps, torch.int64, 3 * slots)
+        self._check(self._L.dflare_set_timing(self._ctx, _ptr(stamps) if stamps is not None else None,
+                                              slots if stamps is not None else 0))
+
     def device_error(self, stream=None) -> int:
         bits = ctypes.c_uint32(0)
         st = self._L.dflare_device_error(self._ctx, ctypes.byref(bits), _stream(stream))

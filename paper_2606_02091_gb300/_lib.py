@@ -35,7 +35,8 @@ EXPORTS = ("dflare_create", "dflare_destroy", "dflare_set_weights", "dflare_rese
            "dflare_verify_logits", "dflare_draft_block_sampled", "dflare_verify_sampled",
            "dflare_read_kv",
            "dflare_ctx_lens", "dflare_device_error", "dflare_last_error",
-           "dflare_synthetic_target", "dflare_set_trace", "dflare_argmax_noalloc")
+           "dflare_synthetic_target", "dflare_set_trace", "dflare_set_timing",
+           "dflare_argmax_noalloc")
 
 NOALLOC_MAX_ROWS = 4096
 
@@ -97,6 +98,7 @@ def load():
         "dflare_last_error": [vp],
         "dflare_synthetic_target": [vp, vp, vp, vp, i32, vp, u32, i32, i32, vp, vp],
         "dflare_set_trace": [vp, TRACE_FN, vp],
+        "dflare_set_timing": [vp, vp, i32],
         "dflare_argmax_noalloc": [vp, i32, i32, vp, vp],
     }
     for name, args in sig.items():

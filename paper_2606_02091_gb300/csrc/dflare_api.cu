@@ -158,7 +158,7 @@ const uint8_t* at(const void* base, size_t elems, size_t esz) {
 // operands in the key and on state that is fixed for the context (the weights: set_weights drops
 // the graphs); everything that varies from step to step (context lengths, accepted counts, step
 // counters) is read by the kernels from device memory. Calls made while the stream is being
-// captured, with a trace hook set, or on the legacy default stream run directly.
+// captured, with a trace hook or GEMM timing set, or on the legacy default stream run directly.
 void drop_slot(GraphSlot& sl) {
     if (sl.exec) cudaGraphExecDestroy(sl.exec);
     sl = GraphSlot{};
@@ -169,7 +169,7 @@ void drop_graph(CallGraph& cg) {
 template <class F>
 dflare_status graphed(dflare_ctx* c, CallGraph& cg, const uint64_t* key, int nk, cudaStream_t s, F&& body) {
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-    if (!s || c->trace_fn || nk > GraphSlot::kKeyLen || cudaStreamIsCapturing(s, &cs) != cudaSuccess ||
+    if (!s || c->trace_fn || c->t_stamps || nk > GraphSlot::kKeyLen || cudaStreamIsCapturing(s, &cs) != cudaSuccess ||
         cs != cudaStreamCaptureStatusNone) {
         cudaGetLastError();
         return body();
@@ -806,6 +806,15 @@ dflare_status dflare_set_trace(dflare_ctx* c, dflare_trace_fn fn, void* user) {
     if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
     c->trace_fn = fn;
     c->trace_user = user;
+    return DFLARE_OK;
+}
+
+dflare_status dflare_set_timing(dflare_ctx* c, unsigned long long* stamps, int slots) {
+    if (!c) return fail(nullptr, DFLARE_EINVAL, "ctx is NULL");
+    if (slots < 0) return fail(c, DFLARE_EINVAL, "slots < 0");
+    c->t_stamps = slots > 0 ? stamps : nullptr;
+    c->t_slots = c->t_stamps ? slots : 0;
+    c->t_next = 0;
     return DFLARE_OK;
 }
 
