@@ -69,13 +69,7 @@ TINY = synth.preset("tiny_f32")
 
 
 def rel_err(x, y):
-    """Max relative error of the vectors along the last axis: max_r ||x_r - y_r|| / ||y_r||.
-
-    A hidden state, a fused context row, a key or value head vector and a row of logits are each
-    compared as one vector. Element-wise ratios are not used: bf16 storage rounding makes any
-    upstream perturbation flip single elements by a full bf16 ulp, so near-zero elements of an
-    otherwise accurate vector would dominate an element-wise maximum.
-    """
+    """Row-wise relative error: max over rows (vectors along the last axis) of ||x_r - y_r|| / ||y_r||."""
     x = np.asarray(x, np.float64)
     y = np.asarray(y, np.float64)
     if not y.size:
@@ -86,16 +80,51 @@ def rel_err(x, y):
     return float(np.max(num / den))
 
 
-def elem_err(x, y):
-    """max_i |x_i - y_i| / max(|y_i|, rms(y)) (reported by the diagnostics, not asserted)."""
+def elem_err(x, y, floor_frac: float):
+    """Element-wise relative error: max_i |x_i - y_i| / max(|y_i|, floor_frac * rms(y)), rms over
+    the whole compared tensor (the floor keeps elements that cancel to near zero from dividing
+    by almost nothing)."""
     x = np.asarray(x, np.float64)
     y = np.asarray(y, np.float64)
-    rms = float(np.sqrt(np.mean(y * y))) if y.size else 1.0
-    return float(np.max(np.abs(x - y) / np.maximum(np.maximum(np.abs(y), rms), 1e-300)))
+    if not y.size:
+        return 0.0
+    rms = float(np.sqrt(np.mean(y * y)))
+    den = np.maximum(np.abs(y), max(floor_frac * rms, 1e-300))
+    return float(np.max(np.abs(x - y) / den))
+
+
+# Element-wise floors. bf16: 1e-3 rms; a tensor computed from the same input bytes on both sides
+# differs only where the final bf16 rounding falls the other way (one ulp, <= 2^-7 relative).
+# fp32: the tensor's rms; fp32 accumulation leaves an absolute error of a few ulp of the terms
+# summed, so an element that cancels to 1e-3 rms carries ~1e-4 relative error on any fp32
+# implementation, while |x - y| <= 1e-5 rms holds.
+BF16_FLOOR = 1e-3
+F32_FLOOR = 1.0
 
 
 def tolerance(w: synth.Workload) -> float:
     return 2e-2 if w.shape.dtype == "bf16" else 1e-5
+
+
+def check_elem(w: synth.Workload, x, y, what=""):
+    """Element-wise check (floor per the storage type), with the row-wise error in the message."""
+    floor = BF16_FLOOR if w.shape.dtype == "bf16" else F32_FLOOR
+    e = elem_err(x, y, floor)
+    assert e <= tolerance(w), (f"{what}: element-wise {e:.3e} (floor {floor} rms) > "
+                               f"{tolerance(w)}; row-wise {rel_err(x, y):.3e}")
+    return e
+
+
+def check_rows(w: synth.Workload, x, y, what=""):
+    """Hidden states and logits: element-wise in fp32; in bf16 row-wise, since every bf16 storage
+    point of the layers (normalised rows, Q/K/V, attention output, SwiGLU product) can round an
+    element to the neighbouring value and the next layer carries that ulp forward."""
+    if w.shape.dtype != "bf16":
+        return check_elem(w, x, y, what)
+    r = rel_err(x, y)
+    assert r <= tolerance(w), (f"{what}: row-wise {r:.3e} > {tolerance(w)}; element-wise "
+                               f"{elem_err(x, y, BF16_FLOOR):.3e} (floor {BF16_FLOOR} rms)")
+    return r
 
 
 def to_device(a: np.ndarray):
@@ -141,9 +170,11 @@ class GpuSide:
         self.lib.reset(w.batch)
         self.torch = torch
 
-    def fuse(self, lens, pos0=None, want_fused=True):
+    def fuse(self, lens, pos0=None, want_fused=True, H=None):
+        """One dflare_fuse_context call on the target states of positions pos0[b] .. + lens[b]
+        (generated here, or the [T][batch][n_max][d] array H). Returns the fused rows."""
         torch = self.torch
-        H = to_device(fill_hidden(self.w, lens, pos0))
+        H = to_device(fill_hidden(self.w, lens, pos0) if H is None else H)
         n_new = torch.tensor(list(lens), dtype=torch.int32, device="cuda")
         fused = None
         if want_fused:
@@ -176,3 +207,101 @@ def f64(t):
 
 def oracle_for(w: synth.Workload, W: dict, **kw):
     return O.DraftOracle(W, w.shape, w.batch, storage=storage_name(w), **kw)
+
+
+def check_kv(w: synth.Workload, o, k, v, F_gpu_i, pos, i, what=""):
+    """Cached keys/values of draft layer i at absolute positions pos against Eq. 4 evaluated by the
+    oracle on the GPU's own fused rows F_gpu_i (the same input bytes), element by element. (Against
+    the oracle's own F they are compared row-wise: an F element rounded to the other bf16
+    neighbour, a rate of ~1e-4 per element, moves every key of its position by ~1e-4 absolute,
+    about 0.1 of a 1e-3 rms floor.)"""
+    s = w.shape
+    w_kv = o._dec("w_qkv", i)[s.d_q:] if o.shared_kv else o._dec("w_kv_ctx", i)
+    kx, vx = O.context_kv(F_gpu_i, w_kv, np.asarray(pos), s.n_kv_heads, s.head_dim, s.rope_theta,
+                          o.store)
+    check_elem(w, k, kx, f"{what} K")
+    check_elem(w, v, vx, f"{what} V")
+
+
+GAP = 1e-2   # near-tie threshold of the token comparison (top-2 logit gap on the oracle's logits)
+
+
+def check_tokens(w: synth.Workload, o, tok, logits, x_last, ot, ol, what=""):
+    """Draft tokens of one sequence (Sec. 3.2, greedy drafting).
+
+    - On the GPU's own fp32 logits the argmax (lowest id among equal maxima) is exact.
+    - The LM head and argmax alone: the oracle's final RMSNorm, LM head and argmax applied to the
+      GPU's last hidden state x_last give the GPU's tokens except where that oracle's top-2 gap is
+      below GAP.
+    - End to end, against the oracle's own chain: a token may differ only where the oracle's top-2
+      gap is below max(GAP, 3 sqrt(2) rms(logits - oracle logits)) of that row, i.e. where the two
+      competing logits' measured discrepancy explains the swap at 3 sigma. With bf16 storage the
+      two chains' rounding decisions drift apart layer by layer (the row-wise logit difference of a
+      d 4096, 8-layer drafter is ~1.3e-2 of the logits' norm, ~0.015 rms), so gaps a little above
+      1e-2 are decided by rounding noise, not by the method.
+    Returns the number of end-to-end mismatches (all of them inside the rule)."""
+    s = w.shape
+    np.testing.assert_array_equal(tok, O.argmax_lowest(logits), err_msg=f"{what}: argmax of own logits")
+    hl = O.lm_head_logits(np.asarray(x_last, np.float64), o._dec("final_norm"), o._dec("lm_head"),
+                          s.rms_eps, o.store)
+    ht = O.argmax_lowest(hl)
+    bad = (tok != ht) & (O.top2_gap(hl) >= GAP)
+    assert not bad.any(), (f"{what}: LM head + argmax on the GPU's last hidden state differs at "
+                           f"{np.nonzero(bad)[0].tolist()} (gaps {O.top2_gap(hl)[bad].tolist()})")
+    mism = tok != ot
+    if mism.any():
+        sigma = np.sqrt(np.mean((np.asarray(logits, np.float64) - ol) ** 2, axis=-1))
+        thr = np.maximum(GAP, 3 * np.sqrt(2) * sigma)
+        gap = O.top2_gap(ol)
+        out = mism & (gap >= thr)
+        assert not out.any(), (f"{what}: tokens differ from the oracle at {np.nonzero(out)[0].tolist()} "
+                               f"with gaps {gap[out].tolist()} above {thr[out].tolist()}")
+    return int(mism.sum())
+
+
+def verified_steps(w: synth.Workload, g: GpuSide, o, n_steps: int):
+    """n_steps block steps on both sides: draft -> synthetic target -> prefix accept -> fuse the
+    tau accepted positions. Both sides continue from the GPU's drafts (the synthetic target, tau and
+    the next token are integer work on them: exact), so every step of every sequence is compared:
+    hidden states after every layer, logits and tokens (check_tokens). Returns the number of
+    (step, sequence) pairs compared."""
+    import torch
+    from paper_2606_02091_gb300 import synthetic_target
+    s = w.shape
+    x_t = synth.initial_tokens(w).astype(np.int64)
+    thr = synth.accept_threshold(w.match_p)
+    lens = [o.ctx_len(b) for b in range(w.batch)]
+    step_ctr = torch.zeros(1, dtype=torch.int32, device="cuda")
+    compared = 0
+    for step in range(n_steps):
+        tok, logits, hidden = g.draft(x_t)
+        u, r, last = synth.target_draws(w, step)
+        tgt = torch.zeros((w.batch, s.block), dtype=torch.int32, device="cuda")
+        acc = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
+        nxt = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
+        dt = torch.tensor(tok, device="cuda")
+        step_ctr.fill_(0)
+        synthetic_target(dt, torch.tensor(u.view(np.int32), device="cuda"),
+                         torch.tensor(r, device="cuda"), torch.tensor(last, device="cuda"),
+                         step_ctr, thr, w.batch, s.block, tgt)
+        g.lib.verify_accept(dt, tgt, acc, nxt)
+        tgt_h, acc_h, nxt_h = tgt.cpu().numpy(), acc.cpu().numpy(), nxt.cpu().numpy()
+        for b in range(w.batch):
+            gt = O.synthetic_target(tok[b], u[0, b], r[0, b], last[0, b], thr)
+            np.testing.assert_array_equal(tgt_h[b], gt)
+            assert (acc_h[b], nxt_h[b]) == O.verify_accept(tok[b], gt)
+            ot, ol, oh = o.draft_block(b, int(x_t[b]))
+            for i in range(oh.shape[0]):
+                check_rows(w, hidden[i, b], oh[i], f"step {step} seq {b} hidden after layer {i - 1}")
+            check_rows(w, logits[b], ol, f"step {step} seq {b} logits")
+            check_tokens(w, o, tok[b], logits[b], hidden[-1, b], ot, ol, f"step {step} seq {b}")
+            compared += 1
+        taus = [int(a) for a in acc_h]
+        g.fuse(taus, pos0=lens, want_fused=False)
+        for b in range(w.batch):
+            o.fuse_context(b, synth.hidden_states(w, b, lens[b], taus[b]))
+            lens[b] += taus[b]
+        x_t = nxt_h.astype(np.int64)
+        assert g.lib.ctx_lens() == lens
+    assert g.lib.device_error() == 0
+    return compared

@@ -1,15 +1,23 @@
-"""GPU path vs the CPU oracle, element by element, on the same seeded inputs (Eq. 3, Eq. 4,
-Sec. 3.2). Tolerances: fused context rows, cached key/value head vectors, hidden states and
-logit rows within max relative error 2e-2 (bf16 storage) or 1e-5 (fp32 storage), each row
-compared as a vector (max over rows of ||x - y|| / ||y||); token ids and acceptance lengths
-bit-exact, except draft positions whose top-2 logit gap (on the oracle's logits) is below 1e-2."""
+"""GPU path vs the CPU oracle on the same seeded inputs (Eq. 3, Eq. 4, Sec. 3.2).
+
+Tolerances: max relative error 2e-2 (bf16 storage) or 1e-5 (fp32 storage).
+- Fused context rows: element by element, |x - y| / max(|y|, c rms(y)) with c = 1e-3 (bf16) or 1
+  (fp32: fp32 accumulation leaves an absolute error of a few ulp of the summed terms).
+- Cached keys/values: element by element against Eq. 4 evaluated by the oracle on the GPU's own
+  fused rows (the same input bytes), and row-wise (max over head vectors of ||x - y|| / ||y||)
+  against the oracle's cache built from its own fused rows.
+- Hidden states and logits: element by element in fp32; row-wise in bf16, where each layer's
+  bf16 storage points carry single-element ulp flips forward.
+- Acceptance lengths and next tokens bit-exact (integer work on the GPU's drafts); draft tokens as in
+  tests.harness.check_tokens."""
 import numpy as np
 import pytest
 
 import oracle as O
 import synth
 from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, MULTI_TILE, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16,
-                           GpuSide, f64, oracle_for, rel_err, tolerance)
+                           GpuSide, check_elem, check_kv, check_rows, check_tokens, f64, oracle_for,
+                           rel_err, tolerance, verified_steps)
 
 pytestmark = pytest.mark.gpu
 GAP = 1e-2
@@ -30,8 +38,7 @@ def test_fusion_matches_oracle(run):
     w, g, o, fused, F = run
     got = f64(fused)
     for b, n in enumerate(w.ctx_lens):
-        err = rel_err(got[:, b, :n], F[b])
-        assert err <= tolerance(w), (b, err)
+        check_elem(w, got[:, b, :n], F[b], f"F seq {b}")
 
 
 def test_context_lengths(run):
@@ -42,25 +49,21 @@ def test_context_lengths(run):
 
 def test_context_kv_matches_oracle(run):
     w, g, o, fused, F = run
+    got = f64(fused)
     for b, n in enumerate(w.ctx_lens):
         for i in range(w.shape.n_draft_layers):
             k, v = g.lib.read_kv(i, b, 0, n)
-            assert rel_err(f64(k), o.ctx_k[b][i]) <= tolerance(w), (b, i, "K")
-            assert rel_err(f64(v), o.ctx_v[b][i]) <= tolerance(w), (b, i, "V")
+            check_kv(w, o, f64(k), f64(v), got[i, b, :n], np.arange(n), i, f"seq {b} layer {i}")
+            check_rows(w, f64(k), o.ctx_k[b][i], f"seq {b} layer {i} K (end to end)")
+            check_rows(w, f64(v), o.ctx_v[b][i], f"seq {b} layer {i} V (end to end)")
 
 
-def _check_draft(w, tok, logits, hidden, o_res):
-    tol = tolerance(w)
+def _check_draft(w, tok, logits, hidden, o_res, o):
     for b, (ot, ol, oh) in enumerate(o_res):
         for i in range(oh.shape[0]):
-            err = rel_err(hidden[i, b], oh[i])
-            assert err <= tol, f"seq {b} hidden after layer {i - 1}: rel err {err}"
-        assert rel_err(logits[b], ol) <= tol, f"seq {b} logits"
-        gap = O.top2_gap(ol)
-        keep = gap >= GAP
-        np.testing.assert_array_equal(tok[b][keep], ot[keep])
-        # the GPU's own argmax decision on its own logits is exact
-        np.testing.assert_array_equal(tok[b], O.argmax_lowest(logits[b]))
+            check_rows(w, hidden[i, b], oh[i], f"seq {b} hidden after layer {i - 1}")
+        check_rows(w, logits[b], ol, f"seq {b} logits")
+        check_tokens(w, o, tok[b], logits[b], hidden[-1, b], ot, ol, f"seq {b}")
 
 
 def test_draft_block_matches_oracle(run):
@@ -68,56 +71,13 @@ def test_draft_block_matches_oracle(run):
     x_t = synth.initial_tokens(w)
     tok, logits, hidden = g.draft(x_t)
     o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
-    _check_draft(w, tok, logits, hidden, o_res)
+    _check_draft(w, tok, logits, hidden, o_res, o)
 
 
 def test_steps_with_verification(run):
     """Two more block steps: draft -> synthetic target -> prefix accept -> fuse tau positions."""
-    import torch
-    from paper_2606_02091_gb300 import synthetic_target
     w, g, o, fused, F = run
-    s = w.shape
-    x_t = synth.initial_tokens(w).astype(np.int64)
-    thr = synth.accept_threshold(w.match_p)
-    lens = list(w.ctx_lens)
-    in_sync = [True] * w.batch
-    step_ctr = torch.zeros(1, dtype=torch.int32, device="cuda")
-    for step in range(2):
-        tok, logits, hidden = g.draft(x_t)
-        o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
-        u, r, last = synth.target_draws(w, step)
-        tgt = torch.zeros((w.batch, s.block), dtype=torch.int32, device="cuda")
-        acc = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
-        nxt = torch.zeros(w.batch, dtype=torch.int32, device="cuda")
-        dt = torch.tensor(tok, device="cuda")
-        step_ctr.fill_(0)
-        synthetic_target(dt, torch.tensor(u.view(np.int32), device="cuda"), torch.tensor(r, device="cuda"),
-                         torch.tensor(last, device="cuda"), step_ctr, thr, w.batch, s.block, tgt)
-        g.lib.verify_accept(dt, tgt, acc, nxt)
-        tgt_h, acc_h, nxt_h = tgt.cpu().numpy(), acc.cpu().numpy(), nxt.cpu().numpy()
-        for b in range(w.batch):
-            # integer work on identical integer inputs: exact
-            gt = O.synthetic_target(tok[b], u[0, b], r[0, b], last[0, b], thr)
-            np.testing.assert_array_equal(tgt_h[b], gt)
-            assert (acc_h[b], nxt_h[b]) == O.verify_accept(tok[b], gt)
-            if not in_sync[b]:
-                continue
-            ot, ol, oh = o_res[b]
-            if not np.array_equal(tok[b], ot):
-                assert np.all(O.top2_gap(ol)[tok[b] != ot] < GAP)
-                in_sync[b] = False      # a near-tie made the two chains diverge
-                continue
-            for i in range(oh.shape[0]):
-                assert rel_err(hidden[i, b], oh[i]) <= tolerance(w)
-        # commit tau positions on both sides and continue from the target's extra token
-        taus = [int(a) for a in acc_h]
-        g.fuse(taus, pos0=lens, want_fused=False)
-        for b in range(w.batch):
-            o.fuse_context(b, synth.hidden_states(w, b, lens[b], taus[b]))
-            lens[b] += taus[b]
-        x_t = nxt_h.astype(np.int64)
-        assert g.lib.ctx_lens() == lens
-    assert g.lib.device_error() == 0
+    assert verified_steps(w, g, o, n_steps=2) >= w.batch
 
 
 def test_rope_off_block_is_mask_permutation_equivariant():
@@ -138,7 +98,7 @@ def test_rope_off_block_is_mask_permutation_equivariant():
             np.testing.assert_array_equal(tok[b, k - 1], tok[b, 0])
         ot, ol, oh = o.draft_block(b, int(synth.initial_tokens(w)[b]))
         for i in range(oh.shape[0]):
-            assert rel_err(hidden[i, b], oh[i]) <= tolerance(w)
+            check_rows(w, hidden[i, b], oh[i], f"seq {b} hidden after layer {i - 1}")
 
 
 def test_raw_fusion_ablation():
@@ -149,7 +109,7 @@ def test_raw_fusion_ablation():
     fused = f64(g.fuse(w.ctx_lens))
     o = oracle_for(w, g.W, softmax_fusion=False)
     F = o.fuse_context(0, synth.hidden_states(w, 0, 0, w.ctx_lens[0]))
-    assert rel_err(fused[:, 0], F) <= tolerance(w)
+    check_elem(w, fused[:, 0], F, "F (-Softmax)")
 
 
 def test_empty_and_capacity_edges():
@@ -166,7 +126,7 @@ def test_empty_and_capacity_edges():
     for b in range(w.batch):
         ot, ol, oh = o.draft_block(b, int(synth.initial_tokens(w)[b]))
         for i in range(oh.shape[0]):
-            assert rel_err(hidden[i, b], oh[i]) <= tolerance(w)
+            check_rows(w, hidden[i, b], oh[i], f"empty context seq {b} hidden after layer {i - 1}")
     g.fuse([65, 300], want_fused=False)
     assert g.lib.device_error() == 0
     g.fuse([5, 11], pos0=[65, 300], want_fused=False)       # 300 + 11 > 310: refused
@@ -206,14 +166,16 @@ def test_wide_token_tiles_match_oracle(w):
     g = GpuSide(w)
     o = oracle_for(w, g.W)
     fused = f64(g.fuse(w.ctx_lens))
+    last = w.shape.n_draft_layers - 1
     for b, n in enumerate(w.ctx_lens):
         F = o.fuse_context(b, synth.hidden_states(w, b, 0, n))
-        assert rel_err(fused[:, b, :n], F) <= tolerance(w), b
-        k, v = g.lib.read_kv(w.shape.n_draft_layers - 1, b, 0, n)
-        assert rel_err(f64(k), o.ctx_k[b][w.shape.n_draft_layers - 1]) <= tolerance(w), b
+        check_elem(w, fused[:, b, :n], F, f"F seq {b}")
+        k, v = g.lib.read_kv(last, b, 0, n)
+        check_kv(w, o, f64(k), f64(v), fused[last, b, :n], np.arange(n), last, f"seq {b}")
+        check_rows(w, f64(k), o.ctx_k[b][last], f"seq {b} K (end to end)")
     x_t = synth.initial_tokens(w)
     tok, logits, hidden = g.draft(x_t)
-    _check_draft(w, tok, logits, hidden, [o.draft_block(b, int(x_t[b])) for b in range(w.batch)])
+    _check_draft(w, tok, logits, hidden, [o.draft_block(b, int(x_t[b])) for b in range(w.batch)], o)
     assert g.lib.device_error() == 0
 
 
@@ -242,24 +204,26 @@ def test_variant_matches_oracle(w, flags, kw):
     F = [o.fuse_context(b, synth.hidden_states(w, b, 0, n)) for b, n in enumerate(w.ctx_lens)]
     x_t = synth.initial_tokens(w)
     o_res = [o.draft_block(b, int(x_t[b])) for b in range(w.batch)]
-    tol = tolerance(w)
     for want_fused in (True, False):
         g = GpuSide(w, flags=flag, weights=W)
         fused = g.fuse(w.ctx_lens, want_fused=want_fused)
         assert g.lib.ctx_lens() == list(w.ctx_lens)
-        if fused is not None:
-            got = f64(fused)
-            slots = 1 if kw.get("dflash_fc") else w.shape.n_draft_layers
-            for b, n in enumerate(w.ctx_lens):
-                err = rel_err(got[:slots, b, :n], F[b][:slots])
-                assert err <= tol, (b, err)
+        got = f64(fused) if fused is not None else None
+        slots = 1 if kw.get("dflash_fc") else w.shape.n_draft_layers
         for b, n in enumerate(w.ctx_lens):
+            if got is not None:
+                # +FC's F' is a product of F, whose single-element bf16 flips it carries: row-wise
+                chk = check_rows if kw.get("fusion_fc") else check_elem
+                chk(w, got[:slots, b, :n], F[b][:slots], f"projected representation seq {b}")
             for i in range(w.shape.n_draft_layers):
                 k, v = g.lib.read_kv(i, b, 0, n)
-                assert rel_err(f64(k), o.ctx_k[b][i]) <= tol, (want_fused, b, i, "K")
-                assert rel_err(f64(v), o.ctx_v[b][i]) <= tol, (want_fused, b, i, "V")
+                if got is not None:
+                    check_kv(w, o, f64(k), f64(v), got[0 if kw.get("dflash_fc") else i, b, :n],
+                             np.arange(n), i, f"seq {b} layer {i}")
+                check_rows(w, f64(k), o.ctx_k[b][i], f"{want_fused} seq {b} layer {i} K (end to end)")
+                check_rows(w, f64(v), o.ctx_v[b][i], f"{want_fused} seq {b} layer {i} V (end to end)")
         tok, logits, hidden = g.draft(x_t)
-        _check_draft(w, tok, logits, hidden, o_res)
+        _check_draft(w, tok, logits, hidden, o_res, o)
         assert g.lib.device_error() == 0
 
 
@@ -379,3 +343,30 @@ def test_repeated_calls_replay_as_graphs():
         assert torch.equal(ta, tb) and torch.equal(lga, lgb) and torch.equal(ha, hb)
     for (ka, va), (kb, vb) in zip(kva, kvb):
         assert torch.equal(ka, kb) and torch.equal(va, vb)
+
+
+def test_gemm_timing_stamps_are_ordered():
+    """dflare_set_timing on a drafted block: each of the 4 D + 1 projection launches (Q/K^d/V^d,
+    O, gate/up, down per layer, then the LM head) records entry <= dependency met <= exit, each
+    launch ends after the one before it, and the slots past the last launch stay untouched."""
+    import torch
+    w = SMALL_HD128
+    g = GpuSide(w)
+    g.fuse(w.ctx_lens, want_fused=False)
+    slots = 64
+    st = torch.empty(3 * slots, dtype=torch.int64, device="cuda")
+    st[:2 * slots].fill_(-1)
+    st[2 * slots:].zero_()
+    g.lib.set_timing(st, slots)
+    g.draft(synth.initial_tokens(w))
+    g.lib.set_timing()
+    torch.cuda.synchronize()
+    a = st.cpu().numpy().view(np.uint64)
+    n = 4 * w.shape.n_draft_layers + 1
+    entry, dep, done = a[:slots], a[slots:2 * slots], a[2 * slots:]
+    for k in range(n):
+        assert 0 < entry[k] <= dep[k] <= done[k], k
+        if k:
+            assert done[k] > done[k - 1], k
+    assert np.all(entry[n:] == np.uint64(2 ** 64 - 1)) and np.all(done[n:] == 0)
+    assert g.lib.device_error() == 0
