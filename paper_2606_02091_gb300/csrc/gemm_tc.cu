@@ -46,8 +46,6 @@ constexpr uint32_t kABytes = kBM * kBK * 2;   // one 128 x 64 bf16 weight tile
 struct TcArgs {
     CUtensorMap map_a, map_a2, map_b;   // weights, up weights (SwiGLU), activations
     int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks;
-    int stream_k;              // 1: CTA c owns (tile, k-block) items [c W / grid, (c + 1) W / grid)
-    int max_contrib;           // workspace slots per tile (splits, or the most CTAs sharing a tile)
     int bn, n_a, stages, n_bufs, tmem_cols;
     int kbs;                   // 64-wide k-blocks per pipeline stage
     uint32_t b_bytes;          // bytes of one activation sub-tile (bn x 64 bf16)
@@ -174,67 +172,24 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
 // addressed for the tensor maps, so every asm with a memory clobber would otherwise reload them).
 struct Geom {
     int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks, n_a, kbs, bn, n_bufs;
-    int stream_k, max_contrib;
     uint32_t b_bytes, stage_bytes, idesc;
 };
-// One CTA's piece of a 128-feature x token tile: k-blocks [kb0, kb1), contribution `contrib` of
-// the `n_contrib` that make up the tile (workspace slot and reduction order).
 struct Unit {
-    int group, n_tile, tok_tile, tile_id, kb0, kb1, contrib, n_contrib;
+    int group, n_tile, tok_tile, split, tile_id, kb0, kb1;
 };
-__device__ __forceinline__ void tile_coords(const Geom& a, Unit& x) {
+__device__ __forceinline__ Unit decode_unit(const Geom& a, int u) {
+    Unit x;
+    x.split = u % a.splits;
+    x.tile_id = u / a.splits;
     int t = x.tile_id;
     x.tok_tile = t % a.tok_tiles;
     t /= a.tok_tiles;
     x.n_tile = t % a.n_tiles;
     x.group = t / a.n_tiles;
+    x.kb0 = x.split * a.kb_per_split;
+    x.kb1 = min(a.k_blocks, x.kb0 + a.kb_per_split);
+    return x;
 }
-// The units of one CTA, in order. Uniform split-K: units blockIdx.x + k gridDim.x of the
-// tiles x splits grid. Stream-K: the (tile, k-block) items W = tiles x k_blocks are cut into
-// gridDim.x contiguous runs of equal length (to one item), CTA c owning [c W / grid, (c + 1) W /
-// grid); a run that crosses a tile boundary gives one unit per tile it touches, and the CTAs
-// sharing a tile reduce through the workspace in CTA order (or add into the residual).
-struct UnitIter {
-    long long i, end, W;
-    int u;
-    __device__ __forceinline__ void init(const Geom& a) {
-        if (a.stream_k) {
-            W = (long long)a.n_units * a.k_blocks;   // n_units = tiles in stream-K mode
-            i = (long long)blockIdx.x * W / gridDim.x;
-            end = (long long)(blockIdx.x + 1) * W / gridDim.x;
-        } else {
-            u = blockIdx.x;
-        }
-    }
-    __device__ __forceinline__ bool next(const Geom& a, Unit& x) {
-        if (a.stream_k) {
-            if (i >= end) return false;
-            const long long KB = a.k_blocks;
-            x.tile_id = (int)(i / KB);
-            x.kb0 = (int)(i % KB);
-            x.kb1 = (int)min((long long)KB, x.kb0 + (end - i));
-            // CTA of item j: the largest c with c W / grid <= j, i.e. ((j + 1) grid - 1) / W
-            const long long G = gridDim.x;
-            const long long t0 = (long long)x.tile_id * KB;
-            const int first = (int)(((t0 + 1) * G - 1) / W);
-            const int last = (int)(((t0 + KB) * G - 1) / W);
-            x.contrib = (int)blockIdx.x - first;
-            x.n_contrib = last - first + 1;
-            i += x.kb1 - x.kb0;
-        } else {
-            if (u >= a.n_units) return false;
-            const int split = u % a.splits;
-            x.tile_id = u / a.splits;
-            x.kb0 = split * a.kb_per_split;
-            x.kb1 = min(a.k_blocks, x.kb0 + a.kb_per_split);
-            x.contrib = split;
-            x.n_contrib = a.splits;
-            u += gridDim.x;
-        }
-        tile_coords(a, x);
-        return true;
-    }
-};
 
 // EPI_RESID with the residual values already in registers: resid[tok][n] += acc.
 __device__ __forceinline__ void load_resid(const EpiParams& ep, int n_tile, int tok0, int t, float* r) {
@@ -276,8 +231,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     G.kbs = args.kbs;
     G.bn = args.bn;
     G.n_bufs = args.n_bufs;
-    G.stream_k = args.stream_k;
-    G.max_contrib = args.max_contrib;
     G.b_bytes = args.b_bytes;
     G.stage_bytes = args.stage_bytes;
     G.idesc = args.idesc;
@@ -368,10 +321,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         tma_load_3d(st + b_base + j * G.b_bytes, mB, kx0 + j * kBK, tok_tile * G.bn, group, bar);
                 }
             };
-            UnitIter it;
-            it.init(G);
-            Unit x;
-            while (ok && it.next(G, x)) {
+            for (int u = blockIdx.x; u < G.n_units && ok; u += gridDim.x) {
+                const Unit x = decode_unit(G, u);
                 for (int kb = x.kb0; kb < x.kb1; kb += G.kbs) {
                     const int nk = min(G.kbs, x.kb1 - kb);
                     if (!bar_wait(empty_bar(stage), phase ^ 1u, abort_flag, err)) {
@@ -441,10 +392,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             uint32_t phase = 0, acc_phase = 0;
             bool ok = true;
             const uint32_t b_base = kABytes * G.n_a * G.kbs;
-            UnitIter it;
-            it.init(G);
-            Unit x;
-            while (ok && it.next(G, x)) {
+            for (int u = blockIdx.x; u < G.n_units && ok; u += gridDim.x) {
+                const Unit x = decode_unit(G, u);
                 if (!bar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d0 = tmem + (uint32_t)(acc * acc_cols);
@@ -498,10 +447,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         uint32_t* const tile_cnt = args.tile_cnt;
         const bool resid = args.ep.kind == EPI_RESID && bn == kChunk;
         const bool resid_red = args.ep.kind == EPI_RESID && args.resid_red;
-        UnitIter it;
-        it.init(G);
-        Unit x;
-        while (it.next(G, x)) {
+        for (int u = blockIdx.x; u < G.n_units; u += gridDim.x) {
+            const Unit x = decode_unit(G, u);
             if (resid_red) {
                 // resid += acc with fp32 reductions in L2: every split adds its own partial sum,
                 // with no workspace, no tile counter and no read of the residual (the order of
@@ -544,9 +491,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             tc_fence_after();
             const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
             bool final_tile = true;
-            if (x.n_contrib > 1) {
-                // partial layout per (tile, contribution): [accumulator][16-token chunk][feature][16]
-                float* dst = ws + ((size_t)x.tile_id * G.max_contrib + x.contrib) * na * bn * 128;
+            if (G.splits > 1) {
+                // partial layout per (tile, split): [accumulator][16-token chunk][feature][16]
+                float* dst = ws + (size_t)(x.tile_id * G.splits + x.split) * na * bn * 128;
                 for (int a = 0; a < na; ++a)
                     for (int c0 = 0; c0 < bn; c0 += kChunk) {
                         float v[kChunk];
@@ -564,8 +511,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 epi_bar();
                 if (t == 0) {
                     const uint32_t prev = atom_add_acq_rel(&tile_cnt[x.tile_id], 1u);
-                    misc[2] = (prev == (uint32_t)(x.n_contrib - 1)) ? 1u : 0u;
-                    if (prev == (uint32_t)(x.n_contrib - 1)) tile_cnt[x.tile_id] = 0;
+                    misc[2] = (prev == (uint32_t)(G.splits - 1)) ? 1u : 0u;
+                    if (prev == (uint32_t)(G.splits - 1)) tile_cnt[x.tile_id] = 0;
                 }
                 epi_bar();
                 final_tile = misc[2] != 0;
@@ -574,7 +521,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 for (int c0 = 0; c0 < bn; c0 += kChunk) {
                     for (int a = 0; a < na; ++a) {
                         float v[kChunk];
-                        if (x.n_contrib == 1) {
+                        if (G.splits == 1) {
                             tmem_ld16(taddr + (uint32_t)(a * bn + c0), v);
                         } else {
                             // sum the splits in split order (deterministic); four 16-byte loads
@@ -584,9 +531,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                             for (int k = 0; k < kChunk / 4; ++k) acc4[k] = make_float4(0.f, 0.f, 0.f, 0.f);
                             const size_t off = ((size_t)(a * (bn / kChunk) + c0 / kChunk) * 128 + t) * kChunk;
 #pragma unroll 4
-                            for (int s = 0; s < x.n_contrib; ++s) {
+                            for (int s = 0; s < G.splits; ++s) {
                                 const float4* src = reinterpret_cast<const float4*>(
-                                    ws + ((size_t)x.tile_id * G.max_contrib + s) * na * bn * 128 + off);
+                                    ws + (size_t)(x.tile_id * G.splits + s) * na * bn * 128 + off);
 #pragma unroll
                                 for (int k = 0; k < kChunk / 4; ++k) {
                                     const float4 w4 = __ldcg(src + k);
@@ -615,7 +562,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     epi_bar();
                 }
             }
-            if (x.n_contrib == 1) {
+            if (G.splits == 1) {
                 tc_fence_before();
                 mbar_arrive(tempty_bar(acc));
             }
@@ -735,26 +682,6 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         return cudaErrorInvalidValue;
     }
     a.n_units = tiles * a.splits;
-    a.max_contrib = a.splits;
-    a.resid_red = (c->cfg.flags & DFLARE_FLAG_DETERMINISTIC) ? 0 : 1;
-    // Stream-K: when the uniform split leaves more than a tenth of the SMs idle (e.g. 96 gate/up
-    // tiles at d 4096, 32 O or down tiles split 4 ways), every SM takes an equal run of the
-    // (tile, k-block) items instead; the CTAs sharing a tile reduce through the workspace in CTA
-    // order, or add into the residual.
-    const long long items = (long long)tiles * a.k_blocks;
-    int grid = std::min(a.n_units, sms);
-    if (g.force_splits == 0 && a.n_units < (9 * sms) / 10 && items >= sms) {
-        const int q = (int)(items / sms);                       // shortest run
-        const int mc = (a.k_blocks + q - 1) / q + 1;            // most CTAs sharing one tile
-        const bool red_only = g.ep.kind == EPI_RESID && a.resid_red;
-        if (red_only || ((size_t)tiles * mc * a.n_a * a.bn * 128 <= c->ws_floats && tiles <= c->tile_cnt_n)) {
-            a.stream_k = 1;
-            a.n_units = tiles;
-            a.splits = 1;
-            a.max_contrib = mc;
-            grid = sms;
-        }
-    }
     a.b_bytes = (uint32_t)a.bn * kBK * 2;
     a.stage_bytes = (uint32_t)a.kbs * (kABytes * a.n_a + a.b_bytes);
     a.evict_first = g.evict_first >= 0 ? 1 : 0;
@@ -780,6 +707,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     // group shared by all (b_shared), or k / b_kgroup groups that the contraction runs across
     const long long a_gr = g.a_group_rows > 0 ? g.a_group_rows : g.n;
     a.b_kg = g.b_kgroup;
+    a.resid_red = (c->cfg.flags & DFLARE_FLAG_DETERMINISTIC) ? 0 : 1;
     a.b_gsel = g.b_shared ? 0 : 1;
     const int b_k = g.b_kgroup > 0 ? g.b_kgroup : g.k;
     const int b_groups = g.b_kgroup > 0 ? g.k / g.b_kgroup : (g.b_shared ? 1 : g.groups);
@@ -801,6 +729,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
     });
     if (ce != cudaSuccess) return ce;
+    const int grid = std::min(a.n_units, sms);
     if (c->t_stamps && c->t_next < c->t_slots) {
         a.t_stamps = c->t_stamps + c->t_next++;
         a.t_slots = c->t_slots;
