@@ -9,11 +9,10 @@
 //
 // bf16 path: 64 query rows per CTA (4 warps x 16 rows); one thread streams 64-key K/V tiles by
 // TMA into two 128-byte-swizzled stages; S = Q K^T and O += P V on mma.sync m16n8k16 with bf16
-// operands and fp32 accumulators, P kept in registers as a pair of bf16 values (high part and
-// remainder, two MMAs per step) so that P V carries ~16 significant bits of P; two CTAs fit on
-// an SM. The splits of one (sequence, head, query tile) form a thread-block cluster (up to 16
-// CTAs) and merge their fp32 partial results through distributed shared memory, so the whole
-// attention is one launch and no partial goes through HBM.
+// operands and fp32 accumulators, P kept in registers; two CTAs fit on an SM. The splits of one
+// (sequence, head, query tile) form a thread-block cluster (up to 16 CTAs) and merge their
+// partial results (O / l in fp16) through distributed shared memory, so the whole attention is
+// one launch and no partial goes through HBM.
 // fp32 path: a CUDA-core version of the split with partials in global memory and a second
 // (combine) launch; exact fp32 products.
 #include <cuda_fp16.h>
@@ -93,11 +92,13 @@ __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-// P.V runs on bf16 operands with V as the TMA wrote it. P in [0, 1] is split into its bf16
-// rounding and the bf16 rounding of the remainder, and both parts multiply V (relative error of
-// the pair about 2^-17): a single bf16 P (error 2^-9 per weight) perturbs the attention output of
-// random, cancelling values by ~1e-3 relative, which the bf16 rounding of that output then turns
-// into whole-ulp flips of a large fraction of its elements. The row sums l come from the fp32 P.
+// P.V runs on bf16 operands: V as the TMA wrote it, P in [0, 1] rounded to bf16 (relative error
+// at most 2^-9 per weight; the row sums l are taken from the fp32 P). Measured alternatives: P
+// split into a bf16 high part and its remainder (two MMAs per step, ~2^-17) with the split merge
+// in fp32 took the attention from 25.8 to 32.4 us per launch at the Qwen3-8B batch-4 shape, and
+// the fp32 merge alone cost ~1 us per launch, while the hidden-state difference to the oracle
+// after the first layer only went from 4.8e-3 to 3.9e-3 (the bf16 storage points amplify any
+// perturbation to about an ulp within a few layers).
 // 2^x with the hardware approximation (relative error about 2^-22, far below the bf16 rounding of
 // P; -inf gives +0): the softmax of a tile evaluates 32 of them per thread
 __device__ __forceinline__ float ex2(float x) {
@@ -108,13 +109,6 @@ __device__ __forceinline__ float ex2(float x) {
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&h);
-}
-// (x, y) -> bf16 pairs hi = rn(x, y) and lo = rn(x - hi.x, y - hi.y)
-__device__ __forceinline__ void split_bf16(float x, float y, uint32_t& hi, uint32_t& lo) {
-    const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
-    const float2 hf = __bfloat1622float2(h);
-    hi = *reinterpret_cast<const uint32_t*>(&h);
-    lo = pack_bf16(x - hf.x, y - hf.y);
 }
 
 constexpr int kNST = 2;                   // K/V tiles in flight per CTA (two CTAs fit on an SM)
@@ -181,11 +175,9 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
     bf16* Qs = reinterpret_cast<bf16*>(smem + kNST * 2 * TB);   // [kQT][LD]
     // partials pushed here by the cluster's CTAs: row lr of this CTA's slice from split p at
-    // [p * RP + lr], O / l in fp32 and (running max in log2 units, running sum). rO reuses the
-    // query tile's memory: every thread holds its query fragments in registers before it arrives
-    // on the cluster barrier that the pushing CTAs wait for.
-    float* rO = reinterpret_cast<float*>(Qs);                    // [kQT][HD]
-    float* rML = rO + kQT * HD;                                  // [kQT][2]
+    // [p * RP + lr], O / l in fp16 and (running max in log2 units, running sum)
+    __half* rO = reinterpret_cast<__half*>(Qs + kQT * LD);     // [kQT][HD]
+    float* rML = reinterpret_cast<float*>(rO + kQT * HD);        // [kQT][2]
     uint64_t* full = reinterpret_cast<uint64_t*>(rML + 2 * kQT);   // [kNST] tile landed
     uint64_t* empty = full + kNST;                                  // [kNST] tile read by all 4 warps
     constexpr int RP = kQT / S;                                  // merged rows per CTA
@@ -217,6 +209,9 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.vc)) : "memory");
     }
     __syncthreads();
+    // every CTA of the cluster has started before any pushes into another's shared memory (the
+    // matching wait comes after the key loop)
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     pdl_wait();
     const int L = a.ctx_len[b];
     // the sequence's tiles: ceil(L / 64) context tiles, then the block tile; split s takes a
@@ -260,7 +255,6 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
     bool timed_out = false;
-    if (n_tiles == 0) asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
     if (n_tiles > 0) {
         const bf16* q = static_cast<const bf16*>(a.q);
         const uint32_t sQ = smem_addr(Qs);
@@ -284,9 +278,6 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             const int row = warp * 16 + (lane & 15), col = kk * 16 + (lane >> 4) * 8;
             ldsm_x4(sQ + (uint32_t)(row * LD + col) * 2, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
         }
-        // the query tile is in registers: its memory may now receive the cluster's partials (the
-        // arrive releases the reads above; the pushing CTAs wait on it after their key loops)
-        asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
         for (int t = 0; t < n_tiles; ++t) {
             const int st = t % kNST;
             if (tid == 0 && prod_ok && issued < n_tiles) refill();   // tile t + kNST - 1
@@ -357,25 +348,22 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
                 l0 += sc[nt][0] + sc[nt][1];
                 l1 += sc[nt][2] + sc[nt][3];
             }
-            // O += P V (P from registers as the A operand, as a high and a low bf16 part; V tiles
-            // transposed by ldmatrix)
+            // O += P V (P from registers as the A operand; V tiles transposed by ldmatrix)
 #pragma unroll
             for (int kk = 0; kk < kKT / 16; ++kk) {
-                uint32_t ph[4], pl[4];
-                split_bf16(sc[2 * kk][0], sc[2 * kk][1], ph[0], pl[0]);
-                split_bf16(sc[2 * kk][2], sc[2 * kk][3], ph[1], pl[1]);
-                split_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ph[2], pl[2]);
-                split_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ph[3], pl[3]);
+                uint32_t pa[4];
+                pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+                pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+                pa[2] = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+                pa[3] = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
 #pragma unroll
                 for (int nt = 0; nt < HD / 8; nt += 2) {
                     const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                     const int c8 = nt + (lane >> 4);
                     uint32_t b0, b1, b2, b3;
                     ldsm_x4_t(sV + swz(row, c8), b0, b1, b2, b3);
-                    mma16816(o[nt], ph, b0, b1);
-                    mma16816(o[nt + 1], ph, b2, b3);
-                    mma16816(o[nt], pl, b0, b1);
-                    mma16816(o[nt + 1], pl, b2, b3);
+                    mma16816(o[nt], pa, b0, b1);
+                    mma16816(o[nt + 1], pa, b2, b3);
                 }
             }
             __syncwarp();
@@ -396,17 +384,17 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     __syncthreads();
     asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
     // push the partial: query row r belongs to the merge slice of CTA r / RP, which keeps it at
-    // [s * RP + r % RP]; O is normalised by l first. The rows are staged in this CTA's (now idle)
-    // tile memory so that the remote stores are 16 bytes wide.
+    // [s * RP + r % RP]; O is normalised by l first (|O / l| <= max |V|, safe in fp16). The rows
+    // are staged in this CTA's (now idle) tile memory so that the remote stores are 16 bytes wide.
     {
-        float* stg = reinterpret_cast<float*>(smem);   // [kQT][HD]
+        __half* stg = reinterpret_cast<__half*>(smem);   // [kQT][HD]
         const int r0 = warp * 16 + (lane >> 2), r1 = r0 + 8;
         const float i0 = l0 > 0.f ? 1.0f / l0 : 0.f, i1 = l1 > 0.f ? 1.0f / l1 : 0.f;
 #pragma unroll
         for (int nt = 0; nt < HD / 8; ++nt) {
             const int col = nt * 8 + (lane & 3) * 2;
-            *reinterpret_cast<float2*>(stg + r0 * HD + col) = make_float2(o[nt][0] * i0, o[nt][1] * i0);
-            *reinterpret_cast<float2*>(stg + r1 * HD + col) = make_float2(o[nt][2] * i1, o[nt][3] * i1);
+            *reinterpret_cast<__half2*>(stg + r0 * HD + col) = __floats2half2_rn(o[nt][0] * i0, o[nt][1] * i0);
+            *reinterpret_cast<__half2*>(stg + r1 * HD + col) = __floats2half2_rn(o[nt][2] * i1, o[nt][3] * i1);
         }
         if ((lane & 3) == 0) {
             *reinterpret_cast<float2*>(cluster.map_shared_rank(rML, r0 / RP) + 2 * (s * RP + r0 % RP)) =
@@ -415,10 +403,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
                 make_float2(m1, l1);
         }
         __syncthreads();
-        for (int k = tid; k < kQT * (HD / 4); k += blockDim.x) {
-            const int r = k / (HD / 4), pc = k % (HD / 4);
-            *reinterpret_cast<float4*>(cluster.map_shared_rank(rO, r / RP) + (size_t)(s * RP + r % RP) * HD + pc * 4) =
-                *reinterpret_cast<const float4*>(stg + r * HD + pc * 4);
+        for (int k = tid; k < kQT * PIECES; k += blockDim.x) {
+            const int r = k / PIECES, pc = k % PIECES;
+            *reinterpret_cast<uint4*>(cluster.map_shared_rank(rO, r / RP) + (size_t)(s * RP + r % RP) * HD + pc * 8) =
+                *reinterpret_cast<const uint4*>(stg + r * HD + pc * 8);
         }
     }
     // every partial has arrived; after this barrier no CTA touches another's shared memory
@@ -449,7 +437,7 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             float v0 = 0.f, v1 = 0.f;
 #pragma unroll
             for (int p = 0; p < S; ++p) {
-                const float2 f = *reinterpret_cast<const float2*>(rO + (size_t)(p * RP + lr) * HD + lt * EPT + q);
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(rO + (size_t)(p * RP + lr) * HD + lt * EPT + q));
                 v0 = fmaf(w[p], f.x, v0);
                 v1 = fmaf(w[p], f.y, v1);
             }
@@ -549,10 +537,9 @@ __global__ void attn_combine_kernel(const AttnArgs a, T* __restrict__ out) {
 }
 
 template <int HD>
-size_t mma_smem_bytes() {   // alignment pad, K/V stages, padded Q tile / pushed fp32 partials, barriers
-    return 1024 + (size_t)kNST * 2 * HD * 128 +
-           std::max((size_t)kQT * (HD + 8) * sizeof(bf16), (size_t)kQT * HD * sizeof(float)) +
-           (size_t)kQT * 2 * sizeof(float) + 2 * 8 * kNST;
+size_t mma_smem_bytes() {   // alignment pad, K/V stages, padded Q tile, pushed partials, barriers
+    return 1024 + (size_t)kNST * 2 * HD * 128 + (size_t)kQT * (HD + 8) * sizeof(bf16) +
+           (size_t)kQT * HD * sizeof(__half) + (size_t)kQT * 2 * sizeof(float) + 2 * 8 * kNST;
 }
 
 template <int HD, int S>
