@@ -183,8 +183,8 @@ __global__ void __launch_bounds__(256) fuse_layers_kernel(
     }
 }
 
-// Many positions (context fill): a persistent grid of one CTA per SM walks the positions (no
-// cluster). Warp-specialised: the last warp's first thread streams the T target rows of each
+// Many positions (context fill): a persistent grid of one or two CTAs per SM walks the positions
+// (no cluster). Warp-specialised: the last warp's first thread streams the T target rows of each
 // position (d contiguous elements each) through a ring of `ns` shared-memory stages of kRB rows as
 // 1-D bulk copies, the stage sequence running on across positions; the other warps (one thread
 // per 8 features) consume the stages. Each stage has a "full" mbarrier (the copies landed) and an
@@ -220,14 +220,46 @@ __device__ __forceinline__ bool fill_wait(uint32_t bar, uint32_t parity, volatil
     }
 }
 
+// Two fp32 lanes in one 64-bit register: the fill's sums use the paired FMA (fma.rn.f32x2, each
+// lane rounded as a scalar fmaf), which halves the instructions of the 8 x D FMAs per row.
+typedef unsigned long long f32x2;
+__device__ __forceinline__ f32x2 pk2(float lo, float hi) {
+    f32x2 r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void upk2(f32x2 v, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ f32x2 fma2(f32x2 a, f32x2 b, f32x2 c) {
+    f32x2 r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+// 8 consecutive elements of a staged row as four fp32 pairs
+__device__ __forceinline__ void load8x2(const bf16* p, f32x2* h) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) h[q] = pk2(__uint_as_float(w[q] << 16), __uint_as_float(w[q] & 0xFFFF0000u));
+}
+__device__ __forceinline__ void load8x2(const float* p, f32x2* h) {
+    const float4 a = *reinterpret_cast<const float4*>(p), b = *reinterpret_cast<const float4*>(p + 4);
+    h[0] = pk2(a.x, a.y);
+    h[1] = pk2(a.z, a.w);
+    h[2] = pk2(b.x, b.y);
+    h[3] = pk2(b.z, b.w);
+}
+
 template <class T, int DMAX>
-__global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
+__device__ __forceinline__ void fuse_rows_body(
     const T* __restrict__ H, const float* __restrict__ alpha, const T* __restrict__ gain,
     T* __restrict__ F, T* __restrict__ F_out, const int32_t* __restrict__ app_cnt, int D, int Tn,
     int batch, int n_max, int d, long long f_layer_rows, float eps, int ns, uint32_t* err) {
     pdl_trigger();
     extern __shared__ __align__(128) uint8_t stage_mem[];   // [ns][kRB][d]
-    __shared__ __align__(16) float s_alpha[64 * DMAX];       // [j][i] (Tn <= 64)
+    constexpr int DP = (DMAX + 1) & ~1;                       // DMAX rounded up to even
+    __shared__ __align__(16) f32x2 s_alpha[64 * DP];          // [j][i] = (alpha_ij, alpha_ij), Tn <= 64
     __shared__ float red[16][DMAX];
     __shared__ float inv_s[DMAX];
     __shared__ __align__(8) uint64_t full_bar[kMaxNS], empty_bar[kMaxNS];
@@ -247,12 +279,11 @@ __global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     pdl_wait();
-    for (int k = tid; k < D * Tn; k += blockDim.x) {
-        const int i = k / Tn, j = k % Tn;
-        s_alpha[j * DMAX + i] = alpha[k];
+    for (int k = tid; k < Tn * DP; k += blockDim.x) {
+        const int j = k / DP, i = k % DP;
+        const float a = i < D ? alpha[i * Tn + j] : 0.f;
+        s_alpha[k] = pk2(a, a);
     }
-    for (int k = tid; k < Tn * DMAX; k += blockDim.x)
-        if (k % DMAX >= D) s_alpha[k] = 0.f;
     __syncthreads();
     volatile int* abrt = &abort_flag;
     const int n_pos = batch * n_max;
@@ -311,11 +342,11 @@ __global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
         bool ok = true;
         for (int pid = first; pid < n_pos && ok; pid = next_pos(pid)) {
             const int b = pid / n_max, r = pid % n_max;
-            float acc[DMAX][8];
+            f32x2 acc2[DMAX][4];
 #pragma unroll
             for (int i = 0; i < DMAX; ++i)
 #pragma unroll
-                for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
+                for (int q = 0; q < 4; ++q) acc2[i][q] = 0ull;
             for (int k = 0; k < nst; ++k, ++g) {
                 const int st = g % ns;
                 if (!fill_wait(fb0 + 8u * st, (uint32_t)((g / ns) & 1), abrt)) {
@@ -327,20 +358,18 @@ __global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
                     for (int u = 0; u < kRB; ++u) {
                         const int j = k * kRB + u;
                         if (j >= Tn) break;
-                        float h[8], a[DMAX];
-                        load8(stg + (size_t)(st * kRB + u) * d + e0, h);
+                        f32x2 h[4], a[DP];
+                        load8x2(stg + (size_t)(st * kRB + u) * d + e0, h);
 #pragma unroll
-                        for (int i = 0; i < DMAX; i += 4) {
-                            const float4 a4 = *reinterpret_cast<const float4*>(&s_alpha[j * DMAX + i]);
-                            a[i] = a4.x;
-                            a[i + 1] = a4.y;
-                            a[i + 2] = a4.z;
-                            a[i + 3] = a4.w;
+                        for (int i = 0; i < DP; i += 2) {
+                            const uint4 a4 = *reinterpret_cast<const uint4*>(&s_alpha[j * DP + i]);
+                            a[i] = ((f32x2)a4.y << 32) | a4.x;
+                            a[i + 1] = ((f32x2)a4.w << 32) | a4.z;
                         }
 #pragma unroll
                         for (int i = 0; i < DMAX; ++i)
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[i][e] = fmaf(a[i], h[e], acc[i][e]);
+                            for (int q = 0; q < 4; ++q) acc2[i][q] = fma2(a[i], h[q], acc2[i][q]);
                     }
                 }
                 __syncwarp();
@@ -350,6 +379,11 @@ __global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
             // the abort flag, which every other consumer sees at the barrier below
             asm volatile("bar.sync 1, %0;" ::"r"(n_ct) : "memory");
             if (!ok || *abrt) break;
+            float acc[DMAX][8];
+#pragma unroll
+            for (int i = 0; i < DMAX; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) upk2(acc2[i][q], acc[i][2 * q], acc[i][2 * q + 1]);
 #pragma unroll
             for (int i = 0; i < DMAX; ++i) {
                 float v = 0.f;
@@ -383,6 +417,24 @@ __global__ void __launch_bounds__(544, 1) fuse_rows_kernel(
     __syncthreads();
 }
 
+#define FUSE_ROWS_PARAMS                                                                            \
+    const T *__restrict__ H, const float *__restrict__ alpha, const T *__restrict__ gain,           \
+        T *__restrict__ F, T *__restrict__ F_out, const int32_t *__restrict__ app_cnt, int D,         \
+        int Tn, int batch, int n_max, int d, long long f_layer_rows, float eps, int ns, uint32_t *err
+#define FUSE_ROWS_ARGS H, alpha, gain, F, F_out, app_cnt, D, Tn, batch, n_max, d, f_layer_rows, eps, ns, err
+// one CTA per SM (up to 512 consumer threads), or two per SM for d <= 2560 and D <= 5 (registers
+// capped; eight sums of eight features do not fit without spills)
+template <class T, int DMAX>
+__global__ void __launch_bounds__(544, 1) fuse_rows_kernel(FUSE_ROWS_PARAMS) {
+    fuse_rows_body<T, DMAX>(FUSE_ROWS_ARGS);
+}
+template <class T, int DMAX>
+__global__ void __launch_bounds__(352, 2) fuse_rows2_kernel(FUSE_ROWS_PARAMS) {
+    fuse_rows_body<T, DMAX>(FUSE_ROWS_ARGS);
+}
+#undef FUSE_ROWS_PARAMS
+#undef FUSE_ROWS_ARGS
+
 template <class T>
 cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,
                           cudaStream_t s) {
@@ -394,19 +446,18 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
     const T* gain = static_cast<const T*>(c->w.fuse_norm);
     T* F = static_cast<T*>(c->fused);
     T* Fo = static_cast<T*>(fused_out);
-    // context fill: one warp-specialised CTA per SM (d / 8 consumer threads and a producer warp),
-    // a ring of as many kRB-row stages as fit in about 200 KB (at most kMaxNS)
+    // context fill: warp-specialised CTAs of d / 8 consumer threads and a producer warp, two per SM
+    // when their registers allow (rings of about 100 KB), else one (about 200 KB); at most kMaxNS
+    // stages of kRB rows
     const int cthreads = ((g.d / 8 + 31) / 32) * 32;
     const size_t stage_bytes = (size_t)kRB * g.d * sizeof(T);
-    const int ns = (int)std::min<size_t>(kMaxNS, (200 * 1024) / stage_bytes);
-    if ((long long)c->batch * n_max >= 2LL * c->num_sms && ns >= 3 && cthreads <= 512 &&
-        g.n_draft_layers <= 8 && g.n_target_layers <= 64) {
-        auto rk = g.n_draft_layers <= 4 ? fuse_rows_kernel<T, 4> : fuse_rows_kernel<T, 8>;
+    if ((long long)c->batch * n_max >= 2LL * c->num_sms && cthreads <= 512 && g.n_draft_layers <= 8 &&
+        g.n_target_layers <= 64 && 3 * stage_bytes <= 200 * 1024) {
         const int threads = cthreads + 32;
-        const size_t rsmem = (size_t)ns * stage_bytes;
         static PerDeviceOnce rconf;
         const cudaError_t re = rconf([] {
-            for (auto k : {fuse_rows_kernel<T, 4>, fuse_rows_kernel<T, 8>}) {
+            for (auto k : {fuse_rows_kernel<T, 4>, fuse_rows_kernel<T, 5>, fuse_rows_kernel<T, 8>,
+                           fuse_rows2_kernel<T, 4>, fuse_rows2_kernel<T, 5>, fuse_rows2_kernel<T, 8>}) {
                 cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                      200 * 1024);
                 if (e != cudaSuccess) return e;
@@ -414,11 +465,22 @@ cudaError_t fuse_layers_t(dflare_ctx* c, const void* hidden, int n_max, void* fu
             return cudaSuccess;
         });
         if (re != cudaSuccess) return re;
-        int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rk, threads, rsmem) != cudaSuccess || per_sm < 1)
-            per_sm = 1;
+        const int Dn = g.n_draft_layers;
+        auto rk1 = Dn <= 4 ? fuse_rows_kernel<T, 4> : Dn == 5 ? fuse_rows_kernel<T, 5> : fuse_rows_kernel<T, 8>;
+        auto rk2 = Dn <= 4 ? fuse_rows2_kernel<T, 4> : Dn == 5 ? fuse_rows2_kernel<T, 5> : fuse_rows2_kernel<T, 8>;
+        auto rk = rk1;
+        int ns = (int)std::min<size_t>(kMaxNS, (200 * 1024) / stage_bytes), per_sm = 1;
+        const int ns2 = (int)std::min<size_t>(kMaxNS, (100 * 1024) / stage_bytes);
+        int fit = 0;
+        if (threads <= 352 && Dn <= 5 && ns2 >= 3 &&
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&fit, rk2, threads, (size_t)ns2 * stage_bytes) ==
+                cudaSuccess && fit >= 2) {
+            rk = rk2;
+            ns = ns2;
+            per_sm = 2;
+        }
         const int grid = (int)std::min<long long>((long long)c->batch * n_max, (long long)per_sm * c->num_sms);
-        return launch_kernel(c->pdl, rk, dim3(grid), dim3(threads), rsmem, s, H,
+        return launch_kernel(c->pdl, rk, dim3(grid), dim3(threads), (size_t)ns * stage_bytes, s, H,
                              (const float*)c->alpha, gain, F, Fo, (const int32_t*)c->app_cnt,
                              g.n_draft_layers, g.n_target_layers, c->batch, n_max, g.d,
                              (long long)g.max_fuse_rows, g.rms_eps, ns, c->err);
