@@ -4,16 +4,18 @@
 One step = one block step of the path on the workload's batch: fuse the previous step's
 accepted positions (Eq. 3, Eq. 4) -> draft a block (Sec. 3.2) -> synthetic target argmax ->
 prefix acceptance (Sec. 3.2). Inputs are seeded synthetic tensors shaped like the named drafter
-(weights N(0, 0.02), target states N(0,1) x U(0.5, 4) per layer). The default workload is the
-Qwen3-4B-shaped drafter: d 2560, 5 draft layers, 36 fused target layers, context 2048, block 16,
-batch 1.
+(weights N(0, 0.02), target states N(0,1) x U(0.5, 4) per layer). The headline workload is the
+largest single-GPU one, the Qwen3-8B-shaped drafter at batch 4: d 4096, 8 draft layers, 36 fused
+target layers, block 16, ragged contexts U{1024..4096}; the line's `configs` object holds the same
+measurement for the other drafter shapes (tiny fp32, Qwen3-4B, Qwen3-8B batch 1, GPT-OSS-20B
+batch 2).
 
 Prints one JSON line (rank 0). `value` = drafted tokens/s (batch x (B-1) per step) over the
 timed CUDA-graph replays with inputs resident in HBM; `e2e` = the same metric through the public
 calls with the step's inputs copied from pinned host memory and results read back every step;
-`roofline` = the dominant kernel's algorithmic bytes per launch / its event-timed duration vs
-the measured HBM copy bandwidth; `cpu_baseline` = the CPU oracle on a bounded sample.
-`--impl reference` times the CPU oracle alone (the reference arm of this build).
+`roofline` = the dominant kernel's (the projection GEMM's) algorithmic bytes over its
+event-timed launch durations vs the measured HBM copy bandwidth; `cpu_baseline` = the CPU oracle
+on a bounded sample. `--impl reference` times the CPU oracle alone (the reference arm).
 """
 from __future__ import annotations
 
@@ -43,7 +45,18 @@ def parse():
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--workload", default="qwen3_4b", choices=sorted(synth.PRESETS))
+    p.add_argument("--workload", default=HEADLINE, choices=sorted(synth.PRESETS))
+    p.add_argument("--headline-only", action="store_true",
+                   help="measure the --workload only (no per-config sub-objects)")
+    p.add_argument("--draft-layers", type=int, default=0,
+                   help="override D of --workload (a smaller case for profiling); implies --headline-only")
+    p.add_argument("--vocab", type=int, default=0,
+                   help="override the vocabulary of --workload; implies --headline-only")
+    p.add_argument("--batch", type=int, default=0,
+                   help="override the batch of --workload (every context as long as the longest); "
+                        "implies --headline-only")
+    p.add_argument("--sub-cpu-seconds", type=float, default=6.0,
+                   help="CPU time budget of the oracle steps of each non-headline workload")
     p.add_argument("--e2e-steps", type=int, default=50)
     p.add_argument("--breakdown-steps", type=int, default=30)
     p.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -132,8 +145,7 @@ def run_reference(args):
         "warmup": args.warmup, "ms_per_step": 1e3 * dt / n, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": w.name, "batch": w.batch, "block": w.shape.block,
-                   "ctx": list(w.ctx_lens)},
+        "config": config_of(w),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -432,9 +444,12 @@ def sampled_steps(w, dev_w, fill_chunks, hid_step, x0, reps=100, temperature=1.0
     return out
 
 
-def graph_breakdown(lib, cs, step, nb):
-    """Per-launch durations: a second CUDA graph of one step with CUDA events recorded by the
-    library's trace hook around every launch, replayed nb times. Returns name -> [ms, ...]."""
+def graph_breakdown(lib, cs, step, nb, only=None):
+    """Per-launch durations: a CUDA graph of one step with CUDA events recorded by the library's
+    trace hook around every launch (or, with `only`, around the launches whose call-site name it
+    accepts; the other launches keep their programmatic dependent launch), replayed nb times.
+    Returns (name -> [ms, ...], ms per traced step). An event pair around a launch also holds that
+    launch's own launch latency, which inside the untraced graph overlaps the previous kernel."""
     import torch
     import paper_2606_02091_gb300 as P
     cr = Cudart()
@@ -443,11 +458,14 @@ def graph_breakdown(lib, cs, step, nb):
 
     @P._lib.TRACE_FN
     def ev_cb(user, name, phase, stream):
+        n = name.decode()
+        if only is not None and not only(n):
+            return
         if len(pool) <= len(rec):
             pool.append(cr.event())
         e = pool[len(rec)]
         cr.record(e, stream)
-        rec.append((name.decode(), phase, e))
+        rec.append((n, phase, e))
 
     L_ = P.load()
     L_.dflare_set_trace(lib.raw, ev_cb, None)
@@ -458,9 +476,14 @@ def graph_breakdown(lib, cs, step, nb):
     L_.dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
     torch.cuda.synchronize()
     per = {}
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    total = 0.0
     for _ in range(nb):
+        t0.record()
         g2.replay()
+        t1.record()
         torch.cuda.synchronize()
+        total += t0.elapsed_time(t1)
         open_ev = {}
         for name, phase, e in rec:
             if phase == 0:
@@ -469,7 +492,61 @@ def graph_breakdown(lib, cs, step, nb):
                 st = open_ev[name].pop()
                 per.setdefault(name, []).append(cr.elapsed(st, e))
     del g2
-    return per
+    return per, total / max(nb, 1)
+
+
+def gemm_timeline(lib, cs, step, nb, slots=256):
+    """Device-side times of every projection-GEMM launch of one step inside a CUDA graph of the
+    step with nothing added between its launches (dflare_set_timing: %globaltimer at the first
+    CTA's entry, at the first CTA's activation dependency, at the last CTA's exit), replayed nb
+    times. Returns (names, [[(entry, ready, exit) ns per launch] per replay])."""
+    import torch
+    import paper_2606_02091_gb300 as P
+    names = []
+
+    @P._lib.TRACE_FN
+    def name_cb(user, name, phase, stream):
+        n = name.decode()
+        if phase == 0 and n.startswith("gemm_"):
+            names.append(n)
+
+    L_ = P.load()
+    stamps = torch.empty(3 * slots, dtype=torch.int64, device="cuda")
+    L_.dflare_set_trace(lib.raw, name_cb, None)
+    lib.set_timing(stamps, slots)
+    g3 = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(cs):
+        with torch.cuda.graph(g3, stream=cs):
+            step()
+    lib.set_timing()
+    L_.dflare_set_trace(lib.raw, P._lib.TRACE_FN(), None)
+    torch.cuda.synchronize()
+    n = min(len(names), slots)
+    runs = []
+    for _ in range(nb):
+        stamps[:2 * slots].fill_(-1)
+        stamps[2 * slots:].zero_()
+        g3.replay()
+        torch.cuda.synchronize()
+        a = stamps.cpu().numpy().view(np.uint64)
+        runs.append([(int(a[k]), int(a[slots + k]), int(a[2 * slots + k])) for k in range(n)])
+    del g3
+    return names[:n], runs
+
+
+def union_ns(spans):
+    """Total length of the union of [start, end) intervals."""
+    tot, cur_s, cur_e = 0, None, None
+    for s0, e0 in sorted(spans):
+        if cur_e is None or s0 > cur_e:
+            if cur_e is not None:
+                tot += cur_e - cur_s
+            cur_s, cur_e = s0, e0
+        else:
+            cur_e = max(cur_e, e0)
+    if cur_e is not None:
+        tot += cur_e - cur_s
+    return tot
 
 
 def replica_aggregate(ms, units_per_step, steps, dist=None, device="cuda"):
@@ -486,31 +563,41 @@ def replica_aggregate(ms, units_per_step, steps, dist=None, device="cuda"):
     return ms, world * units_per_step * steps / (ms / 1e3)
 
 
-def run_ours(args):
+def config_of(w):
+    """The `config` object of a bench line (both arms print the same keys)."""
+    s = w.shape
+    return {"workload": w.name, "dtype": s.dtype, "d": s.d, "draft_layers": s.n_draft_layers,
+            "target_layers": s.n_target_layers, "heads": [s.n_q_heads, s.n_kv_heads],
+            "head_dim": s.head_dim, "ffn": s.ffn, "vocab": s.vocab, "block": s.block,
+            "batch": w.batch, "ctx": list(w.ctx_lens), "match_p": w.match_p}
+
+
+# the benchmark's workloads: the headline (the largest single-GPU workload: Qwen3-8B-shaped,
+# ragged batch 4) and the other drafter shapes, each measured the same way
+HEADLINE = "qwen3_8b_b4"
+CONFIG_SET = ("tiny_f32", "qwen3_4b", "qwen3_8b_b1", "qwen3_8b_b4", "gptoss_20b_b2")
+N_ROT = 4     # per-step target-state buffers rotated through the timed steps
+
+
+def measure(w, args, steps, warmup, e2e_steps, nb, cpu_seconds, extras, dist=None, world=1,
+            rank=0, local=0):
+    """One workload: context fill, then `steps` timed block steps (CUDA-graph replays, inputs
+    resident in HBM), the per-launch breakdown, the end-to-end loop through the public calls
+    and, optionally, the fusion variants, the sampled path and the CPU oracle. Returns the
+    measurement as a dict (the fields of a bench line)."""
     import torch
     import paper_2606_02091_gb300 as P
     from paper_2606_02091_gb300 import DFlare, synthetic_target
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    w = synth.preset(args.workload)
     s = w.shape
-    K, Wm = args.steps, max(args.warmup, 3)
-    E = args.e2e_steps
+    K, Wm, E = steps, max(warmup, 3), e2e_steps
     W = synth.weights(w)
     dev_w = {}
     for k, v in W.items():
         t = torch.from_numpy(v)
         dev_w[k] = (t.view(torch.bfloat16) if v.dtype == np.uint16 else t).cuda()
     chunk = min(args.fill_chunk, max(w.ctx_lens))
-    n_steps_total = Wm + K + E + args.breakdown_steps + 16
+    n_steps_total = Wm + K + E + nb + 16
     max_ctx = max(w.ctx_lens) + s.block * n_steps_total
     lib = DFlare.from_shape(s, max_batch=w.batch, max_ctx=max_ctx,
                             max_fuse_rows=w.batch * max(chunk, s.block),
@@ -518,8 +605,8 @@ def run_ours(args):
     lib.set_weights(dev_w)
     lib.reset(w.batch)
     # context fill in chunks (the target's prompt states): once untimed, then again from an empty
-    # context with CUDA events around the fusion and context-projection launches (Sec. 8 K1/K2
-    # are measured at fill, where n = L positions per call)
+    # context with CUDA events around the fusion and context-projection launches (the fusion and
+    # the context K/V projection are measured at fill, where n = L positions per call)
     dt_np = np.uint16 if s.dtype == "bf16" else np.float32
     fill_chunks = []
     for pos0 in range(0, max(w.ctx_lens), chunk):
@@ -531,6 +618,7 @@ def run_ours(args):
         Ht = torch.from_numpy(H)
         fill_chunks.append(((Ht.view(torch.bfloat16) if dt_np == np.uint16 else Ht).cuda(),
                             torch.tensor(ns, dtype=torch.int32, device="cuda")))
+        del H, Ht
     fill_ev = []
     crf = Cudart()
 
@@ -560,14 +648,17 @@ def run_ours(args):
     e_sz = 2 if s.dtype == "bf16" else 4
     fuse_bytes = n_fill * (s.n_target_layers + s.n_draft_layers) * s.d * e_sz
     kv_flops = 2.0 * n_fill * s.n_draft_layers * 2 * s.d_kv * s.d
-    # per-step buffers: target states of up to B newly committed positions, draws of the
+    # per-step buffers: target states of up to B newly committed positions (N_ROT different
+    # buffers, used in turn, so no step fuses the rows the step before it fused), draws of the
     # synthetic target for n_tab steps, and the loop state (accept_len doubles as next n_new)
-    Hs = np.zeros((s.n_target_layers, w.batch, s.block, s.d), dt_np)
-    for b, L in enumerate(w.ctx_lens):
-        Hs[:, b] = synth.hidden_states(w, b, L, s.block)
-    hid_host = torch.from_numpy(Hs)
-    hid_host = hid_host.view(torch.bfloat16) if dt_np == np.uint16 else hid_host
-    hid_step = hid_host.cuda()
+    hid_host = []
+    for rot in range(N_ROT):
+        Hs = np.zeros((s.n_target_layers, w.batch, s.block, s.d), dt_np)
+        for b, L in enumerate(w.ctx_lens):
+            Hs[:, b] = synth.hidden_states(w, b, L + rot * s.block, s.block)
+        t = torch.from_numpy(Hs)
+        hid_host.append(t.view(torch.bfloat16) if dt_np == np.uint16 else t)
+    hid_dev = [h.cuda() for h in hid_host]
     n_tab = 1024
     u, r, last = synth.target_draws(w, 0, n_tab)
     u_d = torch.from_numpy(u.view(np.int32)).cuda()
@@ -580,11 +671,13 @@ def run_ours(args):
     tgt = torch.zeros((w.batch, s.block), dtype=torch.int32, device="cuda")
     thr = synth.accept_threshold(w.match_p)
 
-    def step():
-        lib.fuse_context(hid_step, acc)
-        lib.draft_block(nxt, draft)
-        synthetic_target(draft, u_d, r_d, last_d, step_ctr, thr, w.batch, s.block, tgt)
-        lib.verify_accept(draft, tgt, acc, nxt)
+    def step_on(hid):
+        def step():
+            lib.fuse_context(hid, acc)
+            lib.draft_block(nxt, draft)
+            synthetic_target(draft, u_d, r_d, last_d, step_ctr, thr, w.batch, s.block, tgt)
+            lib.verify_accept(draft, tgt, acc, nxt)
+        return step
 
     # launch counting through the trace hook
     counts = {}
@@ -597,8 +690,8 @@ def run_ours(args):
 
     L_ = P.load()
     L_.dflare_set_trace(lib.raw, count_cb, None)
-    for _ in range(3):
-        step()
+    for i in range(3):
+        step_on(hid_dev[i % N_ROT])()
     torch.cuda.synchronize()
     kpt = kernels_per_trace(s)
     launches_per_step = sum(kpt.get(k, 1) * v for k, v in counts.items()) / 3 + 1
@@ -606,15 +699,18 @@ def run_ours(args):
 
     cs = torch.cuda.Stream()
     cs.wait_stream(torch.cuda.current_stream())
-    graph = torch.cuda.CUDAGraph()
+    graphs = []
     with torch.cuda.stream(cs):
-        step()
-        torch.cuda.synchronize()
-        with torch.cuda.graph(graph, stream=cs):
-            step()
+        for h in hid_dev:
+            g = torch.cuda.CUDAGraph()
+            step_on(h)()
+            torch.cuda.synchronize()
+            with torch.cuda.graph(g, stream=cs):
+                step_on(h)()
+            graphs.append(g)
     torch.cuda.synchronize()
-    for _ in range(Wm):
-        graph.replay()
+    for i in range(Wm):
+        graphs[i % N_ROT].replay()
     torch.cuda.synchronize()
     if lib.device_error():
         raise RuntimeError("device error during warmup")
@@ -629,8 +725,8 @@ def run_ours(args):
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record()
-    for _ in range(K):
-        graph.replay()
+    for i in range(K):
+        graphs[i % N_ROT].replay()
     ev1.record()
     torch.cuda.synchronize()
     if dist:
@@ -642,11 +738,12 @@ def run_ours(args):
     mean_tau = (sum(lens1) - sum(lens0)) / (K * w.batch)
     drafted_per_step = w.batch * (s.block - 1)
     ms, value = replica_aggregate(ms, drafted_per_step, K, dist)
+    ms_step = ms / K
 
     # ---------------- per-kernel durations (CUDA events around every launch, graph replays)
-    nb = args.breakdown_steps
-    t_b0 = time.perf_counter()
-    per = graph_breakdown(lib, cs, step, nb)
+    hbm, peak_src, peaks = measured_peaks()
+    step0 = step_on(hid_dev[0])
+    per, traced_ms = graph_breakdown(lib, cs, step0, nb)
     kernels = {}
     for name, ts in per.items():
         launches = len(ts) / nb
@@ -656,36 +753,88 @@ def run_ours(args):
                          "us_per_step": avg_us * launches,
                          "algorithmic_bytes": ab,
                          "gbs": (ab / (avg_us * 1e-6) / 1e9) if ab else None}
-    hbm, peak_src, peaks = measured_peaks()
-    # dominant kernel: the tcgen05 projection GEMM (every gemm_* call site launches it); its
-    # achieved bandwidth is the step's algorithmic GEMM bytes over the summed launch durations
-    gk = [k for k in kernels if k.startswith("gemm_")]
-    g_bytes = sum(kernels[k]["algorithmic_bytes"] * kernels[k]["launches_per_step"] for k in gk)
-    g_us = sum(kernels[k]["us_per_step"] for k in gk)
+        if kernels[name]["gbs"]:
+            kernels[name]["frac_of_hbm"] = kernels[name]["gbs"] / hbm
+        if kernels[name]["us_per_step"] > 1e3 * traced_ms:
+            raise RuntimeError(f"{name}: {kernels[name]['us_per_step']:.1f} us per step measured "
+                               f"inside a {1e3 * traced_ms:.1f} us traced step")
+    # dominant kernel: the tcgen05 projection GEMM (every gemm_* call site launches it), timed on
+    # the device inside the step's own graph (no events between launches): each launch's span runs
+    # from its first CTA's entry to its last CTA's exit; the step's GEMM time is the union of the
+    # spans (a span can start early, next to the previous kernel's tail, under programmatic
+    # dependent launch), achieved = the step's algorithmic GEMM bytes over that time
+    names, runs = gemm_timeline(lib, cs, step0, nb) if s.dtype == "bf16" else ([], [])
+    timed = [run for run in runs if run and all(x[2] > 0 and x[0] < 2 ** 63 for x in run)]
+    if timed:
+        g_bytes = sum(algorithmic_bytes(w, k, mean_tau) for k in names)
+        g_us = float(np.mean([union_ns([(x[0], x[2]) for x in run]) for run in timed])) / 1e3
+        g_dep_us = float(np.mean([sum(x[2] - min(max(x[1], x[0]), x[2]) for x in run) for run in timed])) / 1e3
+        span = {}
+        for run in timed:
+            for lname, st3 in zip(names, run):
+                span.setdefault(lname, []).append((st3[2] - st3[0]) / 1e3)
+        dep = {}
+        gaps = {}
+        for run in timed:
+            for li, (lname, st3) in enumerate(zip(names, run)):
+                dep.setdefault(lname, []).append((st3[2] - max(st3[1], st3[0])) / 1e3)
+                if li + 1 < len(run):   # from this launch's exit to the next GEMM's dependency
+                    nx3 = run[li + 1]
+                    gaps.setdefault(f"{lname} -> {names[li + 1]}", []).append((max(nx3[1], nx3[0]) - st3[2]) / 1e3)
+        per_launch = {k: {"launches_per_step": names.count(k),
+                          "avg_span_us": float(np.mean(v)),
+                          "avg_after_dependency_us": float(np.mean(dep[k])),
+                          "frac_of_hbm": algorithmic_bytes(w, k, mean_tau) / (float(np.mean(v)) * 1e-6) / 1e9 / hbm,
+                          "frac_of_hbm_after_dependency":
+                              algorithmic_bytes(w, k, mean_tau) / (float(np.mean(dep[k])) * 1e-6) / 1e9 / hbm}
+                      for k, v in span.items()}
+        between = {k: float(np.mean(v)) for k, v in gaps.items()}
+        how = ("%globaltimer stamps of every GEMM launch inside the step's CUDA graph "
+               "(dflare_set_timing): first-CTA entry to last-CTA exit; us_per_step = union of "
+               "the spans over a step")
+    else:   # fp32 drafter (CUDA-core GEMM): CUDA events around the GEMM launches
+        per_g, _ = graph_breakdown(lib, cs, step0, nb, only=lambda n: n.startswith("gemm_"))
+        names = [k for k, ts in per_g.items() for _ in range(len(ts) // nb)]
+        g_bytes = sum(algorithmic_bytes(w, k, mean_tau) * len(ts) / nb for k, ts in per_g.items())
+        g_us = sum(1e3 * float(np.sum(ts)) / nb for ts in per_g.values())
+        g_dep_us = None
+        per_launch = {k: {"launches_per_step": len(ts) / nb, "avg_span_us": 1e3 * float(np.mean(ts)),
+                          "frac_of_hbm": algorithmic_bytes(w, k, mean_tau) / (1e-3 * float(np.mean(ts))) / 1e9 / hbm}
+                      for k, ts in per_g.items()}
+        how = "CUDA events around the GEMM launches only, in a replay of the step's graph"
+        between = {}
+    if g_us > 1e3 * ms_step:
+        raise RuntimeError(f"GEMM time {g_us:.1f} us per step exceeds the {1e3 * ms_step:.1f} us step")
     achieved = g_bytes / (g_us * 1e-6) / 1e9
-    roofline = {"bound": "hbm", "kernel": "gemm_tc_kernel",
-                "launches_per_step": sum(kernels[k]["launches_per_step"] for k in gk),
+    roofline = {"bound": "hbm", "kernel": "gemm_tc_kernel" if timed else "gemm_simt_kernel",
+                "launches_per_step": len(names),
                 "algorithmic_bytes_per_step": g_bytes, "us_per_step": g_us,
+                "us_per_step_after_dependency": g_dep_us,
                 "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                "traffic": gemm_traffic(w), "peak_source": peak_src,
-                "note": "achieved = algorithmic GEMM bytes of a step / summed CUDA-event launch "
-                        "times (events around each launch add ~4 us each); traffic = ncu DRAM "
-                        "bytes per step from profiles/, null if the GEMM sources changed since"}
-    for k in kernels.values():
-        if k["gbs"]:
-            k["frac_of_hbm"] = k["gbs"] / hbm
+                "frac_after_dependency": (g_bytes / (g_dep_us * 1e-6) / 1e9 / hbm) if g_dep_us else None,
+                "between_gemms_us": between,
+                "traffic": gemm_traffic(w), "peak_source": peak_src, "per_launch": per_launch,
+                "note": "achieved = algorithmic GEMM bytes of a step / GEMM time of a step, timed "
+                        f"by {how}; a span can include a wait for the previous kernel when the "
+                        "launch starts early under programmatic dependent launch, so frac is a lower "
+                        "bound; frac_after_dependency divides by the time from each launch's first "
+                        "met dependency to its exit (weights prefetched before that are not "
+                        "counted in the time); between_gemms_us: from a GEMM's exit to the next "
+                        "GEMM's dependency (the kernels between them and the launch latencies); "
+                        "traffic = ncu DRAM bytes per step from profiles/, null if the GEMM sources "
+                        "changed since"}
     # the whole block step against HBM: every kernel's algorithmic bytes over the graph-timed
     # step (no events between launches)
     s_bytes = sum(k["algorithmic_bytes"] * k["launches_per_step"] for k in kernels.values())
-    s_gbs = s_bytes / (ms / K * 1e-3) / 1e9
-    step_roofline = {"bytes_per_step": s_bytes, "ms_per_step": ms / K, "achieved": s_gbs,
+    s_gbs = s_bytes / (ms_step * 1e-3) / 1e9
+    step_roofline = {"bytes_per_step": s_bytes, "ms_per_step": ms_step, "achieved": s_gbs,
                      "peak": hbm, "unit": "GB/s", "frac": s_gbs / hbm,
                      "lower_bound_ms": s_bytes / (hbm * 1e9) * 1e3,
                      "note": "algorithmic bytes of every kernel of a step (weights, context K/V, "
                              "target states, logits) / the CUDA-graph step time"}
 
     # ---------------- end to end through the public calls with host buffers
-    pin_h = hid_host.pin_memory()
+    pin_h = [h.pin_memory() for h in hid_host]
     pin_u = torch.from_numpy(u.view(np.int32)).pin_memory()
     pin_r = torch.from_numpy(r).pin_memory()
     pin_last = torch.from_numpy(last).pin_memory()
@@ -701,15 +850,17 @@ def run_ours(args):
     io_parts(io_b[1])[1].copy_(nxt)
     out_io = torch.zeros((E, nio), dtype=torch.int32).pin_memory()
     # step inputs double-buffered: while step i computes on the current stream, a copy stream
-    # brings step i + 1's target states and target draws from pinned host memory into the other
-    # buffer (events order each buffer's copy after the step that last read it)
-    hid_b = [hid_step, torch.empty_like(hid_step)]
+    # brings step i + 1's target states (from the next of the N_ROT pinned host buffers) and
+    # target draws into the other device buffer (events order each buffer's copy after the step
+    # that last read it)
+    hid_b = [hid_dev[0], hid_dev[1]]
     u_b = [torch.zeros((1,) + u.shape[1:], dtype=torch.int32, device="cuda") for _ in range(2)]
     r_b = [torch.zeros((1,) + r.shape[1:], dtype=torch.int32, device="cuda") for _ in range(2)]
     l_b = [torch.zeros((1,) + last.shape[1:], dtype=torch.int32, device="cuda") for _ in range(2)]
     # each step's draws are a one-row table, so the synthetic target's row counter stays at 0
     zero_ctr = torch.zeros(1, dtype=torch.int32, device="cuda")
-    h2d = pin_h.numel() * pin_h.element_size() + (u_b[0].numel() + r_b[0].numel() + l_b[0].numel()) * 4
+    h2d = pin_h[0].numel() * pin_h[0].element_size() + \
+        (u_b[0].numel() + r_b[0].numel() + l_b[0].numel()) * 4
     d2h = nio * 4
     cps = torch.cuda.Stream()
     main = torch.cuda.current_stream()
@@ -722,7 +873,7 @@ def run_ours(args):
         with torch.cuda.stream(cps):
             cps.wait_event(used[k])
             j = i % n_tab
-            hid_b[k].copy_(pin_h, non_blocking=True)
+            hid_b[k].copy_(pin_h[i % N_ROT], non_blocking=True)
             u_b[k].copy_(pin_u[j:j + 1], non_blocking=True)
             r_b[k].copy_(pin_r[j:j + 1], non_blocking=True)
             l_b[k].copy_(pin_last[j:j + 1], non_blocking=True)
@@ -768,21 +919,24 @@ def run_ours(args):
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
-        "warmup": Wm, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak",
+        "warmup": Wm, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": s.dtype, "data": "synthetic",
-        "config": {"workload": w.name, "d": s.d, "draft_layers": s.n_draft_layers,
-                   "target_layers": s.n_target_layers, "heads": [s.n_q_heads, s.n_kv_heads],
-                   "head_dim": s.head_dim, "ffn": s.ffn, "vocab": s.vocab, "block": s.block,
-                   "batch": w.batch, "ctx": list(w.ctx_lens), "match_p": w.match_p,
+        "config": {**config_of(w),
                    "l2": "not flushed: each step streams the whole draft weight set "
                          f"({sum(v.nbytes for v in W.values()) / 1e9:.2f} GB) > 129 MB L2",
-                   "timing": "CUDA-graph replay of one block step, K replays between events"},
+                   "timing": f"CUDA-graph replays of one block step each ({N_ROT} graphs over "
+                             f"{N_ROT} target-state buffers, in turn), K replays between events"},
         "block_steps_per_s": K / (ms / 1e3),
         "mean_accept_len": mean_tau,
         "accepted_tokens_per_s": world * w.batch * mean_tau * K / (ms / 1e3),
         "roofline": roofline,
         "step_roofline": step_roofline,
         "kernels": kernels,
+        "kernels_note": "CUDA events around every launch of a step, in a separate replay of the "
+                        "step's graph with those events (each duration includes its launch's own "
+                        "latency, which the untraced graph overlaps); traced_ms_per_step is that "
+                        "replay's step time",
+        "traced_ms_per_step": traced_ms,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "ms_per_step": 1e3 * max(e2e_ms / 1e3, wall) / E,
                 "steps": E, "host_ms_per_step": 1e3 * wall / E, "device_ms_per_step": e2e_ms / E,
@@ -805,22 +959,70 @@ def run_ours(args):
         "launches_per_step": launches_per_step,
         "clocks": clk,
     }
-    if not args.no_variants:
-        line["fusion_variants"] = fusion_variants(w, dev_w, fill_chunks, hid_step,
+    if s.dtype == "bf16" and fill_us.get("gemm_kv_ctx"):
+        bf = peaks.get("bf16_tflops")
+        line["fill"]["kv_ctx_frac_of_bf16_peak"] = (line["fill"]["kv_ctx_tflops"] / bf) if bf else None
+    if extras:
+        line["fusion_variants"] = fusion_variants(w, dev_w, fill_chunks, hid_dev[0],
                                                   max(1, int(round(mean_tau))))
-        line["sampled"] = sampled_steps(w, dev_w, fill_chunks, hid_step,
+        line["sampled"] = sampled_steps(w, dev_w, fill_chunks, hid_dev[0],
                                         torch.from_numpy(synth.initial_tokens(w)).cuda())
-    del fill_chunks
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, dt, tau, n_cpu = oracle_steps(w, W, 10 ** 6, budget_s=args.cpu_seconds)
+    del fill_chunks, graphs
+    lib.close()
+    del dev_w, hid_dev
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and cpu_seconds > 0:
+        v, dt, tau, n_cpu = oracle_steps(w, W, 10 ** 6, budget_s=cpu_seconds)
         line["cpu_baseline"] = {
             "value": v, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
             "sample": f"{n_cpu} full block steps of {w.name} (fp64, bf16 storage "
                       f"rounding) after an untimed oracle fill of {list(w.ctx_lens)} positions",
             "seconds": dt}
+    return line
+
+
+SUB_KEYS = ("value", "unit", "ms_per_step", "block_steps_per_s", "mean_accept_len",
+            "accepted_tokens_per_s", "config", "roofline", "step_roofline", "e2e", "fill",
+            "cpu_baseline", "clocks", "launches_per_step", "kernels")
+
+
+def run_ours(args):
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    cpu_s = 0.0 if args.no_cpu_baseline else args.cpu_seconds
+    w = synth.preset(args.workload)
+    if args.draft_layers or args.vocab or args.batch:
+        import dataclasses
+        shp = dataclasses.replace(w.shape, n_draft_layers=args.draft_layers or w.shape.n_draft_layers,
+                                  vocab=args.vocab or w.shape.vocab)
+        lens = (max(w.ctx_lens),) * args.batch if args.batch else w.ctx_lens
+        w = w.with_(shape=shp, ctx_lens=lens,
+                    name=f"{w.name}_D{shp.n_draft_layers}_V{shp.vocab}_b{len(lens)}")
+        args.headline_only = True
+    line = measure(w, args, args.steps, args.warmup, args.e2e_steps,
+                   args.breakdown_steps, cpu_s, not args.no_variants, dist, world, rank, local)
+    # the other drafter shapes, each measured the same way (one GPU only: under torchrun every
+    # rank runs the headline workload as an independent replica)
+    if world == 1 and not args.headline_only:
+        line["configs"] = {}
+        for name in CONFIG_SET:
+            if name == args.workload:
+                continue
+            sub = measure(synth.preset(name), args, args.steps, args.warmup, args.e2e_steps,
+                          args.breakdown_steps, 0.0 if args.no_cpu_baseline else args.sub_cpu_seconds,
+                          False, local=local)
+            line["configs"][name] = {k: sub[k] for k in SUB_KEYS if k in sub}
     if rank == 0:
         print(json.dumps(line), flush=True)
-    lib.close()
     if dist:
         dist.destroy_process_group()
     return 0
@@ -930,7 +1132,7 @@ def run_sweep(args):
             raise RuntimeError(f"device error at sweep point {pt}")
         kern = {}
         if args.breakdown_steps > 0:
-            per = graph_breakdown(lib, cs, step, args.breakdown_steps)
+            per, _ = graph_breakdown(lib, cs, step, args.breakdown_steps)
             kern = {n: round(1e3 * float(np.sum(ts)) / args.breakdown_steps, 1) for n, ts in per.items()}
         e = 2
         wbytes = e * (s.n_draft_layers * (d * (s.d_q + 2 * s.d_kv) + s.d_q * d + 3 * d * s.ffn + 2 * s.d_kv * d)

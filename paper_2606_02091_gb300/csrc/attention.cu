@@ -46,6 +46,16 @@ struct AttnArgs {
     int block_rows;       // rows of one K^d / V^d tensor-map box (min(64, max_batch * B))
     int B, G, hkv, d_q, d_kv, max_ctx, splits, q_tiles;
     float scale_log2;     // log2(e) / sqrt(hd)
+    // bf16 path with the projection's fp32 sums: Q / K^d / V^d are taken from qkv32
+    // ([batch*B][d_q + 2 d_kv]) with the rotary embedding at the block positions (rope != 0)
+    // applied here; the CTA that holds a block tile writes its head's bf16 K^d / V^d rows to kd_w /
+    // vd_w before its TMA reads them
+    const float* qkv32;
+    const float* rope_cos;   // [positions][hd/2]
+    const float* rope_sin;
+    bf16* kd_w;
+    bf16* vd_w;
+    int rope;
 };
 
 __device__ __forceinline__ void key_range(const AttnArgs& a, int b, int s, int& j0, int& j1, int& L) {
@@ -212,7 +222,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     // every CTA of the cluster has started before any pushes into another's shared memory (the
     // matching wait comes after the key loop)
     asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-    pdl_wait();
+    // The context lengths and the cached context keys/values were written before the kernel
+    // that precedes this one (the Q/K^d/V^d projection, which signals its dependents only after
+    // its own dependency wait), so they are complete here; Q, K^d and V^d are read after the
+    // wait below.
     const int L = a.ctx_len[b];
     // the sequence's tiles: ceil(L / 64) context tiles, then the block tile; split s takes a
     // contiguous run of them (the counts differ by at most one)
@@ -247,6 +260,45 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             prod_ok = tile_wait(ebar + 8u * (issued % kNST), (uint32_t)(issued / kNST - 1) & 1u);
         if (prod_ok) issue(issued++);
     };
+    // the first context tile streams in while the projection drains; the block tile waits
+    if (tid == 0)
+        for (; issued < min(kNST - 1, n_ct); ++issued) issue(issued);
+    pdl_wait();
+    if (a.qkv32 && n_tiles > n_ct) {
+        // this CTA holds the block tile: its head's K^d (rotated) and V^d rows, rounded to bf16,
+        // go to kd / vd for the tile's TMA load (identical values from every query tile's CTA)
+        const int nb = a.B * (HD / 16), n32 = a.d_q + 2 * a.d_kv;
+        for (int it = tid; it < 2 * nb; it += blockDim.x) {
+            const bool is_v = it >= nb;
+            const int k = (it % nb) / (HD / 16), j0 = ((it % nb) % (HD / 16)) * 8;
+            const float* src = a.qkv32 + ((size_t)b * a.B + k) * n32 + a.d_q + (is_v ? a.d_kv : 0) + g * HD;
+            float x1[8], x2[8], o1[8], o2[8];
+            load8(src + j0, x1);
+            load8(src + j0 + HD / 2, x2);
+            if (!is_v && a.rope) {
+                float cs[8], sn[8];
+                load8(a.rope_cos + (size_t)(L + k) * (HD / 2) + j0, cs);
+                load8(a.rope_sin + (size_t)(L + k) * (HD / 2) + j0, sn);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    o1[e] = x1[e] * cs[e] - x2[e] * sn[e];
+                    o2[e] = x2[e] * cs[e] + x1[e] * sn[e];
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    o1[e] = x1[e];
+                    o2[e] = x2[e];
+                }
+            }
+            bf16* dst = (is_v ? a.vd_w : a.kd_w) + ((size_t)b * a.B + k) * a.d_kv + g * HD + j0;
+            store8(dst, o1);
+            store8(dst + HD / 2, o2);
+        }
+        // the generic stores above before the tensor-memory-access reads of the block tile
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+        __syncthreads();
+    }
     if (tid == 0)
         for (; issued < min(kNST - 1, n_tiles); ++issued) issue(issued);
 
@@ -259,13 +311,51 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
         const bf16* q = static_cast<const bf16*>(a.q);
         const uint32_t sQ = smem_addr(Qs);
         // query rows of this tile: row r -> block position r / G, head g*G + r % G
-        for (int idx = tid; idx < kQT * PIECES; idx += blockDim.x) {
-            const int r = idx / PIECES, pc = idx % PIECES;
-            const int rr = qt * kQT + r;
-            const bool ok = rr < R;
-            const int kpos = ok ? rr / a.G : 0, hh = ok ? rr % a.G : 0;
-            const bf16* src = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + pc * 8;
-            cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
+        if (a.qkv32) {
+            // from the fp32 sums: the rotary embedding at position L + block position, then bf16
+            const int n32 = a.d_q + 2 * a.d_kv;
+            for (int idx = tid; idx < kQT * (HD / 16); idx += blockDim.x) {
+                const int r = idx / (HD / 16), j0 = (idx % (HD / 16)) * 8;
+                const int rr = qt * kQT + r;
+                float o1[8], o2[8];
+                if (rr < R) {
+                    const int kpos = rr / a.G, hh = rr % a.G;
+                    const float* src = a.qkv32 + ((size_t)b * a.B + kpos) * n32 + (size_t)(g * a.G + hh) * HD;
+                    float x1[8], x2[8];
+                    load8(src + j0, x1);
+                    load8(src + j0 + HD / 2, x2);
+                    if (a.rope) {
+                        float cs[8], sn[8];
+                        load8(a.rope_cos + (size_t)(L + kpos) * (HD / 2) + j0, cs);
+                        load8(a.rope_sin + (size_t)(L + kpos) * (HD / 2) + j0, sn);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            o1[e] = x1[e] * cs[e] - x2[e] * sn[e];
+                            o2[e] = x2[e] * cs[e] + x1[e] * sn[e];
+                        }
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            o1[e] = x1[e];
+                            o2[e] = x2[e];
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) o1[e] = o2[e] = 0.f;
+                }
+                store8(Qs + r * LD + j0, o1);
+                store8(Qs + r * LD + j0 + HD / 2, o2);
+            }
+        } else {
+            for (int idx = tid; idx < kQT * PIECES; idx += blockDim.x) {
+                const int r = idx / PIECES, pc = idx % PIECES;
+                const int rr = qt * kQT + r;
+                const bool ok = rr < R;
+                const int kpos = ok ? rr / a.G : 0, hh = ok ? rr % a.G : 0;
+                const bf16* src = q + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + pc * 8;
+                cp_async16(sQ + (uint32_t)(r * LD + pc * 8) * 2, src, ok);
+            }
         }
         cp_commit();
         // the query tile is complete in shared memory before the loop (the only CTA barrier on
@@ -688,6 +778,14 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
         return g.head_dim == 64 ? run_simt<float, 64>(c, a, s) : run_simt<float, 128>(c, a, s);
     }
     a.err = c->err;
+    if (c->qkv32 && !(g.flags & (DFLARE_FLAG_DETERMINISTIC | DFLARE_FLAG_SIMT_GEMM))) {
+        a.qkv32 = c->qkv32;
+        a.rope_cos = c->rope_cos;
+        a.rope_sin = c->rope_sin;
+        a.kd_w = static_cast<bf16*>(c->kd);
+        a.vd_w = static_cast<bf16*>(c->vd);
+        a.rope = (g.flags & DFLARE_FLAG_NO_BLOCK_ROPE) ? 0 : 1;
+    }
     // tensor maps of every layer's K/V cache and of K^d / V^d, built once per context
     if (c->attn_maps.empty()) {
         std::vector<CUtensorMap> m((size_t)2 * g.n_draft_layers + 2);

@@ -381,6 +381,7 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
     ALLOC(c->q, rows * d_q * esz);
     ALLOC(c->kd, rows * d_kv * esz);
     ALLOC(c->vd, rows * d_kv * esz);
+    if (g.dtype == DFLARE_BF16) ALLOC(c->qkv32, rows * (d_q + 2 * d_kv) * sizeof(float));
     ALLOC(c->attn, rows * d_q * esz);
     ALLOC(c->act, rows * F * esz);
     ALLOC(c->xh, mrows * d * esz);
@@ -407,8 +408,9 @@ dflare_status dflare_create(const dflare_config* cfg, dflare_ctx** out) {
         {c->fused, D * (size_t)g.max_fuse_rows * d * esz}, {c->x, rows * d * 4},
         // every row the attention reads past the valid keys holds a written value or zero
         {c->kcache, kv * esz}, {c->vcache, kv * esz}, {c->kd, rows * d_kv * esz},
-        {c->vd, rows * d_kv * esz}};
+        {c->vd, rows * d_kv * esz}, {c->qkv32, c->qkv32 ? rows * (d_q + 2 * d_kv) * 4 : 0}};
     for (auto& z : zs) {
+        if (!z.p || !z.n) continue;
         e = cudaMemset(z.p, 0, z.n);
         if (e != cudaSuccess) return bail(DFLARE_ECUDA, std::string("cudaMemset: ") + cudaGetErrorString(e));
     }
@@ -545,10 +547,17 @@ dflare_status draft_block_impl(dflare_ctx* c, const int32_t* last_token, int32_t
     }
     if (hidden_out)
         CUDA_TRY(cudaMemcpyAsync(hidden_out, c->x, hid_stride * 4, cudaMemcpyDeviceToDevice, s));
+    // bf16 tensor-core path: the Q/K^d/V^d splits add their fp32 partials into qkv32 with L2
+    // reductions and the attention applies the rotary embedding and rounds as it loads them (no
+    // split-K workspace, tile counter or last-CTA epilogue on the critical path); qkv32 is cleared
+    // by the embedding (first layer) and by each pre-attention RMSNorm. The deterministic mode
+    // keeps the fixed-order reduction.
+    const bool red32 = c->qkv32 && !(g.flags & (DFLARE_FLAG_DETERMINISTIC | DFLARE_FLAG_SIMT_GEMM));
     for (int i = 0; i < g.n_draft_layers; ++i) {
         if (i > 0) {
             Trace t(c, "rmsnorm", s);
-            CUDA_TRY(launch_rmsnorm(c, at(c->w.attn_norm, i * d, esz), rows, false, c->xn, s));
+            CUDA_TRY(launch_rmsnorm(c, at(c->w.attn_norm, i * d, esz), rows, false, c->xn, s,
+                                    red32 ? c->qkv32 : nullptr));
         }
         // Q = X~ W_Q, K^d = X~ W_K^d, V^d = X~ W_V^d with the rotary embedding (Eq. 4)
         GemmDesc q{};
@@ -568,6 +577,11 @@ dflare_status draft_block_impl(dflare_ctx* c, const int32_t* last_token, int32_t
         q.ep.vd = c->vd;
         q.ep.ctx_len = c->ctx_len;
         q.ep.rope = (g.flags & DFLARE_FLAG_NO_BLOCK_ROPE) ? 0 : 1;
+        if (red32) {
+            q.ep.kind = EPI_RED32;
+            q.ep.out = c->qkv32;
+            q.ep.ldo = q.n;
+        }
         dflare_status st = traced_gemm(c, "gemm_qkv", q, s);
         if (st != DFLARE_OK) return st;
         // bidirectional attention over [context ; block] (Sec. 3.2)

@@ -17,8 +17,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
                                                         int m_tok, long long a_group_rows,
                                                         long long b_group_rows, int b_shared,
                                                         int b_kgroup, int n_tiles, EpiParams ep) {
-    pdl_trigger();
     pdl_wait();
+    pdl_trigger();   // after the wait: see gemm_tc_kernel
     __shared__ float sA[2][kTN][kTK + 1];
     __shared__ float sB[kTT][kTK + 1];
     __shared__ __align__(16) float tile[2 * kTT * kTN];

@@ -247,7 +247,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    pdl_trigger();
     unsigned long long* const tst = args.t_stamps;
     if (tst && threadIdx.x == 0) atomicMin(tst, (unsigned long long)globaltimer_ns());
     if (warp == 4 && lane == 0) {
@@ -439,6 +438,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     } else {
         // ---------------- epilogue warps 0-3 (thread t <-> TMEM lane t <-> feature t of a tile)
         pdl_wait();
+        // dependents may start once every CTA has passed its own dependency wait: everything the
+        // kernels before this one wrote is then complete (the attention that follows the Q/K^d/V^d
+        // projection reads the context cache before its own wait)
+        if (threadIdx.x == 0) pdl_trigger();
         const int t = threadIdx.x;
         int acc = 0;
         uint32_t acc_phase = 0;
@@ -447,6 +450,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         uint32_t* const tile_cnt = args.tile_cnt;
         const bool resid = args.ep.kind == EPI_RESID && bn == kChunk;
         const bool resid_red = args.ep.kind == EPI_RESID && args.resid_red;
+        const bool red32 = args.ep.kind == EPI_RED32;
         for (int u = blockIdx.x; u < G.n_units; u += gridDim.x) {
             const Unit x = decode_unit(G, u);
             if (resid_red) {
@@ -475,6 +479,48 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                                              "f"(v[c])
                                              : "memory");
                     }
+                }
+                if (G.n_bufs == 2) {
+                    acc ^= 1;
+                    if (acc == 0) acc_phase ^= 1u;
+                } else {
+                    acc_phase ^= 1u;
+                }
+                continue;
+            }
+            if (red32) {
+                // out += acc with fp32 L2 reductions: each 16-token chunk is turned token-major in
+                // shared memory, then every thread adds 16 consecutive features of one token with
+                // four 16-byte reductions (no workspace, no tile counter, no read back)
+                if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, err)) break;
+                tc_fence_after();
+                const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
+                const int cc = t >> 3, f0 = (t & 7) * 16;
+                const int n0 = x.n_tile * 128 + f0;
+                float* const out32 = reinterpret_cast<float*>(args.ep.out);
+                for (int c0 = 0; c0 < bn; c0 += kChunk) {
+                    float v[kChunk];
+                    tmem_ld16(taddr + (uint32_t)c0, v);
+                    if (c0 + kChunk >= bn) {
+                        tc_fence_before();
+                        mbar_arrive(tempty_bar(acc));
+                    }
+#pragma unroll
+                    for (int c = 0; c < kChunk; ++c) epi[c * 128 + t] = v[c];
+                    epi_bar();
+                    const int tok = x.tok_tile * bn + c0 + cc;
+                    if (tok < args.ep.m_tok && n0 < args.ep.n) {
+                        float* dst = out32 + (size_t)tok * args.ep.ldo + n0;
+                        const float* srow = epi + cc * 128 + f0;
+#pragma unroll
+                        for (int q4 = 0; q4 < 4; ++q4) {
+                            const float4 w4 = *reinterpret_cast<const float4*>(srow + 4 * q4);
+                            asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst + 4 * q4),
+                                         "f"(w4.x), "f"(w4.y), "f"(w4.z), "f"(w4.w)
+                                         : "memory");
+                        }
+                    }
+                    epi_bar();
                 }
                 if (G.n_bufs == 2) {
                     acc ^= 1;

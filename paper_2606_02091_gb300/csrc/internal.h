@@ -21,7 +21,8 @@ enum EpiKind : int {
     EPI_RESID = 2,      // resid[tok][n] += acc                   (fp32 residual stream)
     EPI_QKV = 3,        // Q / K^d / V^d with rotary embedding on Q and K^d at the block positions
     EPI_KV_APPEND = 4,  // context K^t (rotated) / V^t appended to the layer's cache
-    EPI_SWIGLU = 5      // out[tok][n] = silu(gate) * up          (two accumulators)
+    EPI_SWIGLU = 5,     // out[tok][n] = silu(gate) * up          (two accumulators)
+    EPI_RED32 = 6       // out[tok][n] += acc with fp32 L2 reductions (every split adds its part)
 };
 
 struct EpiParams {
@@ -149,6 +150,7 @@ struct dflare_ctx {
     void* q = nullptr;             // [max_batch*B][d_q]
     void* kd = nullptr;            // [max_batch*B][d_kv]
     void* vd = nullptr;
+    float* qkv32 = nullptr;        // [max_batch*B][d_q + 2 d_kv] fp32 sums of the Q/K^d/V^d splits (bf16 path)
     void* attn = nullptr;          // [max_batch*B][d_q]
     void* act = nullptr;           // [max_batch*B][F]
     void* xh = nullptr;            // [max_batch*(B-1)][d]
@@ -240,8 +242,9 @@ cudaError_t launch_fuse_begin(dflare_ctx* c, const int32_t* n_new, int n_max, cu
 cudaError_t launch_fuse_layers(dflare_ctx* c, const void* hidden, int n_max, void* fused_out,
                                cudaStream_t s);
 cudaError_t launch_embed(dflare_ctx* c, const int32_t* last_token, cudaStream_t s);
+// zero32 (optional): the fp32 Q/K^d/V^d sums of the next projection, rows x (d_q + 2 d_kv), cleared
 cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gather_mask_rows,
-                           void* out, cudaStream_t s);
+                           void* out, cudaStream_t s, float* zero32 = nullptr);
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s);
 cudaError_t launch_argmax(dflare_ctx* c, const float* logits, int rows, int32_t* tokens,
                           cudaStream_t s);

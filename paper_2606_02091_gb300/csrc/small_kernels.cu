@@ -13,15 +13,21 @@ namespace {
 // X^0 = [E[x_t]; E[mask] x (B-1)] (Sec. 3.2: the block is the target decode token followed by
 // B-1 mask positions, embedded with the target's shared table, Sec. 3.3), kept in fp32, and the
 // first layer's normalised input RMSNorm(X^0) in the storage type.
+// qkv32 (when given, n32 floats per block row) is cleared here, at the start of every drafted
+// block, so that the first layer's Q/K^d/V^d reductions start from zero even after an aborted call.
 template <class T>
 __global__ void embed_kernel(const T* __restrict__ E, const int32_t* __restrict__ last_token,
                              int mask_id, int V, int B, int d, float* __restrict__ X,
                              T* __restrict__ Xn, const T* __restrict__ gain, float eps,
-                             uint32_t* err) {
+                             uint32_t* err, float* __restrict__ qkv32, int n32) {
     pdl_trigger();
     pdl_wait();
     __shared__ float red[32];
     const int k = blockIdx.x, b = blockIdx.y;
+    if (qkv32) {
+        float4* z = reinterpret_cast<float4*>(qkv32 + ((size_t)b * B + k) * n32);
+        for (int i = threadIdx.x; i < n32 / 4; i += blockDim.x) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     int tok = k == 0 ? last_token[b] : mask_id;
     if (tok < 0 || tok >= V) {
         if (threadIdx.x == 0) atomicOr(err, DFLARE_DEVERR_TOKEN);
@@ -50,14 +56,21 @@ __global__ void embed_kernel(const T* __restrict__ E, const int32_t* __restrict_
 }
 
 // out[r] = gain * X[row(r)] / sqrt(mean(X^2) + eps). With `gather`, output row r reads the mask
-// row k = r % (B-1) + 1 of sequence r / (B-1) (the LM head only needs the mask positions).
+// row k = r % (B-1) + 1 of sequence r / (B-1) (the LM head only needs the mask positions). With
+// zero32, row r of it (n32 floats) is cleared: the fp32 sums the next Q/K^d/V^d projection adds
+// into (the previous layer's attention, which read them, is complete by now).
 template <class T>
 __global__ void rmsnorm_kernel(const float* __restrict__ X, const T* __restrict__ gain,
-                               T* __restrict__ out, int d, int B, int gather, float eps) {
+                               T* __restrict__ out, int d, int B, int gather, float eps,
+                               float* __restrict__ zero32, int n32) {
     pdl_trigger();
     pdl_wait();
     __shared__ float red[32];
     const int r = blockIdx.x;
+    if (zero32) {
+        float4* z = reinterpret_cast<float4*>(zero32 + (size_t)r * n32);
+        for (int i = threadIdx.x; i < n32 / 4; i += blockDim.x) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     const size_t in_row = gather ? (size_t)(r / (B - 1)) * B + (r % (B - 1)) + 1 : (size_t)r;
     const int e0 = threadIdx.x * 8;
     const bool act = e0 < d;
@@ -224,23 +237,26 @@ cudaError_t launch_embed(dflare_ctx* c, const int32_t* last_token, cudaStream_t 
         return launch_kernel(c->pdl, embed_kernel<float>, grid, block, 0, s,
                              (const float*)c->w.embed, last_token, g.mask_token_id, g.vocab, g.block,
                              g.d, c->x, (float*)c->xn, (const float*)c->w.attn_norm, g.rms_eps,
-                             c->err);
+                             c->err, (float*)nullptr, 0);
     return launch_kernel(c->pdl, embed_kernel<bf16>, grid, block, 0, s, (const bf16*)c->w.embed,
                          last_token, g.mask_token_id, g.vocab, g.block, g.d, c->x, (bf16*)c->xn,
-                         (const bf16*)c->w.attn_norm, g.rms_eps, c->err);
+                         (const bf16*)c->w.attn_norm, g.rms_eps, c->err, c->qkv32,
+                         (g.n_q_heads + 2 * g.n_kv_heads) * g.head_dim);
 }
 
 cudaError_t launch_rmsnorm(dflare_ctx* c, const void* gain, int rows, bool gather, void* out,
-                           cudaStream_t s) {
+                           cudaStream_t s, float* zero32) {
     const dflare_config& g = c->cfg;
     if (rows <= 0) return cudaSuccess;
     const dim3 block(((g.d / 8 + 31) / 32) * 32);
+    const int n32 = (g.n_q_heads + 2 * g.n_kv_heads) * g.head_dim;
     if (g.dtype == DFLARE_F32)
         return launch_kernel(c->pdl, rmsnorm_kernel<float>, dim3(rows), block, 0, s, c->x,
                              (const float*)gain, (float*)out, g.d, g.block, gather ? 1 : 0,
-                             g.rms_eps);
+                             g.rms_eps, zero32, n32);
     return launch_kernel(c->pdl, rmsnorm_kernel<bf16>, dim3(rows), block, 0, s, c->x,
-                         (const bf16*)gain, (bf16*)out, g.d, g.block, gather ? 1 : 0, g.rms_eps);
+                         (const bf16*)gain, (bf16*)out, g.d, g.block, gather ? 1 : 0, g.rms_eps,
+                         zero32, n32);
 }
 
 cudaError_t launch_argmax(dflare_ctx* c, const float* logits, int rows, int32_t* tokens,
