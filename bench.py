@@ -55,6 +55,8 @@ def parse():
     p.add_argument("--batch", type=int, default=0,
                    help="override the batch of --workload (every context as long as the longest); "
                         "implies --headline-only")
+    p.add_argument("--ctx", type=int, default=0,
+                   help="override every context length of --workload; implies --headline-only")
     p.add_argument("--sub-cpu-seconds", type=float, default=6.0,
                    help="CPU time budget of the oracle steps of each non-headline workload")
     p.add_argument("--e2e-steps", type=int, default=50)
@@ -256,15 +258,17 @@ def kernels_per_trace(shape):
     return {"attention": 1 if shape.dtype == "bf16" else 2}
 
 
-def algorithmic_bytes(w, name, mean_tau):
-    """Bytes a launch of `name` must move at minimum (weights, activations, caches, outputs)."""
+def algorithmic_bytes(w, name, mean_tau, mean_ctx=None):
+    """Bytes a launch of `name` must move at minimum (weights, activations, caches, outputs).
+    mean_ctx: the sequences' mean context length when the launch ran (default: the workload's
+    initial contexts; the benchmark's contexts grow by tau every step)."""
     s = w.shape
     b, B, d, F, V = w.batch, s.block, s.d, s.ffn, s.vocab
     e = 2 if s.dtype == "bf16" else 4
     dq, dkv = s.d_q, s.d_kv
     M = b * B
     Mh = b * (B - 1)
-    L = float(np.mean(w.ctx_lens))
+    L = float(np.mean(w.ctx_lens)) if mean_ctx is None else float(mean_ctx)
     if name == "gemm_lm_head":
         return V * d * e + Mh * d * e + Mh * V * 4
     if name == "gemm_gate_up":
@@ -496,9 +500,9 @@ def graph_breakdown(lib, cs, step, nb, only=None):
 
 
 def gemm_timeline(lib, cs, step, nb, slots=256):
-    """Device-side times of every projection-GEMM launch of one step inside a CUDA graph of the
-    step with nothing added between its launches (dflare_set_timing: %globaltimer at the first
-    CTA's entry, at the first CTA's activation dependency, at the last CTA's exit), replayed nb
+    """Device-side times of every projection-GEMM and attention launch of one step inside a CUDA
+    graph of the step with nothing added between its launches (dflare_set_timing: %globaltimer at
+    the first CTA's entry, at the first CTA's met dependency, at the last CTA's exit), replayed nb
     times. Returns (names, [[(entry, ready, exit) ns per launch] per replay])."""
     import torch
     import paper_2606_02091_gb300 as P
@@ -507,7 +511,7 @@ def gemm_timeline(lib, cs, step, nb, slots=256):
     @P._lib.TRACE_FN
     def name_cb(user, name, phase, stream):
         n = name.decode()
-        if phase == 0 and n.startswith("gemm_"):
+        if phase == 0 and (n.startswith("gemm_") or n == "attention"):
             names.append(n)
 
     L_ = P.load()
@@ -743,12 +747,13 @@ def measure(w, args, steps, warmup, e2e_steps, nb, cpu_seconds, extras, dist=Non
     # ---------------- per-kernel durations (CUDA events around every launch, graph replays)
     hbm, peak_src, peaks = measured_peaks()
     step0 = step_on(hid_dev[0])
+    ctx_now = float(np.mean(lib.ctx_lens()))   # the contexts the timed steps and breakdowns see
     per, traced_ms = graph_breakdown(lib, cs, step0, nb)
     kernels = {}
     for name, ts in per.items():
         launches = len(ts) / nb
         avg_us = 1e3 * float(np.mean(ts))
-        ab = algorithmic_bytes(w, name, mean_tau)
+        ab = algorithmic_bytes(w, name, mean_tau, ctx_now)
         kernels[name] = {"launches_per_step": launches, "avg_us": avg_us,
                          "us_per_step": avg_us * launches,
                          "algorithmic_bytes": ab,
@@ -765,22 +770,33 @@ def measure(w, args, steps, warmup, e2e_steps, nb, cpu_seconds, extras, dist=Non
     # dependent launch), achieved = the step's algorithmic GEMM bytes over that time
     names, runs = gemm_timeline(lib, cs, step0, nb) if s.dtype == "bf16" else ([], [])
     timed = [run for run in runs if run and all(x[2] > 0 and x[0] < 2 ** 63 for x in run)]
+    attn_tl = None
     if timed:
+        all_names = names
+        gi = [i for i, k in enumerate(all_names) if k.startswith("gemm_")]
+        names = [all_names[i] for i in gi]
         g_bytes = sum(algorithmic_bytes(w, k, mean_tau) for k in names)
-        g_us = float(np.mean([union_ns([(x[0], x[2]) for x in run]) for run in timed])) / 1e3
-        g_dep_us = float(np.mean([sum(x[2] - min(max(x[1], x[0]), x[2]) for x in run) for run in timed])) / 1e3
+        g_us = float(np.mean([union_ns([(run[i][0], run[i][2]) for i in gi]) for run in timed])) / 1e3
+        g_dep_us = float(np.mean([sum(run[i][2] - min(max(run[i][1], run[i][0]), run[i][2]) for i in gi)
+                                  for run in timed])) / 1e3
         span = {}
-        for run in timed:
-            for lname, st3 in zip(names, run):
-                span.setdefault(lname, []).append((st3[2] - st3[0]) / 1e3)
         dep = {}
         gaps = {}
         for run in timed:
-            for li, (lname, st3) in enumerate(zip(names, run)):
+            for li, (lname, st3) in enumerate(zip(all_names, run)):
+                span.setdefault(lname, []).append((st3[2] - st3[0]) / 1e3)
                 dep.setdefault(lname, []).append((st3[2] - max(st3[1], st3[0])) / 1e3)
-                if li + 1 < len(run):   # from this launch's exit to the next GEMM's dependency
+                if li + 1 < len(run):   # from this launch's exit to the next timed launch's dependency
                     nx3 = run[li + 1]
-                    gaps.setdefault(f"{lname} -> {names[li + 1]}", []).append((max(nx3[1], nx3[0]) - st3[2]) / 1e3)
+                    gaps.setdefault(f"{lname} -> {all_names[li + 1]}", []).append((max(nx3[1], nx3[0]) - st3[2]) / 1e3)
+        if "attention" in dep:
+            ab = algorithmic_bytes(w, "attention", mean_tau, ctx_now)
+            attn_tl = {"avg_after_dependency_us": float(np.mean(dep["attention"])),
+                       "avg_span_us": float(np.mean(span["attention"])),
+                       "algorithmic_bytes": ab,
+                       "frac_of_hbm_after_dependency": ab / (float(np.mean(dep["attention"])) * 1e-6) / 1e9 / hbm,
+                       "note": "attention launches timed on the device like the GEMMs (dflare_set_timing)"}
+        span = {k: v for k, v in span.items() if k.startswith("gemm_")}
         per_launch = {k: {"launches_per_step": names.count(k),
                           "avg_span_us": float(np.mean(v)),
                           "avg_after_dependency_us": float(np.mean(dep[k])),
@@ -930,6 +946,7 @@ def measure(w, args, steps, warmup, e2e_steps, nb, cpu_seconds, extras, dist=Non
         "mean_accept_len": mean_tau,
         "accepted_tokens_per_s": world * w.batch * mean_tau * K / (ms / 1e3),
         "roofline": roofline,
+        "attention_timing": attn_tl,
         "step_roofline": step_roofline,
         "kernels": kernels,
         "kernels_note": "CUDA events around every launch of a step, in a separate replay of the "
@@ -983,7 +1000,7 @@ def measure(w, args, steps, warmup, e2e_steps, nb, cpu_seconds, extras, dist=Non
 
 
 SUB_KEYS = ("value", "unit", "ms_per_step", "block_steps_per_s", "mean_accept_len",
-            "accepted_tokens_per_s", "config", "roofline", "step_roofline", "e2e", "fill",
+            "accepted_tokens_per_s", "config", "roofline", "attention_timing", "step_roofline", "e2e", "fill",
             "cpu_baseline", "clocks", "launches_per_step", "kernels")
 
 
@@ -1000,13 +1017,15 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     cpu_s = 0.0 if args.no_cpu_baseline else args.cpu_seconds
     w = synth.preset(args.workload)
-    if args.draft_layers or args.vocab or args.batch:
+    if args.draft_layers or args.vocab or args.batch or args.ctx:
         import dataclasses
         shp = dataclasses.replace(w.shape, n_draft_layers=args.draft_layers or w.shape.n_draft_layers,
                                   vocab=args.vocab or w.shape.vocab)
         lens = (max(w.ctx_lens),) * args.batch if args.batch else w.ctx_lens
+        if args.ctx:
+            lens = (args.ctx,) * len(lens)
         w = w.with_(shape=shp, ctx_lens=lens,
-                    name=f"{w.name}_D{shp.n_draft_layers}_V{shp.vocab}_b{len(lens)}")
+                    name=f"{w.name}_D{shp.n_draft_layers}_V{shp.vocab}_b{len(lens)}_L{max(lens)}")
         args.headline_only = True
     line = measure(w, args, args.steps, args.warmup, args.e2e_steps,
                    args.breakdown_steps, cpu_s, not args.no_variants, dist, world, rank, local)

@@ -301,11 +301,11 @@ typedef void (*dflare_trace_fn)(void* user, const char* name, int phase, void* s
 dflare_status dflare_set_trace(dflare_ctx* ctx, dflare_trace_fn fn, void* user);
 
 /* Optional device-side timing of the projection GEMM launches (the tcgen05 kernel behind every
- * "gemm_*" trace name). stamps_dev: caller-owned device array of 3 * slots uint64, laid out as
- * [0, slots) first-CTA entry times, [slots, 2 slots) times at which the first CTA's activation
- * dependency on the previous kernel was met, [2 slots, 3 slots) last-CTA exit times, all in
- * %globaltimer nanoseconds. After this call, GEMM launch number k (counted from this call, k <
- * slots) folds its CTAs' times into slot k with atomicMin (entry, dependency) and atomicMax
+ * "gemm_*" trace name) and of the bf16 attention launches ("attention"). stamps_dev: caller-owned device array of 3 * slots uint64, laid out as
+ * [0, slots) first-CTA entry times, [slots, 2 slots) times at which the first CTA's dependency
+ * on the previous kernel was met, [2 slots, 3 slots) last-CTA exit times, all in %globaltimer
+ * nanoseconds. After this call, timed launch number k (GEMM and attention launches in issue
+ * order, counted from this call, k < slots) folds its CTAs' times into slot k with atomicMin (entry, dependency) and atomicMax
  * (exit); later launches are not timed. The caller sets the first two ranges to all-ones and the
  * third to zero before the launches it reads, and may capture the launches into a CUDA graph
  * (the slot numbers are fixed at capture). Adds two global atomics per CTA while enabled.

@@ -56,6 +56,8 @@ struct AttnArgs {
     bf16* kd_w;
     bf16* vd_w;
     int rope;
+    unsigned long long* t_stamps;   // launch timing (dflare_set_timing): entry, dependency, exit
+    int t_slots;
 };
 
 __device__ __forceinline__ void key_range(const AttnArgs& a, int b, int s, int& j0, int& j1, int& L) {
@@ -178,6 +180,7 @@ template <int HD, int S>
 __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ AttnMaps maps,
                                                        const AttnArgs a, bf16* __restrict__ out) {
     pdl_trigger();
+    if (a.t_stamps && threadIdx.x == 0) atomicMin(a.t_stamps, (unsigned long long)globaltimer_ns());
     constexpr int LD = HD + 8;                 // padded Q row (elements)
     constexpr int PIECES = HD / 8;             // 16-byte pieces per row
     constexpr uint32_t TB = HD * 128;          // bytes of one 64-key K (or V) tile
@@ -264,6 +267,7 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     if (tid == 0)
         for (; issued < min(kNST - 1, n_ct); ++issued) issue(issued);
     pdl_wait();
+    if (a.t_stamps && tid == 0) atomicMin(a.t_stamps + a.t_slots, (unsigned long long)globaltimer_ns());
     if (a.qkv32 && n_tiles > n_ct) {
         // this CTA holds the block tile: its head's K^d (rotated) and V^d rows, rounded to bf16,
         // go to kd / vd for the tile's TMA load (identical values from every query tile's CTA)
@@ -534,6 +538,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
             *reinterpret_cast<__nv_bfloat162*>(orow + q) = __floats2bfloat162_rn(v0 * inv, v1 * inv);
         }
     }
+    if (a.t_stamps) {
+        __syncthreads();
+        if (tid == 0) atomicMax(a.t_stamps + 2 * a.t_slots, (unsigned long long)globaltimer_ns());
+    }
 }
 
 // ------------------------------------------------------------------ CUDA-core path
@@ -724,33 +732,59 @@ int attention_splits(const dflare_config& g, int batch, int num_sms, int len_ub)
 }
 
 // Tensor-core path: the splits of one (sequence, head, query tile) are one cluster of 1, 2, 4, 8
-// or 16 CTAs, at most one per 64-key tile: the most that still run as one wave at two CTAs per
-// SM, unless that leaves a CTA more than 12 tiles; then as many as give about two CTAs per SM in
-// all. Measured: with a few tiles per CTA the fixed cost of a CTA (launch, first tile, partial
+// or 16 CTAs, at most one per 64-key tile: the most that still run as one wave at the CTAs per SM
+// the kernel fits (per_sm: two at head_dim 128, four at head_dim 64), unless that leaves a CTA
+// more than 12 tiles; then as many as give about per_sm CTAs per SM in all. Measured: with a few tiles per CTA the fixed cost of a CTA (launch, first tile, partial
 // push, cluster barrier, merge: ~6 us) dominates and one wave wins (Qwen3-8B-shaped batch 4,
 // 32 (sequence, head) pairs at L <= 4096: 8 splits, 1.256 ms per step, against 16 splits in two
 // waves, 1.327 ms); with long runs per CTA two waves of shorter CTAs overlap the next kernel
 // better (GPT-OSS-shaped batch 2, L 8192: 16 splits 1.046 ms, 8 splits 1.048 ms).
 int attention_cluster_splits(const dflare_config& g, int batch, int num_sms, int len_ub,
-                             int max_cluster) {
+                             int max_cluster, int per_sm) {
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + kQT - 1) / kQT;
     const int base = batch * g.n_kv_heads * q_tiles;
     const int tiles = (len_ub + g.block + kKT - 1) / kKT;
+    const int slots = per_sm * num_sms;
     int sp = 1;
-    while (sp < max_cluster && 2 * sp <= tiles && base * 2 * sp <= 2 * num_sms) sp *= 2;
+    while (sp < max_cluster && 2 * sp <= tiles && base * 2 * sp <= slots) sp *= 2;
     if ((tiles + sp - 1) / sp > 12) {
-        const int want = (2 * num_sms + base - 1) / base;
+        const int want = (slots + base - 1) / base;
         while (sp < max_cluster && sp < want && 2 * sp <= tiles) sp *= 2;
     }
     return sp;
+}
+
+// CTAs of the tensor-core attention that fit on one SM (registers and shared memory; queried once
+// per device): two at head_dim 128, four at head_dim 64, at most four.
+template <int HD>
+int attention_ctas_per_sm() {
+    static std::atomic<int> cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 2;
+    }
+    std::atomic<int>& slot = cache[dev & 63];
+    if (const int known = slot.load(std::memory_order_acquire)) return known;
+    int n = 0;
+    if (cudaFuncSetAttribute(attn_mma_kernel<HD, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)mma_smem_bytes<HD>()) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attn_mma_kernel<HD, 16>, 128,
+                                                      mma_smem_bytes<HD>()) != cudaSuccess || n < 1)
+        n = 2;
+    cudaGetLastError();
+    n = std::min(n, 4);
+    slot.store(n, std::memory_order_release);
+    return n;
 }
 
 int attention_launch_splits(const dflare_ctx* c) {
     const dflare_config& g = c->cfg;
     if (g.dtype == DFLARE_F32) return attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
     const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
-    return attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc);
+    const int per_sm = g.head_dim == 64 ? attention_ctas_per_sm<64>() : attention_ctas_per_sm<128>();
+    return attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc, per_sm);
 }
 
 cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
@@ -814,7 +848,12 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
     maps.vd = c->attn_maps[2 * g.n_draft_layers + 1];
     a.block_rows = std::min(kKT, g.max_batch * g.block);
     const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
-    a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc);
+    const int per_sm = g.head_dim == 64 ? attention_ctas_per_sm<64>() : attention_ctas_per_sm<128>();
+    a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc, per_sm);
+    if (c->t_stamps && c->t_next < c->t_slots) {
+        a.t_stamps = c->t_stamps + c->t_next++;
+        a.t_slots = c->t_slots;
+    }
     return g.head_dim == 64 ? run_mma<64>(c, maps, a, s) : run_mma<128>(c, maps, a, s);
 }
 

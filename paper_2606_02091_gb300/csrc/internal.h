@@ -176,7 +176,7 @@ struct dflare_ctx {
     CallGraph draft_graph, fuse_graph;   // graphs of repeated dflare_draft_block / _fuse_context calls
     dflare_trace_fn trace_fn = nullptr;
     void* trace_user = nullptr;
-    unsigned long long* t_stamps = nullptr;   // GEMM launch timing (dflare_set_timing)
+    unsigned long long* t_stamps = nullptr;   // GEMM and attention launch timing (dflare_set_timing)
     int t_slots = 0;
     int t_next = 0;
     std::string msg;

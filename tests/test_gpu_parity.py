@@ -346,9 +346,10 @@ def test_repeated_calls_replay_as_graphs():
 
 
 def test_gemm_timing_stamps_are_ordered():
-    """dflare_set_timing on a drafted block: each of the 4 D + 1 projection launches (Q/K^d/V^d,
-    O, gate/up, down per layer, then the LM head) records entry <= dependency met <= exit, each
-    launch ends after the one before it, and the slots past the last launch stay untouched."""
+    """dflare_set_timing on a drafted block: each of the 5 D + 1 timed launches (Q/K^d/V^d,
+    attention, O, gate/up, down per layer, then the LM head) records entry <= dependency met <=
+    exit, each launch ends after the one before it, and the slots past the last launch stay
+    untouched."""
     import torch
     w = SMALL_HD128
     g = GpuSide(w)
@@ -362,7 +363,7 @@ def test_gemm_timing_stamps_are_ordered():
     g.lib.set_timing()
     torch.cuda.synchronize()
     a = st.cpu().numpy().view(np.uint64)
-    n = 4 * w.shape.n_draft_layers + 1
+    n = 5 * w.shape.n_draft_layers + 1
     entry, dep, done = a[:slots], a[slots:2 * slots], a[2 * slots:]
     for k in range(n):
         assert 0 < entry[k] <= dep[k] <= done[k], k
