@@ -60,6 +60,7 @@ struct TcArgs {
     int b_kg;                  // > 0: activation group z holds contraction indices [z b_kg, (z+1) b_kg)
     int b_gsel;                // 1: activation group = weight group; 0: one activation group for all
     int resid_red;             // EPI_RESID: each split adds its partial to resid with L2 reductions
+    int resid_vec;             // ... as 16-byte reductions of token-major rows (aligned residual)
     unsigned long long* t_stamps;   // launch timing: entry, dependency met, exit (nullptr: off)
     int t_slots;
 };
@@ -449,8 +450,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         float* const ws = args.ws;
         uint32_t* const tile_cnt = args.tile_cnt;
         const bool resid = args.ep.kind == EPI_RESID && bn == kChunk;
-        const bool resid_red = args.ep.kind == EPI_RESID && args.resid_red;
-        const bool red32 = args.ep.kind == EPI_RED32;
+        const bool resid_red = args.ep.kind == EPI_RESID && args.resid_red && !args.resid_vec;
+        const bool red32 = args.ep.kind == EPI_RED32 || (args.ep.kind == EPI_RESID && args.resid_red && args.resid_vec);
+        float* const red_out = args.ep.kind == EPI_RED32 ? reinterpret_cast<float*>(args.ep.out) : args.ep.resid;
+        const int red_ld = args.ep.kind == EPI_RED32 ? args.ep.ldo : args.ep.ld_resid;
         for (int u = blockIdx.x; u < G.n_units; u += gridDim.x) {
             const Unit x = decode_unit(G, u);
             if (resid_red) {
@@ -489,15 +492,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 continue;
             }
             if (red32) {
-                // out += acc with fp32 L2 reductions: each 16-token chunk is turned token-major in
-                // shared memory, then every thread adds 16 consecutive features of one token with
-                // four 16-byte reductions (no workspace, no tile counter, no read back)
+                // out += acc with fp32 L2 reductions (EPI_RED32, and the residual projections when
+                // the residual rows are 16-byte aligned): each 16-token chunk is turned token-major
+                // in shared memory, then every thread adds 16 consecutive features of one token
+                // with four 16-byte reductions (no workspace, no tile counter, no read back; the
+                // order of the additions, and so the last bit of a sum, can vary between runs)
                 if (!bar_wait(tfull_bar(acc), acc_phase, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(acc * acc_cols);
                 const int cc = t >> 3, f0 = (t & 7) * 16;
                 const int n0 = x.n_tile * 128 + f0;
-                float* const out32 = reinterpret_cast<float*>(args.ep.out);
+                float* const out32 = red_out;
                 for (int c0 = 0; c0 < bn; c0 += kChunk) {
                     float v[kChunk];
                     tmem_ld16(taddr + (uint32_t)c0, v);
@@ -510,7 +515,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     epi_bar();
                     const int tok = x.tok_tile * bn + c0 + cc;
                     if (tok < args.ep.m_tok && n0 < args.ep.n) {
-                        float* dst = out32 + (size_t)tok * args.ep.ldo + n0;
+                        float* dst = out32 + (size_t)tok * red_ld + n0;
                         const float* srow = epi + cc * 128 + f0;
 #pragma unroll
                         for (int q4 = 0; q4 < 4; ++q4) {
@@ -754,6 +759,8 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     const long long a_gr = g.a_group_rows > 0 ? g.a_group_rows : g.n;
     a.b_kg = g.b_kgroup;
     a.resid_red = (c->cfg.flags & DFLARE_FLAG_DETERMINISTIC) ? 0 : 1;
+    a.resid_vec = g.ep.kind == EPI_RESID && g.ep.n % 16 == 0 && g.ep.ld_resid % 4 == 0 &&
+                  (reinterpret_cast<uintptr_t>(g.ep.resid) & 15u) == 0;
     a.b_gsel = g.b_shared ? 0 : 1;
     const int b_k = g.b_kgroup > 0 ? g.b_kgroup : g.k;
     const int b_groups = g.b_kgroup > 0 ? g.k / g.b_kgroup : (g.b_shared ? 1 : g.groups);

@@ -64,6 +64,10 @@ __global__ void rmsnorm_kernel(const float* __restrict__ X, const T* __restrict_
                                T* __restrict__ out, int d, int B, int gather, float eps,
                                float* __restrict__ zero32, int n32) {
     pdl_trigger();
+    const int e0 = threadIdx.x * 8;
+    const bool act = e0 < d;
+    float g[8];
+    if (act) load8(gain + e0, g);   // a weight: read before the dependency wait
     pdl_wait();
     __shared__ float red[32];
     const int r = blockIdx.x;
@@ -72,8 +76,6 @@ __global__ void rmsnorm_kernel(const float* __restrict__ X, const T* __restrict_
         for (int i = threadIdx.x; i < n32 / 4; i += blockDim.x) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
     const size_t in_row = gather ? (size_t)(r / (B - 1)) * B + (r % (B - 1)) + 1 : (size_t)r;
-    const int e0 = threadIdx.x * 8;
-    const bool act = e0 < d;
     float v[8];
     float ss = 0.f;
     if (act) {
@@ -84,8 +86,7 @@ __global__ void rmsnorm_kernel(const float* __restrict__ X, const T* __restrict_
     ss = block_sum(ss, red);
     if (act) {
         const float inv = inv_rms(ss, d, eps);
-        float g[8], o[8];
-        load8(gain + e0, g);
+        float o[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) o[e] = g[e] * (v[e] * inv);
         store8(out + (size_t)r * d + e0, o);
