@@ -67,6 +67,8 @@ def parse():
     p.add_argument("--fill-chunk", type=int, default=2048)
     p.add_argument("--serial-launch", action="store_true",
                    help="no programmatic dependent launch between kernels (A/B measurement)")
+    p.add_argument("--mma-sync-attention", action="store_true",
+                   help="the mma.sync attention kernel instead of the tcgen05 one (A/B measurement)")
     p.add_argument("--sweep", action="store_true",
                    help="throughput sweep around the Qwen3-8B-shaped drafter (one JSON line per point)")
     p.add_argument("--sweep-points", default="",
@@ -605,7 +607,8 @@ def measure(w, args, steps, warmup, e2e_steps, nb, cpu_seconds, extras, dist=Non
     max_ctx = max(w.ctx_lens) + s.block * n_steps_total
     lib = DFlare.from_shape(s, max_batch=w.batch, max_ctx=max_ctx,
                             max_fuse_rows=w.batch * max(chunk, s.block),
-                            flags=P.FLAG_SERIAL_LAUNCH if args.serial_launch else 0)
+                            flags=(P.FLAG_SERIAL_LAUNCH if args.serial_launch else 0) |
+                            (P.FLAG_MMA_SYNC_ATTENTION if args.mma_sync_attention else 0))
     lib.set_weights(dev_w)
     lib.reset(w.batch)
     # context fill in chunks (the target's prompt states): once untimed, then again from an empty

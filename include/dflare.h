@@ -97,6 +97,10 @@ typedef enum { DFLARE_BF16 = 0, DFLARE_F32 = 1 } dflare_dtype;
                                            the order of those additions, and so the last bit of
                                            the residual, free to vary between runs (the
                                            verification decides every emitted token either way) */
+#define DFLARE_FLAG_MMA_SYNC_ATTENTION 0x100u /* bf16 only: run the attention on the mma.sync
+                                           (warp-level) tensor-core kernel, 64 query rows per CTA
+                                           with P in registers, instead of the tcgen05 kernel
+                                           (a cross-check and a measurement baseline) */
 
 /* Device error word bits (dflare_device_error) */
 #define DFLARE_DEVERR_TOKEN     0x1u    /* a token id outside [0, vocab) was read (clamped to 0) */

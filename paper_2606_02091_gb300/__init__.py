@@ -13,6 +13,7 @@ from . import _lib
 from ._lib import (  # noqa: F401
     DFlareError, DFLARE_BF16, DFLARE_F32, FLAG_NO_BLOCK_ROPE, FLAG_RAW_FUSION, FLAG_SIMT_GEMM,
     FLAG_SERIAL_LAUNCH, FLAG_SHARED_KV, FLAG_FUSION_FC, FLAG_DFLASH_FC, FLAG_DETERMINISTIC,
+    FLAG_MMA_SYNC_ATTENTION,
     DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT, EXPORTS, WEIGHT_FIELDS, NOALLOC_MAX_ROWS, load,
 )
 

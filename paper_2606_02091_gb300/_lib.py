@@ -24,6 +24,7 @@ FLAG_SHARED_KV = 0x10
 FLAG_FUSION_FC = 0x20
 FLAG_DFLASH_FC = 0x40
 FLAG_DETERMINISTIC = 0x80
+FLAG_MMA_SYNC_ATTENTION = 0x100
 DEVERR_TOKEN, DEVERR_CAPACITY, DEVERR_TIMEOUT = 0x1, 0x2, 0x4
 
 STATUS_NAMES = {0: "DFLARE_OK", 1: "DFLARE_EINVAL", 2: "DFLARE_ECAPACITY", 3: "DFLARE_ECUDA",

@@ -141,18 +141,27 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) {
 __device__ __forceinline__ uint32_t swz(int r, int c8) {
     return (uint32_t)((c8 >> 3) * 8192 + r * 128 + (((c8 & 7) ^ (r & 7)) << 4));
 }
+__device__ __forceinline__ bool try_wait_parity(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait. The global timer is read only once the phase has not completed within the first
+// 64 polls: measured, a timer read at the start of every wait put a few hundred nanoseconds into
+// each hand-off of the tcgen05 attention's pipeline.
 __device__ __forceinline__ bool tile_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok = 0;
+    for (int i = 0; i < 64; ++i)
+        if (try_wait_parity(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
-        asm volatile(
-            "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-            "selp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(ok)
-            : "r"(bar), "r"(parity)
-            : "memory");
-        if (ok) return true;
+        for (int i = 0; i < 64; ++i)
+            if (try_wait_parity(bar, parity)) return true;
         if (globaltimer_ns() - t0 > kWaitNs) return false;
     }
 }
@@ -544,6 +553,627 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
     }
 }
 
+// ------------------------------------------------------------------ bf16, tcgen05 (Blackwell)
+//
+// The same split-KV cluster attention on the fifth-generation tensor cores. One CTA per (key
+// split, KV head, 128-row query tile, sequence); the 128 query rows are the UMMA M (the B x G
+// rows of a KV head: 64 for the Qwen3 shapes, the rest zero; 128 for GPT-OSS, whose two 64-row
+// halves then read every key tile once instead of twice). Per 64-key tile t:
+//   S_t = Q K_t^T   M 128 x N 64 x K head_dim into TMEM; Q and K K-major in 128-byte-swizzled
+//                   shared memory;
+//   softmax         thread r of a softmax warpgroup = query row r = TMEM lane r: P_t = 2^(s - m)
+//                   rounded to bf16 into a K-major swizzled shared tile, the row sum l taken from
+//                   the fp32 P;
+//   O += P_t V_t    M 128 x N head_dim x K 64; V read MN-major as the TMA wrote it; O stays in
+//                   TMEM for the whole key range.
+// Two softmax warpgroups take alternate tiles, each with its own S, P and O buffers and its own
+// running (m, l), so each SM sub-partition always has a second softmax warp to switch to; their
+// two partial results are combined per row at the end. Within a warpgroup the maximum m that a
+// row's P and O are taken against is raised only when a tile's maximum exceeds it by more than
+// 2^8; then the row's O (P V of the group's previous tile has completed by then) and its l are
+// scaled by 2^(m_old - m_new) before the tile's P is written. Otherwise P <= 2^8, which bf16 and
+// the fp32 accumulators carry with the same relative precision, and O / l does not depend on
+// the choice of m.
+// One warp streams the K/V tiles by TMA into a ring of stages. Two threads in two more warps issue
+// the MMAs: one S_t as soon as tile t has landed and S_{t-2} has been read out of TMEM (so S runs
+// two tiles ahead of the softmax), the other P_t V_t as soon as P_t is written. Measured: every
+// M 128 MMA with N <= 128 occupies the tensor pipe for about 71 cycles, a commit-to-wait round
+// trip of four MMAs takes about 740 cycles, and one thread issuing both kinds, on a sub-partition
+// shared with two softmax warps, took 0.3-0.45 us per hand-off; the issuing warps sit on the
+// sub-partitions that the 64-row (Qwen3-shaped) tiles leave free of softmax work.
+// Every hand-off is an mbarrier with a bounded wait; the splits merge through the cluster as in
+// the mma.sync kernel.
+constexpr int kTQ = 128;            // query rows per CTA (UMMA M)
+constexpr int kTThreads = 384;      // warps 0-3, 4-7: softmax groups; 8: TMA; 9: TMEM; 10, 11: MMA
+constexpr float kRescale = 8.0f;    // growth (log2) of a row maximum that triggers a rescale
+
+template <int HD>
+struct TcAttnLayout {
+    static constexpr int NS = HD == 128 ? 4 : 8;               // K/V stages
+    static constexpr uint32_t TB = HD * 128;                    // one 64-key K or V tile
+    static constexpr uint32_t Q = NS * 2 * TB;                  // Q [HD/64][128 rows][128 B]
+    static constexpr uint32_t P = Q + (uint32_t)kTQ * HD * 2;   // P [group][128 rows][64 keys] bf16
+    static constexpr uint32_t RO = P + 2u * kTQ * 128;          // pushed partials O / l, fp16
+    static constexpr uint32_t RML = RO + (uint32_t)kTQ * HD * 2;   // pushed (m, l)
+    static constexpr uint32_t BARS = RML + (uint32_t)kTQ * 8;   // mbarriers, then two words
+    static constexpr int NBARS = 2 * NS + 10;
+    static constexpr uint32_t BYTES = BARS + NBARS * 8 + 16;
+    static constexpr uint32_t TMEM_COLS = 512;                  // S_A, S_B (64 each), O_A, O_B
+    static_assert(1024 + BYTES <= 232448, "tcgen05 attention exceeds 227 KB of shared memory");
+};
+template <int HD>
+size_t tc_attn_smem_bytes() { return 1024 + TcAttnLayout<HD>::BYTES; }
+
+__device__ __forceinline__ void ta_mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void ta_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void ta_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+// Bounded wait for the phase of `bar` with parity `parity`: false after kWaitNs (which sets the
+// CTA's abort flag and the device error) or once another thread of the CTA has aborted. The timer
+// is read only after 64 unsuccessful polls (as in tile_wait).
+__device__ __noinline__ bool ta_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          uint32_t* err) {
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        for (int i = 0; i < 64; ++i)
+            if (try_wait_parity(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (globaltimer_ns() - t0 > kWaitNs) {
+            *abort_flag = 1;
+            atomicOr(err, DFLARE_DEVERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+__device__ __forceinline__ bool ta_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                        uint32_t* err) {
+    for (int i = 0; i < 64; ++i)
+        if (try_wait_parity(bar, parity)) return true;
+    return ta_wait_slow(bar, parity, abort_flag, err);
+}
+__device__ __forceinline__ void ta_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void ta_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Shared-memory matrix descriptors (128-byte swizzle, version 1). K-major: 128-byte rows, 8-row
+// groups 1024 bytes apart. MN-major (V: the head dims contiguous, the keys the contraction):
+// 64-element swizzle atoms along N 8192 bytes apart, 8-key groups 1024 bytes apart.
+__device__ __forceinline__ uint64_t ta_desc_k(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+__device__ __forceinline__ uint64_t ta_desc_mn(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(8192 >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+__device__ __forceinline__ void ta_mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void ta_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void ta_ld32(uint32_t taddr, float* v) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void ta_st32(uint32_t taddr, const float* v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+        "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]),
+        "f"(v[8]), "f"(v[9]), "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]),
+        "f"(v[16]), "f"(v[17]), "f"(v[18]), "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]),
+        "f"(v[24]), "f"(v[25]), "f"(v[26]), "f"(v[27]), "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+        : "memory");
+}
+// rotate-half rotary embedding of 8 + 8 head dims (j0 .. j0+7 and j0 + hd/2 ..) at one position
+__device__ __forceinline__ void rope8(const float* x1, const float* x2, const float* cs, const float* sn,
+                                      float* o1, float* o2) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        o1[e] = x1[e] * cs[e] - x2[e] * sn[e];
+        o2[e] = x2[e] * cs[e] + x1[e] * sn[e];
+    }
+}
+
+template <int HD, int S>
+__global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_constant__ AttnMaps maps,
+                                                              const AttnArgs a, bf16* __restrict__ out) {
+    using LY = TcAttnLayout<HD>;
+    constexpr int NS = LY::NS;
+    constexpr uint32_t TB = LY::TB;
+    constexpr int RP = kTQ / S;                 // merged rows per CTA
+    if (a.t_stamps && threadIdx.x == 0) atomicMin(a.t_stamps, (unsigned long long)globaltimer_ns());
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    const uint32_t sbase = smem_addr(smem);
+    __half* rO = reinterpret_cast<__half*>(smem + LY::RO);
+    float* rML = reinterpret_cast<float*>(smem + LY::RML);
+    const uint32_t bar0 = sbase + LY::BARS;
+    // full[NS] (tile landed), empty[NS] (its P V completed); per softmax group q: sfull[q] (S of
+    // the group's tile in TMEM), sfree[q] (read by the group's 4 warps), pready[q] (its P
+    // written), odone[q] (its P V completed); one drain barrier per MMA-issuing thread
+    auto full_bar = [&](int st) { return bar0 + 8u * st; };
+    auto empty_bar = [&](int st) { return bar0 + 8u * (NS + st); };
+    auto sfull_bar = [&](int q) { return bar0 + 8u * (2 * NS + q); };
+    auto sfree_bar = [&](int q) { return bar0 + 8u * (2 * NS + 2 + q); };
+    auto pready_bar = [&](int q) { return bar0 + 8u * (2 * NS + 4 + q); };
+    auto odone_bar = [&](int q) { return bar0 + 8u * (2 * NS + 6 + q); };
+    auto drain_bar = [&](int i) { return bar0 + 8u * (2 * NS + 8 + i); };
+    uint32_t* misc = reinterpret_cast<uint32_t*>(smem + LY::BARS + LY::NBARS * 8);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(&misc[1]);
+    cg::cluster_group cluster = cg::this_cluster();
+    const int s = (int)cluster.block_rank();
+    const int g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int R = a.B * a.G;
+
+    // rows [block_rows, 64) of the V stages are never written by the block tile's copy: zero
+    // them once (P is 0 there, and 0 x garbage could be NaN)
+    if (a.block_rows < kKT) {
+        const int zr = kKT - a.block_rows;
+        for (int k = tid; k < NS * (HD / 64) * zr * 8; k += blockDim.x) {
+            const int piece = k & 7, r = a.block_rows + (k >> 3) % zr, sub = (k >> 3) / zr;
+            const int st = sub / (HD / 64), h = sub % (HD / 64);
+            *reinterpret_cast<uint4*>(smem + (size_t)st * 2 * TB + TB + h * 8192 + r * 128 + piece * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (tid == 0) {
+        for (int i = 0; i < NS; ++i) {
+            ta_mbar_init(full_bar(i), 1);
+            ta_mbar_init(empty_bar(i), 1);
+        }
+        for (int q = 0; q < 2; ++q) {
+            ta_mbar_init(sfull_bar(q), 1);
+            ta_mbar_init(sfree_bar(q), 4);
+            ta_mbar_init(pready_bar(q), 4);
+            ta_mbar_init(odone_bar(q), 1);
+        }
+        ta_mbar_init(drain_bar(0), 1);
+        ta_mbar_init(drain_bar(1), 1);
+        misc[1] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.kc)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.vc)) : "memory");
+    }
+    if (warp == 9) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_addr(&misc[0])),
+                     "r"(LY::TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    ta_fence_before();
+    __syncthreads();
+    ta_fence_after();
+    const uint32_t tmem = misc[0];
+    // dependents are released only once this CTA holds its tensor memory, so a dependent CTA
+    // that allocates before its own dependency wait can never hold columns this CTA waits for
+    pdl_trigger();
+    // every CTA of the cluster has started before any pushes into another's shared memory
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // The context lengths and cached keys/values were written before the kernel that precedes
+    // this one (which signals its dependents only after its own dependency wait); Q, K^d and V^d
+    // are read after the wait below.
+    const int L = a.ctx_len[b];
+    const int n_ctx_tiles = (L + kKT - 1) / kKT, T = n_ctx_tiles + 1;
+    const int t0 = s * (T / S) + min(s, T % S);
+    const int n_tiles = T / S + (s < T % S ? 1 : 0);
+    const int n_ct = max(0, min(t0 + n_tiles, n_ctx_tiles) - t0);
+    // tile t -> stage t % NS: K at [stage][0, TB), V at [stage][TB, 2 TB)
+    auto issue = [&](int t) {
+        const int st = t % NS;
+        const uint32_t kdst = sbase + (uint32_t)st * 2 * TB, bar = full_bar(st);
+        const uint32_t bytes = t < n_ct ? 2 * TB : 2u * (HD / 64) * (uint32_t)a.block_rows * 128u;
+        ta_expect_tx(bar, bytes);
+        for (int h = 0; h < HD / 64; ++h) {
+            if (t < n_ct) {
+                const int y = (t0 + t) * kKT, z = b * a.hkv + g;
+                tma_tile(kdst + h * 8192, &maps.kc, h * 64, y, z, bar);
+                tma_tile(kdst + TB + h * 8192, &maps.vc, h * 64, y, z, bar);
+            } else {
+                tma_tile(kdst + h * 8192, &maps.kd, h * 64, b * a.B, g, bar);
+                tma_tile(kdst + TB + h * 8192, &maps.vd, h * 64, b * a.B, g, bar);
+            }
+        }
+    };
+    int issued = 0;   // warp 8, lane 0
+    // the first context tiles stream in while the projection drains; the block tile waits
+    if (warp == 8 && lane == 0)
+        for (; issued < min(NS, n_ct); ++issued) issue(issued);
+    pdl_wait();
+    if (a.t_stamps && tid == 0) atomicMin(a.t_stamps + a.t_slots, (unsigned long long)globaltimer_ns());
+    const int n32 = a.d_q + 2 * a.d_kv;
+    if (a.qkv32 && n_tiles > n_ct) {
+        // this CTA holds the block tile: its head's K^d (rotated) and V^d rows, rounded to bf16,
+        // go to kd / vd for the tile's TMA load (identical values from every query tile's CTA)
+        const int nb = a.B * (HD / 16);
+        for (int it = tid; it < 2 * nb; it += blockDim.x) {
+            const bool is_v = it >= nb;
+            const int k = (it % nb) / (HD / 16), j0 = ((it % nb) % (HD / 16)) * 8;
+            const float* src = a.qkv32 + ((size_t)b * a.B + k) * n32 + a.d_q + (is_v ? a.d_kv : 0) + g * HD;
+            float x1[8], x2[8], o1[8], o2[8];
+            load8(src + j0, x1);
+            load8(src + j0 + HD / 2, x2);
+            if (!is_v && a.rope) {
+                float cs[8], sn[8];
+                load8(a.rope_cos + (size_t)(L + k) * (HD / 2) + j0, cs);
+                load8(a.rope_sin + (size_t)(L + k) * (HD / 2) + j0, sn);
+                rope8(x1, x2, cs, sn, o1, o2);
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    o1[e] = x1[e];
+                    o2[e] = x2[e];
+                }
+            }
+            bf16* dst = (is_v ? a.vd_w : a.kd_w) + ((size_t)b * a.B + k) * a.d_kv + g * HD + j0;
+            store8(dst, o1);
+            store8(dst + HD / 2, o2);
+        }
+        // the generic stores above before the tensor-memory-access reads of the block tile
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+    }
+    // Q: row r of the tile is block position (qt * 128 + r) / G of query head
+    // g G + (qt * 128 + r) % G, stored K-major and swizzled as [HD/64][128 rows][128 B]; rows
+    // past R are zero. Four items per thread are loaded before any is converted, so that their
+    // global reads are in flight together.
+    if (n_tiles > 0) {
+        constexpr int NQ = kTQ * (HD / 16), U = (NQ + kTThreads - 1) / kTThreads;
+        const bool rot = a.qkv32 && a.rope;
+        float x1[U][8], x2[U][8], cs[U][8], sn[U][8];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int idx = tid + u * kTThreads;
+            const int r = idx / (HD / 16), j0 = (idx % (HD / 16)) * 8;
+            const int rr = qt * kTQ + r;
+            if (idx < NQ && rr < R) {
+                const int kpos = rr / a.G, hh = rr % a.G;
+                if (a.qkv32) {
+                    const float* src = a.qkv32 + ((size_t)b * a.B + kpos) * n32 + (size_t)(g * a.G + hh) * HD;
+                    load8(src + j0, x1[u]);
+                    load8(src + j0 + HD / 2, x2[u]);
+                    if (rot) {
+                        load8(a.rope_cos + (size_t)(L + kpos) * (HD / 2) + j0, cs[u]);
+                        load8(a.rope_sin + (size_t)(L + kpos) * (HD / 2) + j0, sn[u]);
+                    }
+                } else {
+                    const bf16* src = static_cast<const bf16*>(a.q) + ((size_t)b * a.B + kpos) * a.d_q +
+                                      (size_t)(g * a.G + hh) * HD;
+                    load8(src + j0, x1[u]);
+                    load8(src + j0 + HD / 2, x2[u]);
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x1[u][e] = x2[u][e] = 0.f;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int idx = tid + u * kTThreads;
+            if (idx >= NQ) break;
+            const int r = idx / (HD / 16), j0 = (idx % (HD / 16)) * 8;
+            float o1[8], o2[8];
+            if (rot && qt * kTQ + r < R) {
+                rope8(x1[u], x2[u], cs[u], sn[u], o1, o2);
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    o1[e] = x1[u][e];
+                    o2[e] = x2[u][e];
+                }
+            }
+            const int c1 = j0 / 8, c2 = (j0 + HD / 2) / 8;   // 16-byte chunks of the row
+            store8(reinterpret_cast<bf16*>(smem + LY::Q + (c1 >> 3) * (kTQ * 128) + r * 128 +
+                                           (((c1 & 7) ^ (r & 7)) << 4)), o1);
+            store8(reinterpret_cast<bf16*>(smem + LY::Q + (c2 >> 3) * (kTQ * 128) + r * 128 +
+                                           (((c2 & 7) ^ (r & 7)) << 4)), o2);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    __syncthreads();
+
+    // instruction descriptors: fp32 accumulator, bf16 A and B, M 128; S: N 64, both K-major;
+    // P V: N = HD, B (V) MN-major
+    constexpr uint32_t kIdS = (1u << 4) | (1u << 7) | (1u << 10) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
+    constexpr uint32_t kIdO = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | (((uint32_t)HD >> 3) << 17) |
+                              ((128u >> 4) << 24);
+    // TMEM columns: S of group q at [64 q, 64 q + 64), O of group q at [128 + 128 q, + HD)
+    auto tS = [&](int q) { return tmem + 64u * q; };
+    auto tO = [&](int q) { return tmem + 128u + 128u * q; };
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+
+    if (warp == 8) {
+        if (lane == 0) {
+            // ---------------- TMA producer: the stage of tile t is refilled once P V of tile
+            // t - NS has completed
+            for (; issued < n_tiles; ++issued) {
+                const int st = issued % NS;
+                if (issued >= NS && !(ok = ta_wait(empty_bar(st), (uint32_t)(issued / NS - 1) & 1u, abort_flag, a.err)))
+                    break;
+                issue(issued);
+            }
+            // after an abort, the copies in flight land before the shared memory is released
+            if (!ok) {
+                volatile int never = 0;
+                for (int t = max(0, issued - NS); t < issued; ++t)
+                    ta_wait(full_bar(t % NS), (uint32_t)(t / NS) & 1u, &never, a.err);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 10) {
+        if (lane == 0 && n_tiles > 0) {
+            // ---------------- S issue (one thread): S_t into the S buffer of group t & 1 once
+            // the tile has landed and the group has read S_{t-2}; descriptors advance by
+            // address >> 4
+            const uint64_t dQ = ta_desc_k(sbase + LY::Q);
+            for (int t = 0; t < n_tiles && ok; ++t) {
+                const int st = t % NS, q = t & 1;
+                if (!(ok = ta_wait(full_bar(st), (uint32_t)(t / NS) & 1u, abort_flag, a.err))) break;
+                if (t >= 2 && !(ok = ta_wait(sfree_bar(q), (uint32_t)((t >> 1) - 1) & 1u, abort_flag, a.err))) break;
+                ta_fence_after();
+                const uint64_t dK = ta_desc_k(sbase + (uint32_t)st * 2 * TB);
+#pragma unroll
+                for (int kk = 0; kk < HD / 16; ++kk)
+                    ta_mma(tS(q), dQ + (uint64_t)((kk >> 2) * (kTQ * 128 / 16) + (kk & 3) * 2),
+                           dK + (uint64_t)((kk >> 2) * (8192 / 16) + (kk & 3) * 2), kIdS, kk > 0 ? 1u : 0u);
+                ta_commit(sfull_bar(q));
+            }
+            // every MMA this thread issued has completed before the tensor memory is released
+            ta_commit(drain_bar(0));
+            volatile int never = 0;
+            ta_wait(drain_bar(0), 0, &never, a.err);
+        }
+        __syncwarp();
+    } else if (warp == 11) {
+        if (lane == 0 && n_tiles > 0) {
+            // ---------------- P V issue (one thread): O_q += P_t V_t once group q = t & 1 has
+            // written P_t (S_t, which read the stage's K, completed before that); the stage is
+            // released when this P V completes
+            const uint64_t dP = ta_desc_k(sbase + LY::P);
+            for (int t = 0; t < n_tiles && ok; ++t) {
+                const int st = t % NS, q = t & 1;
+                if (!(ok = ta_wait(pready_bar(q), (uint32_t)(t >> 1) & 1u, abort_flag, a.err))) break;
+                ta_fence_after();
+                const uint64_t dV = ta_desc_mn(sbase + (uint32_t)st * 2 * TB + TB);
+                const uint64_t dPq = dP + (uint64_t)(q * (kTQ * 128 / 16));
+#pragma unroll
+                for (int kk = 0; kk < kKT / 16; ++kk)
+                    ta_mma(tO(q), dPq + (uint64_t)(kk * 2), dV + (uint64_t)(kk * 128), kIdO,
+                           (t >= 2 || kk > 0) ? 1u : 0u);
+                ta_commit(odone_bar(q));
+                ta_commit(empty_bar(st));
+            }
+            ta_commit(drain_bar(1));
+            volatile int never = 0;
+            ta_wait(drain_bar(1), 0, &never, a.err);
+        }
+        __syncwarp();
+    } else if (warp >= 8) {
+        // warp 9 holds the tensor memory allocation only
+    } else {
+        // ---------------- softmax group q (warps 4q .. 4q + 3) takes tiles q, q + 2, ...; thread
+        // = query row tid % 128 = TMEM lane. Every wait is taken by the whole warp and its
+        // outcome made warp-uniform (the tcgen05 loads and stores below are warp-collective).
+        const int q = warp >> 2, row = tid & 127;
+        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        const bool warp_rows = qt * kTQ + (warp & 3) * 32 < R;   // the warp holds a query row
+        auto wwait = [&](uint32_t bar, uint32_t parity) {
+            const bool r = ta_wait(bar, parity, abort_flag, a.err);
+            return __all_sync(0xffffffffu, r) != 0;
+        };
+        uint8_t* const prow = smem + LY::P + (uint32_t)q * (kTQ * 128) + row * 128;
+        for (int t = q; t < n_tiles && ok; t += 2) {
+            if (!(ok = wwait(sfull_bar(q), (uint32_t)(t >> 1) & 1u))) break;
+            ta_fence_after();
+            float sv[64];
+            if (warp_rows) {
+                ta_ld32(tS(q) + lane_base, sv);
+                ta_ld32(tS(q) + lane_base + 32, sv + 32);
+            }
+            ta_fence_before();
+            __syncwarp();
+            if (lane == 0) ta_arrive(sfree_bar(q));
+            // keys past the tile's valid count (ragged last tile, block tile) get -inf
+            const int valid = t < n_ct ? min(kKT, L - (t0 + t) * kKT) : a.B;
+            float mx = -INFINITY;
+            if (warp_rows) {
+                if (valid < kKT) {
+#pragma unroll
+                    for (int j = 0; j < 64; ++j) sv[j] = j < valid ? sv[j] : -INFINITY;
+                }
+                // row maximum of the raw scores as a tree, then in log2 units (scale > 0)
+                float m8[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) m8[e] = fmaxf(sv[e], sv[8 + e]);
+#pragma unroll
+                for (int j = 16; j < 64; j += 8)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) m8[e] = fmaxf(m8[e], sv[j + e]);
+                mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                           fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7]))) * a.scale_log2;
+            }
+            // P V of the group's previous tile has completed: its O is stable and P buffer q free
+            if (t >= 2 && !(ok = wwait(odone_bar(q), (uint32_t)((t >> 1) - 1) & 1u))) break;
+            ta_fence_after();
+            if (warp_rows) {
+                const bool raise = mx > m_used + kRescale;
+                if (__any_sync(0xffffffffu, raise && t >= 2)) {
+                    const float alpha = raise ? ex2(m_used - mx) : 1.0f;
+#pragma unroll
+                    for (int c = 0; c < HD / 32; ++c) {
+                        float ov[32];
+                        ta_ld32(tO(q) + lane_base + c * 32, ov);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) ov[i] *= alpha;
+                        ta_st32(tO(q) + lane_base + c * 32, ov);
+                    }
+                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                }
+                if (raise) {
+                    l *= ex2(m_used - mx);   // 0 on the group's first tile (m_used = -inf)
+                    m_used = mx;
+                }
+                // P = 2^(s scale - m): one FMA and one ex2 per key; eight partial row sums
+                const float neg_m = -m_used;
+                float ls[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    float p[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        p[e] = ex2(fmaf(sv[c * 8 + e], a.scale_log2, neg_m));
+                        ls[e] += p[e];
+                    }
+                    uint4 u;
+                    u.x = pack_bf16(p[0], p[1]);
+                    u.y = pack_bf16(p[2], p[3]);
+                    u.z = pack_bf16(p[4], p[5]);
+                    u.w = pack_bf16(p[6], p[7]);
+                    *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) = u;
+                }
+                l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            }
+            ta_fence_before();
+            __syncwarp();
+            if (lane == 0) ta_arrive(pready_bar(q));
+        }
+        // the group's last P V has completed: O_q holds the group's whole key range
+        const int last = q + ((n_tiles - 1 - q) >> 1) * 2;   // the group's last tile
+        if (ok && n_tiles > q) ok = wwait(odone_bar(q), (uint32_t)(last >> 1) & 1u);
+        ta_fence_after();
+        // group 1 leaves its (m, l) for group 0 in its own (now unused) P buffer
+        if (q == 1) {
+            float2* xml = reinterpret_cast<float2*>(smem + LY::P + kTQ * 128);
+            xml[row] = make_float2(n_tiles > 1 && ok ? m_used : -INFINITY, n_tiles > 1 && ok ? l : 0.f);
+        }
+    }
+    if (!ok && lane == 0) atomicOr(a.err, DFLARE_DEVERR_TIMEOUT);
+    __syncthreads();
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+    // Push the partial: group 0 combines both groups' (m, l, O) of row r and writes it to CTA
+    // r / RP at [s * RP + r % RP]. ok is warp-uniform, so the tcgen05 loads stay collective; a
+    // group without tiles (m = -inf) contributes nothing and its O is not read.
+    if (warp < 4 && qt * kTQ + warp * 32 < R) {
+        const int r = tid;
+        const bool row_ok = qt * kTQ + r < R;
+        const float2 mlB = reinterpret_cast<const float2*>(smem + LY::P + kTQ * 128)[r];
+        const bool hA = ok && n_tiles > 0, hB = hA && mlB.x != -INFINITY;
+        const float mA = hA ? m_used : -INFINITY;
+        const float M = fmaxf(mA, mlB.x);
+        const float wA = hA ? ex2(mA - M) : 0.f, wB = hB ? ex2(mlB.x - M) : 0.f;
+        const float lt = (hA ? l * wA : 0.f) + (hB ? mlB.y * wB : 0.f);
+        const float inv = lt > 0.f ? 1.0f / lt : 0.f;
+        const float cA = wA * inv, cB = wB * inv;
+        __half* dst = cluster.map_shared_rank(rO, r / RP) + (size_t)(s * RP + r % RP) * HD;
+        const uint32_t lb = (uint32_t)(warp * 32) << 16;
+#pragma unroll
+        for (int c = 0; c < HD / 32; ++c) {
+            float ov[32], ob[32];
+            if (hA) {
+                ta_ld32(tO(0) + lb + c * 32, ov);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) ov[i] = 0.f;
+            }
+            if (__any_sync(0xffffffffu, hB)) ta_ld32(tO(1) + lb + c * 32, ob);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] = hB ? fmaf(ob[i], cB, ov[i] * cA) : ov[i] * cA;
+            if (row_ok) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    uint4 u;
+                    __half2* h = reinterpret_cast<__half2*>(&u);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(ov[k * 8 + 2 * e], ov[k * 8 + 2 * e + 1]);
+                    *reinterpret_cast<uint4*>(dst + c * 32 + k * 8) = u;
+                }
+            }
+        }
+        if (row_ok)
+            *reinterpret_cast<float2*>(cluster.map_shared_rank(rML, r / RP) + 2 * (s * RP + r % RP)) =
+                make_float2(hA ? M : -INFINITY, lt);
+    }
+    // every partial has arrived; after this barrier no CTA touches another's shared memory
+    ta_fence_before();
+    cluster.sync();
+    if (warp == 9) {
+        ta_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(LY::TMEM_COLS)
+                     : "memory");
+    }
+    // merge this CTA's RP rows: TPR threads per row, EPT contiguous output elements per thread
+    constexpr int TPR = 128 / RP, EPT = HD / TPR;
+    static_assert(EPT % 2 == 0, "merge slice must be a whole number of half2");
+    const int lr = tid / TPR, lt = tid % TPR;
+    const int rg = qt * kTQ + s * RP + lr;
+    if (tid < 128 && rg < R) {
+        float w[S];
+        float M = -INFINITY;
+#pragma unroll
+        for (int p = 0; p < S; ++p) M = fmaxf(M, rML[2 * (p * RP + lr)]);
+        float den = 0.f;
+#pragma unroll
+        for (int p = 0; p < S; ++p) {
+            const float mp = rML[2 * (p * RP + lr)], lp = rML[2 * (p * RP + lr) + 1];
+            w[p] = mp == -INFINITY ? 0.f : lp * exp2f(mp - M);
+            den += w[p];
+        }
+        const float inv = 1.0f / den;
+        const int kpos = rg / a.G, hh = rg % a.G;
+        bf16* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + lt * EPT;
+#pragma unroll
+        for (int k = 0; k < EPT; k += 2) {
+            float v0 = 0.f, v1 = 0.f;
+#pragma unroll
+            for (int p = 0; p < S; ++p) {
+                const float2 f = __half22float2(
+                    *reinterpret_cast<const __half2*>(rO + (size_t)(p * RP + lr) * HD + lt * EPT + k));
+                v0 = fmaf(w[p], f.x, v0);
+                v1 = fmaf(w[p], f.y, v1);
+            }
+            *reinterpret_cast<__nv_bfloat162*>(orow + k) = __floats2bfloat162_rn(v0 * inv, v1 * inv);
+        }
+    }
+    if (a.t_stamps) {
+        __syncthreads();
+        if (tid == 0) atomicMax(a.t_stamps + 2 * a.t_slots, (unsigned long long)globaltimer_ns());
+    }
+}
+
 // ------------------------------------------------------------------ CUDA-core path
 
 template <class T, int HD>
@@ -705,6 +1335,80 @@ int max_attention_cluster() {
     return cached;
 }
 
+template <int HD, int S>
+cudaError_t configure_tc() {
+    static PerDeviceOnce configured;
+    return configured([] {
+        cudaError_t r = cudaFuncSetAttribute(attn_tc_kernel<HD, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)tc_attn_smem_bytes<HD>());
+        if (r == cudaSuccess && S > 8)
+            r = cudaFuncSetAttribute(attn_tc_kernel<HD, S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        return r;
+    });
+}
+
+template <int HD, int S>
+cudaError_t launch_tc(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
+    const cudaError_t e = configure_tc<HD, S>();
+    if (e != cudaSuccess) return e;
+    return launch_cluster(c->pdl, S, attn_tc_kernel<HD, S>, dim3(S, a.hkv * a.q_tiles, c->batch),
+                          dim3(kTThreads), tc_attn_smem_bytes<HD>(), s, maps, a, static_cast<bf16*>(c->attn));
+}
+
+template <int HD>
+cudaError_t run_tc(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
+    switch (a.splits) {
+        case 1: return launch_tc<HD, 1>(c, maps, a, s);
+        case 2: return launch_tc<HD, 2>(c, maps, a, s);
+        case 4: return launch_tc<HD, 4>(c, maps, a, s);
+        case 8: return launch_tc<HD, 8>(c, maps, a, s);
+        default: return launch_tc<HD, 16>(c, maps, a, s);
+    }
+}
+
+// Clusters of S tcgen05-attention CTAs (one per SM) that the device runs at once; queried once per
+// device (0 where the cluster size cannot be scheduled).
+template <int HD, int S>
+int tc_active_clusters() {
+    static std::atomic<int> cache[64];   // per device (modulo 64): 0 = not yet queried
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    std::atomic<int>& slot = cache[dev & 63];
+    if (const int known = slot.load(std::memory_order_acquire)) return known - 1;
+    int n = 0;
+    if (configure_tc<HD, S>() == cudaSuccess) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(S, 1, 1);
+        cfg.blockDim = dim3(kTThreads);
+        cfg.dynamicSmemBytes = tc_attn_smem_bytes<HD>();
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = S;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<HD, S>, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    slot.store(n + 1, std::memory_order_release);
+    return n;
+}
+
+template <int HD>
+int tc_active_clusters_of(int sp) {
+    switch (sp) {
+        case 1: return tc_active_clusters<HD, 1>();
+        case 2: return tc_active_clusters<HD, 2>();
+        case 4: return tc_active_clusters<HD, 4>();
+        case 8: return tc_active_clusters<HD, 8>();
+        default: return tc_active_clusters<HD, 16>();
+    }
+}
+
 template <class T, int HD>
 cudaError_t run_simt(dflare_ctx* c, const AttnArgs& a, cudaStream_t s) {
     cudaError_t e = launch_kernel(c->pdl, attn_simt_kernel<T, HD>,
@@ -779,9 +1483,30 @@ int attention_ctas_per_sm() {
     return n;
 }
 
+// tcgen05 path: one CTA per SM, 128 query rows per CTA. The largest cluster (16, 8, 4, 2) of
+// which all batch x H_kv x query-tile clusters run at once (the device's count of co-resident
+// clusters of that size, queried once), with at least two 64-key tiles per CTA at the host's upper
+// bound of the context length; else one CTA per (sequence, head, query tile).
+int attention_tc_splits(const dflare_config& g, int batch, int len_ub, int (*active)(int)) {
+    const int G = g.n_q_heads / g.n_kv_heads;
+    const int q_tiles = (g.block * G + kTQ - 1) / kTQ;
+    const int base = batch * g.n_kv_heads * q_tiles;
+    const int tiles = (len_ub + g.block + kKT - 1) / kKT;
+    for (int sp = 16; sp > 1; sp >>= 1)
+        if (2 * sp <= tiles && base <= active(sp)) return sp;
+    return 1;
+}
+
+static bool use_tc_attention(const dflare_config& g) {
+    return g.dtype == DFLARE_BF16 && !(g.flags & DFLARE_FLAG_MMA_SYNC_ATTENTION);
+}
+
 int attention_launch_splits(const dflare_ctx* c) {
     const dflare_config& g = c->cfg;
     if (g.dtype == DFLARE_F32) return attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
+    if (use_tc_attention(g))
+        return attention_tc_splits(g, c->batch, c->ctx_ub,
+                                   g.head_dim == 64 ? tc_active_clusters_of<64> : tc_active_clusters_of<128>);
     const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
     const int per_sm = g.head_dim == 64 ? attention_ctas_per_sm<64>() : attention_ctas_per_sm<128>();
     return attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc, per_sm);
@@ -847,12 +1572,14 @@ cudaError_t launch_attention(dflare_ctx* c, int layer, cudaStream_t s) {
     maps.kd = c->attn_maps[2 * g.n_draft_layers];
     maps.vd = c->attn_maps[2 * g.n_draft_layers + 1];
     a.block_rows = std::min(kKT, g.max_batch * g.block);
-    const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
-    const int per_sm = g.head_dim == 64 ? attention_ctas_per_sm<64>() : attention_ctas_per_sm<128>();
-    a.splits = attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc, per_sm);
+    a.splits = attention_launch_splits(c);
     if (c->t_stamps && c->t_next < c->t_slots) {
         a.t_stamps = c->t_stamps + c->t_next++;
         a.t_slots = c->t_slots;
+    }
+    if (use_tc_attention(g)) {
+        a.q_tiles = (a.B * a.G + kTQ - 1) / kTQ;
+        return g.head_dim == 64 ? run_tc<64>(c, maps, a, s) : run_tc<128>(c, maps, a, s);
     }
     return g.head_dim == 64 ? run_mma<64>(c, maps, a, s) : run_mma<128>(c, maps, a, s);
 }

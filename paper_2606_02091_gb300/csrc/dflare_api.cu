@@ -63,7 +63,7 @@ bool check_config(const dflare_config* g, std::string* why) {
     if (g->dtype != DFLARE_BF16 && g->dtype != DFLARE_F32) return bad("dtype must be DFLARE_BF16 or DFLARE_F32");
     if (g->flags & ~(DFLARE_FLAG_NO_BLOCK_ROPE | DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_SIMT_GEMM |
                      DFLARE_FLAG_SERIAL_LAUNCH | DFLARE_FLAG_SHARED_KV | DFLARE_FLAG_FUSION_FC |
-                     DFLARE_FLAG_DFLASH_FC | DFLARE_FLAG_DETERMINISTIC))
+                     DFLARE_FLAG_DFLASH_FC | DFLARE_FLAG_DETERMINISTIC | DFLARE_FLAG_MMA_SYNC_ATTENTION))
         return bad("unknown flag bits");
     if ((g->flags & DFLARE_FLAG_DFLASH_FC) &&
         (g->flags & (DFLARE_FLAG_RAW_FUSION | DFLARE_FLAG_FUSION_FC)))

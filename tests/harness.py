@@ -65,6 +65,13 @@ BLOCK2 = synth.Workload(
     synth.Shape(d=256, n_draft_layers=2, n_target_layers=2, n_q_heads=4, n_kv_heads=2,
                 head_dim=128, ffn=256, vocab=300, block=2),
     (64, 129), 0.8, seed=18)
+# 160 query rows per KV head (G 10, block 16): two 128-row query tiles of the tcgen05 attention,
+# the second holding 32 rows, and three 64-row tiles of the mma.sync attention
+QT2 = synth.Workload(
+    "qt2_bf16_g10",
+    synth.Shape(d=512, n_draft_layers=2, n_target_layers=2, n_q_heads=20, n_kv_heads=2,
+                head_dim=64, ffn=512, vocab=600, block=16),
+    (210, 77), 0.8, seed=20)
 TINY = synth.preset("tiny_f32")
 
 

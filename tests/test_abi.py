@@ -52,7 +52,7 @@ def _cfg(**kw):
     ("n_target_layers", 0), ("n_target_layers", 65), ("head_dim", 96), ("n_q_heads", 3),
     ("n_kv_heads", 0), ("ffn", 100), ("vocab", 1), ("mask_token_id", 4096), ("mask_token_id", -1),
     ("block", 0), ("block", 33), ("max_batch", 0), ("max_batch", 65), ("max_ctx", 0),
-    ("max_fuse_rows", 0), ("rms_eps", -1.0), ("rope_theta", 0.0), ("dtype", 2), ("flags", 0x100), ("flags", 0x200),
+    ("max_fuse_rows", 0), ("rms_eps", -1.0), ("rope_theta", 0.0), ("dtype", 2), ("flags", 0x200), ("flags", 0x400),
     ("flags", 0x40 | 0x2), ("flags", 0x40 | 0x20),   # DFlash FC with -Softmax / +FC
 ])
 def test_create_rejects_bad_config_on_host(lib, field, value):

@@ -15,7 +15,8 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, MULTI_TILE, SMALL_HD128, SMALL_HD64, TINY, WIDE_B16,
+from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, MULTI_TILE, QT2, SMALL_HD128, SMALL_HD64, TINY,
+                           WIDE_B16,
                            GpuSide, check_elem, check_kv, check_rows, check_tokens, f64, oracle_for,
                            rel_err, tolerance, verified_steps)
 
@@ -156,6 +157,26 @@ def test_simt_gemm_agrees_with_tcgen05_gemm():
     tb, lb, hb = b.draft(x_t)
     assert rel_err(ha, hb) <= tolerance(w)
     assert rel_err(la, lb) <= tolerance(w)
+
+
+@pytest.mark.parametrize("w", [SMALL_HD128, G8, QT2, D10, BLOCK1], ids=lambda w: w.name)
+@pytest.mark.parametrize("kernel", ["tcgen05", "mma_sync"])
+def test_attention_kernels_match_oracle(w, kernel):
+    """Both bf16 attention kernels (the tcgen05 one, 128 query rows per CTA, and the mma.sync one,
+    64 per CTA) on query-row counts per KV head of 64, 128, 160 (two 128-row tiles, the second
+    ragged), 8 (a partial warp) and 2: the drafted block and two verified steps against the
+    oracle."""
+    from paper_2606_02091_gb300 import FLAG_MMA_SYNC_ATTENTION
+    g = GpuSide(w, flags=FLAG_MMA_SYNC_ATTENTION if kernel == "mma_sync" else 0)
+    o = oracle_for(w, g.W)
+    g.fuse(w.ctx_lens, want_fused=False)
+    for b, n in enumerate(w.ctx_lens):
+        o.fuse_context(b, synth.hidden_states(w, b, 0, n))
+    x_t = synth.initial_tokens(w)
+    tok, logits, hidden = g.draft(x_t)
+    _check_draft(w, tok, logits, hidden, [o.draft_block(b, int(x_t[b])) for b in range(w.batch)], o)
+    assert verified_steps(w, g, o, n_steps=2) >= w.batch
+    assert g.lib.device_error() == 0
 
 
 @pytest.mark.parametrize("w", [WIDE_B16, BLOCK32, MULTI_TILE], ids=lambda w: w.name)
