@@ -587,18 +587,24 @@ constexpr int kTQ = 128;            // query rows per CTA (UMMA M)
 constexpr int kTThreads = 384;      // warps 0-3, 4-7: softmax groups; 8: TMA; 9: TMEM; 10, 11: MMA
 constexpr float kRescale = 8.0f;    // growth (log2) of a row maximum that triggers a rescale
 
+constexpr int kMaxSplits = 16;     // cluster size limit (non-portable above 8)
 template <int HD>
 struct TcAttnLayout {
-    static constexpr int NS = HD == 128 ? 4 : 8;               // K/V stages
+    static constexpr int NS = HD == 128 ? 5 : 10;              // K/V stages
     static constexpr uint32_t TB = HD * 128;                    // one 64-key K or V tile
     static constexpr uint32_t Q = NS * 2 * TB;                  // Q [HD/64][128 rows][128 B]
     static constexpr uint32_t P = Q + (uint32_t)kTQ * HD * 2;   // P [group][128 rows][64 keys] bf16
-    static constexpr uint32_t RO = P + 2u * kTQ * 128;          // pushed partials O / l, fp16
-    static constexpr uint32_t RML = RO + (uint32_t)kTQ * HD * 2;   // pushed (m, l)
-    static constexpr uint32_t BARS = RML + (uint32_t)kTQ * 8;   // mbarriers, then two words
+    static constexpr uint32_t BARS = P + 2u * kTQ * 128;        // mbarriers, then two words
     static constexpr int NBARS = 2 * NS + 10;
     static constexpr uint32_t BYTES = BARS + NBARS * 8 + 16;
+    // After the key loop the (then idle) stages hold the cluster merge: the pushed partials O / l
+    // in fp16 [S RP <= 128 + 15 rows][HD], their (m, l) and the merge weights [RP][S].
+    static constexpr int MR = kTQ + kMaxSplits;
+    static constexpr uint32_t RO = 0;
+    static constexpr uint32_t RML = (uint32_t)MR * HD * 2;
+    static constexpr uint32_t RW = RML + (uint32_t)MR * 8;
     static constexpr uint32_t TMEM_COLS = 512;                  // S_A, S_B (64 each), O_A, O_B
+    static_assert(RW + (uint32_t)MR * kMaxSplits * 4 <= NS * 2 * TB, "merge buffers exceed the stages");
     static_assert(1024 + BYTES <= 232448, "tcgen05 attention exceeds 227 KB of shared memory");
 };
 template <int HD>
@@ -705,19 +711,17 @@ __device__ __forceinline__ void rope8(const float* x1, const float* x2, const fl
     }
 }
 
-template <int HD, int S>
+template <int HD>
 __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_constant__ AttnMaps maps,
                                                               const AttnArgs a, bf16* __restrict__ out) {
     using LY = TcAttnLayout<HD>;
     constexpr int NS = LY::NS;
     constexpr uint32_t TB = LY::TB;
-    constexpr int RP = kTQ / S;                 // merged rows per CTA
+    const int S = a.splits;                     // the cluster: one CTA per split
     if (a.t_stamps && threadIdx.x == 0) atomicMin(a.t_stamps, (unsigned long long)globaltimer_ns());
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_addr(smem);
-    __half* rO = reinterpret_cast<__half*>(smem + LY::RO);
-    float* rML = reinterpret_cast<float*>(smem + LY::RML);
     const uint32_t bar0 = sbase + LY::BARS;
     // full[NS] (tile landed), empty[NS] (its P V completed); per softmax group q: sfull[q] (S of
     // the group's tile in TMEM), sfree[q] (read by the group's 4 warps), pready[q] (its P
@@ -736,6 +740,7 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
     const int g = blockIdx.y % a.hkv, qt = blockIdx.y / a.hkv, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = a.B * a.G;
+    const int rows = min(kTQ, R - qt * kTQ);    // query rows of this tile
 
     // rows [block_rows, 64) of the V stages are never written by the block tile's copy: zero
     // them once (P is 0 there, and 0 x garbage could be NaN)
@@ -781,8 +786,6 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
     // dependents are released only once this CTA holds its tensor memory, so a dependent CTA
     // that allocates before its own dependency wait can never hold columns this CTA waits for
     pdl_trigger();
-    // every CTA of the cluster has started before any pushes into another's shared memory
-    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     // The context lengths and cached keys/values were written before the kernel that precedes
     // this one (which signals its dependents only after its own dependency wait); Q, K^d and V^d
     // are read after the wait below.
@@ -1082,14 +1085,20 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         }
     }
     if (!ok && lane == 0) atomicOr(a.err, DFLARE_DEVERR_TIMEOUT);
+    // every CTA of the cluster has finished with its stages (copies landed, MMAs drained) before
+    // any partial is pushed into them
     __syncthreads();
-    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
-    // Push the partial: group 0 combines both groups' (m, l, O) of row r and writes it to CTA
-    // r / RP at [s * RP + r % RP]. ok is warp-uniform, so the tcgen05 loads stay collective; a
+    cluster.sync();
+    // Push the partial: group 0 combines both groups' (m, l, O) of query row r and writes it to
+    // CTA r / RP at [s RP + r % RP]. ok is warp-uniform, so the tcgen05 loads stay collective; a
     // group without tiles (m = -inf) contributes nothing and its O is not read.
-    if (warp < 4 && qt * kTQ + warp * 32 < R) {
+    const int RP = (rows + S - 1) / S;
+    __half* rO = reinterpret_cast<__half*>(smem + LY::RO);
+    float2* rML = reinterpret_cast<float2*>(smem + LY::RML);
+    float* rW = reinterpret_cast<float*>(smem + LY::RW);
+    if (warp < 4 && warp * 32 < rows) {
         const int r = tid;
-        const bool row_ok = qt * kTQ + r < R;
+        const bool row_ok = r < rows;
         const float2 mlB = reinterpret_cast<const float2*>(smem + LY::P + kTQ * 128)[r];
         const bool hA = ok && n_tiles > 0, hB = hA && mlB.x != -INFINITY;
         const float mA = hA ? m_used : -INFINITY;
@@ -1098,34 +1107,30 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         const float lt = (hA ? l * wA : 0.f) + (hB ? mlB.y * wB : 0.f);
         const float inv = lt > 0.f ? 1.0f / lt : 0.f;
         const float cA = wA * inv, cB = wB * inv;
-        __half* dst = cluster.map_shared_rank(rO, r / RP) + (size_t)(s * RP + r % RP) * HD;
+        const int dst_cta = row_ok ? r / RP : 0, dst_row = s * RP + (row_ok ? r % RP : 0);
+        __half* dst = cluster.map_shared_rank(rO, dst_cta) + (size_t)dst_row * HD;
         const uint32_t lb = (uint32_t)(warp * 32) << 16;
+        if (hA) {
 #pragma unroll
-        for (int c = 0; c < HD / 32; ++c) {
-            float ov[32], ob[32];
-            if (hA) {
+            for (int c = 0; c < HD / 32; ++c) {
+                float ov[32], ob[32];
                 ta_ld32(tO(0) + lb + c * 32, ov);
-            } else {
+                if (__any_sync(0xffffffffu, hB)) ta_ld32(tO(1) + lb + c * 32, ob);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) ov[i] = 0.f;
-            }
-            if (__any_sync(0xffffffffu, hB)) ta_ld32(tO(1) + lb + c * 32, ob);
+                for (int i = 0; i < 32; ++i) ov[i] = hB ? fmaf(ob[i], cB, ov[i] * cA) : ov[i] * cA;
+                if (row_ok) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) ov[i] = hB ? fmaf(ob[i], cB, ov[i] * cA) : ov[i] * cA;
-            if (row_ok) {
+                    for (int k = 0; k < 4; ++k) {
+                        uint4 u;
+                        __half2* h = reinterpret_cast<__half2*>(&u);
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    uint4 u;
-                    __half2* h = reinterpret_cast<__half2*>(&u);
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(ov[k * 8 + 2 * e], ov[k * 8 + 2 * e + 1]);
-                    *reinterpret_cast<uint4*>(dst + c * 32 + k * 8) = u;
+                        for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(ov[k * 8 + 2 * e], ov[k * 8 + 2 * e + 1]);
+                        *reinterpret_cast<uint4*>(dst + c * 32 + k * 8) = u;
+                    }
                 }
             }
         }
-        if (row_ok)
-            *reinterpret_cast<float2*>(cluster.map_shared_rank(rML, r / RP) + 2 * (s * RP + r % RP)) =
-                make_float2(hA ? M : -INFINITY, lt);
+        if (row_ok) *cluster.map_shared_rank(rML + dst_row, dst_cta) = make_float2(hA ? M : -INFINITY, lt);
     }
     // every partial has arrived; after this barrier no CTA touches another's shared memory
     ta_fence_before();
@@ -1135,38 +1140,41 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(LY::TMEM_COLS)
                      : "memory");
     }
-    // merge this CTA's RP rows: TPR threads per row, EPT contiguous output elements per thread
-    constexpr int TPR = 128 / RP, EPT = HD / TPR;
-    static_assert(EPT % 2 == 0, "merge slice must be a whole number of half2");
-    const int lr = tid / TPR, lt = tid % TPR;
-    const int rg = qt * kTQ + s * RP + lr;
-    if (tid < 128 && rg < R) {
-        float w[S];
+    // merge this CTA's rows [s RP, min(rows, s RP + RP)): the weights of the S partials of each
+    // row (a partial with m = -inf weighs 0 and its O is not read), then 8 output elements per item
+    const int r0 = s * RP, nr = max(0, min(rows - r0, RP));
+    for (int i = tid; i < nr; i += kTThreads) {
         float M = -INFINITY;
-#pragma unroll
-        for (int p = 0; p < S; ++p) M = fmaxf(M, rML[2 * (p * RP + lr)]);
+        for (int p = 0; p < S; ++p) M = fmaxf(M, rML[p * RP + i].x);
         float den = 0.f;
-#pragma unroll
         for (int p = 0; p < S; ++p) {
-            const float mp = rML[2 * (p * RP + lr)], lp = rML[2 * (p * RP + lr) + 1];
-            w[p] = mp == -INFINITY ? 0.f : lp * exp2f(mp - M);
-            den += w[p];
+            const float2 ml = rML[p * RP + i];
+            const float w = ml.x == -INFINITY ? 0.f : ml.y * exp2f(ml.x - M);
+            rW[i * kMaxSplits + p] = w;
+            den += w;
         }
         const float inv = 1.0f / den;
-        const int kpos = rg / a.G, hh = rg % a.G;
-        bf16* orow = out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + lt * EPT;
+        for (int p = 0; p < S; ++p) rW[i * kMaxSplits + p] *= inv;
+    }
+    __syncthreads();
+    for (int it = tid; it < nr * (HD / 8); it += kTThreads) {
+        const int i = it / (HD / 8), c = it % (HD / 8);
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int p = 0; p < S; ++p) {
+            const float w = rW[i * kMaxSplits + p];
+            if (w != 0.f) {
+                const uint4 v = *reinterpret_cast<const uint4*>(rO + (size_t)(p * RP + i) * HD + c * 8);
+                const __half2* hv = reinterpret_cast<const __half2*>(&v);
 #pragma unroll
-        for (int k = 0; k < EPT; k += 2) {
-            float v0 = 0.f, v1 = 0.f;
-#pragma unroll
-            for (int p = 0; p < S; ++p) {
-                const float2 f = __half22float2(
-                    *reinterpret_cast<const __half2*>(rO + (size_t)(p * RP + lr) * HD + lt * EPT + k));
-                v0 = fmaf(w[p], f.x, v0);
-                v1 = fmaf(w[p], f.y, v1);
+                for (int e = 0; e < 4; ++e) {
+                    const float2 f = __half22float2(hv[e]);
+                    acc[2 * e] = fmaf(w, f.x, acc[2 * e]);
+                    acc[2 * e + 1] = fmaf(w, f.y, acc[2 * e + 1]);
+                }
             }
-            *reinterpret_cast<__nv_bfloat162*>(orow + k) = __floats2bfloat162_rn(v0 * inv, v1 * inv);
         }
+        const int rg = qt * kTQ + r0 + i, kpos = rg / a.G, hh = rg % a.G;
+        store8(out + ((size_t)b * a.B + kpos) * a.d_q + (size_t)(g * a.G + hh) * HD + c * 8, acc);
     }
     if (a.t_stamps) {
         __syncthreads();
@@ -1335,78 +1343,56 @@ int max_attention_cluster() {
     return cached;
 }
 
-template <int HD, int S>
+template <int HD>
 cudaError_t configure_tc() {
     static PerDeviceOnce configured;
     return configured([] {
-        cudaError_t r = cudaFuncSetAttribute(attn_tc_kernel<HD, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t r = cudaFuncSetAttribute(attn_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)tc_attn_smem_bytes<HD>());
-        if (r == cudaSuccess && S > 8)
-            r = cudaFuncSetAttribute(attn_tc_kernel<HD, S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (r == cudaSuccess)
+            r = cudaFuncSetAttribute(attn_tc_kernel<HD>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         return r;
     });
 }
 
-template <int HD, int S>
-cudaError_t launch_tc(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
-    const cudaError_t e = configure_tc<HD, S>();
+template <int HD>
+cudaError_t run_tc(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
+    const cudaError_t e = configure_tc<HD>();
     if (e != cudaSuccess) return e;
-    return launch_cluster(c->pdl, S, attn_tc_kernel<HD, S>, dim3(S, a.hkv * a.q_tiles, c->batch),
+    return launch_cluster(c->pdl, a.splits, attn_tc_kernel<HD>, dim3(a.splits, a.hkv * a.q_tiles, c->batch),
                           dim3(kTThreads), tc_attn_smem_bytes<HD>(), s, maps, a, static_cast<bf16*>(c->attn));
 }
 
+// Clusters of sp tcgen05-attention CTAs (one per SM) that the device runs at once, sp = 1 .. 16;
+// queried once per device (0 where the cluster size cannot be scheduled).
 template <int HD>
-cudaError_t run_tc(dflare_ctx* c, const AttnMaps& maps, const AttnArgs& a, cudaStream_t s) {
-    switch (a.splits) {
-        case 1: return launch_tc<HD, 1>(c, maps, a, s);
-        case 2: return launch_tc<HD, 2>(c, maps, a, s);
-        case 4: return launch_tc<HD, 4>(c, maps, a, s);
-        case 8: return launch_tc<HD, 8>(c, maps, a, s);
-        default: return launch_tc<HD, 16>(c, maps, a, s);
-    }
-}
-
-// Clusters of S tcgen05-attention CTAs (one per SM) that the device runs at once; queried once per
-// device (0 where the cluster size cannot be scheduled).
-template <int HD, int S>
-int tc_active_clusters() {
-    static std::atomic<int> cache[64];   // per device (modulo 64): 0 = not yet queried
+int tc_active_clusters(int sp) {
+    static std::atomic<int> cache[64][kMaxSplits];   // per device (modulo 64): 0 = not yet queried
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) {
+    if (sp < 1 || sp > kMaxSplits || cudaGetDevice(&dev) != cudaSuccess) {
         cudaGetLastError();
         return 0;
     }
-    std::atomic<int>& slot = cache[dev & 63];
+    std::atomic<int>& slot = cache[dev & 63][sp - 1];
     if (const int known = slot.load(std::memory_order_acquire)) return known - 1;
     int n = 0;
-    if (configure_tc<HD, S>() == cudaSuccess) {
+    if (configure_tc<HD>() == cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(S, 1, 1);
+        cfg.gridDim = dim3(sp, 1, 1);
         cfg.blockDim = dim3(kTThreads);
         cfg.dynamicSmemBytes = tc_attn_smem_bytes<HD>();
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = S;
+        attr[0].val.clusterDim.x = sp;
         attr[0].val.clusterDim.y = 1;
         attr[0].val.clusterDim.z = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<HD, S>, &cfg) != cudaSuccess) n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<HD>, &cfg) != cudaSuccess) n = 0;
     }
     cudaGetLastError();
     slot.store(n + 1, std::memory_order_release);
     return n;
-}
-
-template <int HD>
-int tc_active_clusters_of(int sp) {
-    switch (sp) {
-        case 1: return tc_active_clusters<HD, 1>();
-        case 2: return tc_active_clusters<HD, 2>();
-        case 4: return tc_active_clusters<HD, 4>();
-        case 8: return tc_active_clusters<HD, 8>();
-        default: return tc_active_clusters<HD, 16>();
-    }
 }
 
 template <class T, int HD>
@@ -1483,16 +1469,18 @@ int attention_ctas_per_sm() {
     return n;
 }
 
-// tcgen05 path: one CTA per SM, 128 query rows per CTA. The largest cluster (16, 8, 4, 2) of
-// which all batch x H_kv x query-tile clusters run at once (the device's count of co-resident
-// clusters of that size, queried once), with at least two 64-key tiles per CTA at the host's upper
-// bound of the context length; else one CTA per (sequence, head, query tile).
+// tcgen05 path: one CTA per SM, 128 query rows per CTA. The largest cluster size sp (1 .. 16, not
+// only powers of two) for which all batch x H_kv x query-tile clusters run at once (the device's
+// count of co-resident clusters of that size, queried once), with at least two 64-key tiles per
+// CTA at the host's upper bound of the context length. At one CTA per SM a GB300 runs 36 clusters
+// of 4, 23 of 6, 15 of 8, 8 of 12 and 7 of 16, so e.g. 16 (sequence, head) pairs take 6 splits
+// (96 SMs) rather than 4, and 8 pairs take 12 rather than 8.
 int attention_tc_splits(const dflare_config& g, int batch, int len_ub, int (*active)(int)) {
     const int G = g.n_q_heads / g.n_kv_heads;
     const int q_tiles = (g.block * G + kTQ - 1) / kTQ;
     const int base = batch * g.n_kv_heads * q_tiles;
     const int tiles = (len_ub + g.block + kKT - 1) / kKT;
-    for (int sp = 16; sp > 1; sp >>= 1)
+    for (int sp = kMaxSplits; sp > 1; --sp)
         if (2 * sp <= tiles && base <= active(sp)) return sp;
     return 1;
 }
@@ -1506,7 +1494,7 @@ int attention_launch_splits(const dflare_ctx* c) {
     if (g.dtype == DFLARE_F32) return attention_splits(g, c->batch, c->num_sms, c->ctx_ub);
     if (use_tc_attention(g))
         return attention_tc_splits(g, c->batch, c->ctx_ub,
-                                   g.head_dim == 64 ? tc_active_clusters_of<64> : tc_active_clusters_of<128>);
+                                   g.head_dim == 64 ? tc_active_clusters<64> : tc_active_clusters<128>);
     const int maxc = g.head_dim == 64 ? max_attention_cluster<64>() : max_attention_cluster<128>();
     const int per_sm = g.head_dim == 64 ? attention_ctas_per_sm<64>() : attention_ctas_per_sm<128>();
     return attention_cluster_splits(g, c->batch, c->num_sms, c->ctx_ub, maxc, per_sm);
