@@ -7,12 +7,17 @@
 // sees every key. The keys of one (sequence, head) are cut into contiguous ranges so that
 // batch x H_kv x splits CTAs cover the GPU even for a single sequence.
 //
-// bf16 path: 64 query rows per CTA (4 warps x 16 rows); one thread streams 64-key K/V tiles by
-// TMA into two 128-byte-swizzled stages; S = Q K^T and O += P V on mma.sync m16n8k16 with bf16
-// operands and fp32 accumulators, P kept in registers; two CTAs fit on an SM. The splits of one
-// (sequence, head, query tile) form a thread-block cluster (up to 16 CTAs) and merge their
-// partial results (O / l in fp16) through distributed shared memory, so the whole attention is
-// one launch and no partial goes through HBM.
+// In both bf16 kernels the splits of one (sequence, head, query tile) form a thread-block
+// cluster (up to 16 CTAs) and merge their partial results (O / l in fp16) through distributed
+// shared memory, so the whole attention is one launch and no partial goes through HBM.
+// bf16, tcgen05 (attn_tc_kernel, the default; details at its definition): 128 query rows per
+// CTA as the UMMA M, 64-key K/V tiles streamed by TMA, S = Q K^T and O += P V on the fifth-
+// generation tensor cores with S and O in TMEM, two softmax warpgroups on alternate tiles, one
+// CTA per SM.
+// bf16, mma.sync (attn_mma_kernel, DFLARE_FLAG_MMA_SYNC_ATTENTION): 64 query rows per CTA (4 warps
+// x 16 rows); one thread streams 64-key K/V tiles by TMA into two 128-byte-swizzled stages;
+// S = Q K^T and O += P V on mma.sync m16n8k16 with bf16 operands and fp32 accumulators, P kept in
+// registers; two to four CTAs fit on an SM.
 // fp32 path: a CUDA-core version of the split with partials in global memory and a second
 // (combine) launch; exact fp32 products.
 #include <cuda_fp16.h>
@@ -73,7 +78,7 @@ __device__ __forceinline__ size_t part_index(const AttnArgs& a, int b, int g, in
     return (((size_t)b * a.hkv + g) * a.q_tiles + qt) * a.splits + s;
 }
 
-// ------------------------------------------------------------------ bf16, tensor cores
+// ------------------------------------------------------------------ bf16, mma.sync (warp-level tensor cores)
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
@@ -581,8 +586,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ A
 // trip of four MMAs takes about 740 cycles, and one thread issuing both kinds, on a sub-partition
 // shared with two softmax warps, took 0.3-0.45 us per hand-off; the issuing warps sit on the
 // sub-partitions that the 64-row (Qwen3-shaped) tiles leave free of softmax work.
-// Every hand-off is an mbarrier with a bounded wait; the splits merge through the cluster as in
-// the mma.sync kernel.
+// Every hand-off is an mbarrier with a bounded wait. The cluster may hold any number of splits
+// from 1 to 16 (at one CTA per SM, the largest size whose clusters all fit at once); after the key
+// loop and a cluster barrier each CTA pushes its combined partial of every query row into the
+// (then idle) K/V stages of the CTA that merges that row.
 constexpr int kTQ = 128;            // query rows per CTA (UMMA M)
 constexpr int kTThreads = 384;      // warps 0-3, 4-7: softmax groups; 8: TMA; 9: TMEM; 10, 11: MMA
 constexpr float kRescale = 8.0f;    // growth (log2) of a row maximum that triggers a rescale
