@@ -597,20 +597,28 @@ constexpr float kRescale = 8.0f;    // growth (log2) of a row maximum that trigg
 constexpr int kMaxSplits = 16;     // cluster size limit (non-portable above 8)
 template <int HD>
 struct TcAttnLayout {
-    static constexpr int NS = HD == 128 ? 5 : 10;              // K/V stages
+    static constexpr int NS = HD == 128 ? 4 : 10;              // 64-key K and V slots (even)
     static constexpr uint32_t TB = HD * 128;                    // one 64-key K or V tile
+    static constexpr uint32_t KR = 0;                           // K ring [HD/64][NS][64 rows][128 B]
+    static constexpr uint32_t VR = NS * TB;                     // V ring [NS][HD/64][64 rows][128 B]
     static constexpr uint32_t Q = NS * 2 * TB;                  // Q [HD/64][128 rows][128 B]
     static constexpr uint32_t P = Q + (uint32_t)kTQ * HD * 2;   // P [group][128 rows][64 keys] bf16
     static constexpr uint32_t BARS = P + 2u * kTQ * 128;        // mbarriers, then two words
-    static constexpr int NBARS = 2 * NS + 10;
+    static constexpr int NBARS = 4 * NS + 10;
     static constexpr uint32_t BYTES = BARS + NBARS * 8 + 16;
+    // head_dim 128: S of two adjacent 64-key tiles in one N 128 MMA chain (half the S MMAs; the
+    // kernel is tensor-bound there); head_dim 64: S per tile (its S MMAs are cheap and the softmax
+    // groups overlap better when they alternate than when they work on a pair in lockstep)
+    static constexpr bool PAIR = HD == 128;
+    static constexpr int W = PAIR ? 2 : 1;                      // 64-key tiles per S unit
+    static_assert(NS % 2 == 0, "pairs of adjacent K slots form one N 128 operand");
     // After the key loop the (then idle) stages hold the cluster merge: the pushed partials O / l
     // in fp16 [S RP <= 128 + 15 rows][HD], their (m, l) and the merge weights [RP][S].
     static constexpr int MR = kTQ + kMaxSplits;
     static constexpr uint32_t RO = 0;
     static constexpr uint32_t RML = (uint32_t)MR * HD * 2;
     static constexpr uint32_t RW = RML + (uint32_t)MR * 8;
-    static constexpr uint32_t TMEM_COLS = 512;                  // S_A, S_B (64 each), O_A, O_B
+    static constexpr uint32_t TMEM_COLS = 512;                  // S of two tile pairs (128 each), O_A, O_B
     static_assert(RW + (uint32_t)MR * kMaxSplits * 4 <= NS * 2 * TB, "merge buffers exceed the stages");
     static_assert(1024 + BYTES <= 232448, "tcgen05 attention exceeds 227 KB of shared memory");
 };
@@ -627,15 +635,28 @@ __device__ __forceinline__ void ta_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                  : "memory");
 }
+// try_wait with a suspend-time hint: the thread sleeps until the phase completes or the hint
+// (ns) elapses instead of spinning, which leaves its sub-partition's issue slots to the softmax
+// warps there
+__device__ __forceinline__ bool try_wait_parity_sleep(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(100000u)
+        : "memory");
+    return ok != 0;
+}
 // Bounded wait for the phase of `bar` with parity `parity`: false after kWaitNs (which sets the
 // CTA's abort flag and the device error) or once another thread of the CTA has aborted. The timer
-// is read only after 64 unsuccessful polls (as in tile_wait).
+// is read only when the first (sleeping) poll has not seen the phase complete.
 __device__ __noinline__ bool ta_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                           uint32_t* err) {
     const uint64_t t0 = globaltimer_ns();
     while (true) {
-        for (int i = 0; i < 64; ++i)
-            if (try_wait_parity(bar, parity)) return true;
+        if (try_wait_parity_sleep(bar, parity)) return true;
         if (*abort_flag) return false;
         if (globaltimer_ns() - t0 > kWaitNs) {
             *abort_flag = 1;
@@ -646,8 +667,7 @@ __device__ __noinline__ bool ta_wait_slow(uint32_t bar, uint32_t parity, volatil
 }
 __device__ __forceinline__ bool ta_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                         uint32_t* err) {
-    for (int i = 0; i < 64; ++i)
-        if (try_wait_parity(bar, parity)) return true;
+    if (try_wait_parity_sleep(bar, parity)) return true;
     return ta_wait_slow(bar, parity, abort_flag, err);
 }
 __device__ __forceinline__ void ta_fence_before() {
@@ -730,16 +750,20 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
     uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_addr(smem);
     const uint32_t bar0 = sbase + LY::BARS;
-    // full[NS] (tile landed), empty[NS] (its P V completed); per softmax group q: sfull[q] (S of
-    // the group's tile in TMEM), sfree[q] (read by the group's 4 warps), pready[q] (its P
-    // written), odone[q] (its P V completed); one drain barrier per MMA-issuing thread
-    auto full_bar = [&](int st) { return bar0 + 8u * st; };
-    auto empty_bar = [&](int st) { return bar0 + 8u * (NS + st); };
-    auto sfull_bar = [&](int q) { return bar0 + 8u * (2 * NS + q); };
-    auto sfree_bar = [&](int q) { return bar0 + 8u * (2 * NS + 2 + q); };
-    auto pready_bar = [&](int q) { return bar0 + 8u * (2 * NS + 4 + q); };
-    auto odone_bar = [&](int q) { return bar0 + 8u * (2 * NS + 6 + q); };
-    auto drain_bar = [&](int i) { return bar0 + 8u * (2 * NS + 8 + i); };
+    // kfull / vfull[NS] (the slot's K / V tile landed), kempty[NS] (the S that read it completed),
+    // vempty[NS] (its P V completed); per S buffer i (S units u with u % 2 = i; a unit is a tile
+    // pair at head_dim 128, a tile at 64): sfull[i] (S of the unit in TMEM), sfree[i] (read by the
+    // softmax warps of the unit: 8 for a pair, 4 for a tile); per softmax group q: pready[q] (its P
+    // written), odone[q] (its P V completed); one drain per MMA-issuing thread
+    auto kfull_bar = [&](int st) { return bar0 + 8u * st; };
+    auto kempty_bar = [&](int st) { return bar0 + 8u * (NS + st); };
+    auto vfull_bar = [&](int st) { return bar0 + 8u * (2 * NS + st); };
+    auto vempty_bar = [&](int st) { return bar0 + 8u * (3 * NS + st); };
+    auto sfull_bar = [&](int i) { return bar0 + 8u * (4 * NS + i); };
+    auto sfree_bar = [&](int i) { return bar0 + 8u * (4 * NS + 2 + i); };
+    auto pready_bar = [&](int q) { return bar0 + 8u * (4 * NS + 4 + q); };
+    auto odone_bar = [&](int q) { return bar0 + 8u * (4 * NS + 6 + q); };
+    auto drain_bar = [&](int i) { return bar0 + 8u * (4 * NS + 8 + i); };
     uint32_t* misc = reinterpret_cast<uint32_t*>(smem + LY::BARS + LY::NBARS * 8);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(&misc[1]);
     cg::cluster_group cluster = cg::this_cluster();
@@ -756,19 +780,21 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         for (int k = tid; k < NS * (HD / 64) * zr * 8; k += blockDim.x) {
             const int piece = k & 7, r = a.block_rows + (k >> 3) % zr, sub = (k >> 3) / zr;
             const int st = sub / (HD / 64), h = sub % (HD / 64);
-            *reinterpret_cast<uint4*>(smem + (size_t)st * 2 * TB + TB + h * 8192 + r * 128 + piece * 16) =
+            *reinterpret_cast<uint4*>(smem + LY::VR + (size_t)st * TB + h * 8192 + r * 128 + piece * 16) =
                 make_uint4(0u, 0u, 0u, 0u);
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     if (tid == 0) {
         for (int i = 0; i < NS; ++i) {
-            ta_mbar_init(full_bar(i), 1);
-            ta_mbar_init(empty_bar(i), 1);
+            ta_mbar_init(kfull_bar(i), 1);
+            ta_mbar_init(kempty_bar(i), 1);
+            ta_mbar_init(vfull_bar(i), 1);
+            ta_mbar_init(vempty_bar(i), 1);
         }
         for (int q = 0; q < 2; ++q) {
             ta_mbar_init(sfull_bar(q), 1);
-            ta_mbar_init(sfree_bar(q), 4);
+            ta_mbar_init(sfree_bar(q), LY::PAIR ? 8 : 4);
             ta_mbar_init(pready_bar(q), 4);
             ta_mbar_init(odone_bar(q), 1);
         }
@@ -801,27 +827,27 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
     const int t0 = s * (T / S) + min(s, T % S);
     const int n_tiles = T / S + (s < T % S ? 1 : 0);
     const int n_ct = max(0, min(t0 + n_tiles, n_ctx_tiles) - t0);
-    // tile t -> stage t % NS: K at [stage][0, TB), V at [stage][TB, 2 TB)
-    auto issue = [&](int t) {
+    constexpr int W = LY::W;
+    const int n_units = (n_tiles + W - 1) / W;   // S units: tiles W u .. W u + W - 1
+    // 64-key tile t -> slot t % NS: K atom h at KR + (h NS + slot) 8192 (two adjacent slots of an
+    // atom are one 128-row operand), V at VR + slot TB + h 8192
+    auto issue = [&](int t, bool v) {
         const int st = t % NS;
-        const uint32_t kdst = sbase + (uint32_t)st * 2 * TB, bar = full_bar(st);
-        const uint32_t bytes = t < n_ct ? 2 * TB : 2u * (HD / 64) * (uint32_t)a.block_rows * 128u;
-        ta_expect_tx(bar, bytes);
+        const uint32_t bar = v ? vfull_bar(st) : kfull_bar(st);
+        ta_expect_tx(bar, t < n_ct ? TB : (HD / 64) * (uint32_t)a.block_rows * 128u);
         for (int h = 0; h < HD / 64; ++h) {
-            if (t < n_ct) {
-                const int y = (t0 + t) * kKT, z = b * a.hkv + g;
-                tma_tile(kdst + h * 8192, &maps.kc, h * 64, y, z, bar);
-                tma_tile(kdst + TB + h * 8192, &maps.vc, h * 64, y, z, bar);
-            } else {
-                tma_tile(kdst + h * 8192, &maps.kd, h * 64, b * a.B, g, bar);
-                tma_tile(kdst + TB + h * 8192, &maps.vd, h * 64, b * a.B, g, bar);
-            }
+            const uint32_t dst = v ? sbase + LY::VR + (uint32_t)st * TB + h * 8192u
+                                   : sbase + LY::KR + (uint32_t)(h * NS + st) * 8192u;
+            if (t < n_ct)
+                tma_tile(dst, v ? &maps.vc : &maps.kc, h * 64, (t0 + t) * kKT, b * a.hkv + g, bar);
+            else
+                tma_tile(dst, v ? &maps.vd : &maps.kd, h * 64, b * a.B, g, bar);
         }
     };
-    int issued = 0;   // warp 8, lane 0
+    int issued = 0;   // warps 8 (K) and 9 (V), lane 0
     // the first context tiles stream in while the projection drains; the block tile waits
-    if (warp == 8 && lane == 0)
-        for (; issued < min(NS, n_ct); ++issued) issue(issued);
+    if ((warp == 8 || warp == 9) && lane == 0)
+        for (; issued < min(NS, n_ct); ++issued) issue(issued, warp == 9);
     pdl_wait();
     if (a.t_stamps && tid == 0) atomicMin(a.t_stamps + a.t_slots, (unsigned long long)globaltimer_ns());
     const int n32 = a.d_q + 2 * a.d_kv;
@@ -914,52 +940,59 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
     }
     __syncthreads();
 
-    // instruction descriptors: fp32 accumulator, bf16 A and B, M 128; S: N 64, both K-major;
-    // P V: N = HD, B (V) MN-major
-    constexpr uint32_t kIdS = (1u << 4) | (1u << 7) | (1u << 10) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
-    constexpr uint32_t kIdO = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | (((uint32_t)HD >> 3) << 17) |
-                              ((128u >> 4) << 24);
-    // TMEM columns: S of group q at [64 q, 64 q + 64), O of group q at [128 + 128 q, + HD)
-    auto tS = [&](int q) { return tmem + 64u * q; };
-    auto tO = [&](int q) { return tmem + 128u + 128u * q; };
+    // instruction descriptors: fp32 accumulator, bf16 A and B, M 128; S: N 64 per tile of the unit
+    // (128 for a pair), both K-major; P V: N = HD, B (V) MN-major
+    constexpr uint32_t kIdBase = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 4) << 24);
+    constexpr uint32_t kIdS2 = kIdBase | ((128u >> 3) << 17), kIdS1 = kIdBase | ((64u >> 3) << 17);
+    constexpr uint32_t kIdO = kIdBase | (1u << 16) | (((uint32_t)HD >> 3) << 17);
+    // TMEM columns: S of unit u at [128 (u % 2), + 64 W) (tile W u + h in columns 64 h + ...), O of
+    // softmax group q at [256 + HD q, + HD)
+    auto tS = [&](int i) { return tmem + 128u * i; };
+    auto tO = [&](int q) { return tmem + 256u + (uint32_t)HD * q; };
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
 
-    if (warp == 8) {
+    if (warp == 8 || warp == 9) {
         if (lane == 0) {
-            // ---------------- TMA producer: the stage of tile t is refilled once P V of tile
-            // t - NS has completed
+            // ---------------- TMA producers, warp 8 for K and warp 9 for V: the slot of tile t is
+            // refilled once the S (K) or the P V (V) of tile t - NS has completed
+            const bool v = warp == 9;
             for (; issued < n_tiles; ++issued) {
                 const int st = issued % NS;
-                if (issued >= NS && !(ok = ta_wait(empty_bar(st), (uint32_t)(issued / NS - 1) & 1u, abort_flag, a.err)))
+                if (issued >= NS && !(ok = ta_wait(v ? vempty_bar(st) : kempty_bar(st), (uint32_t)(issued / NS - 1) & 1u,
+                                                   abort_flag, a.err)))
                     break;
-                issue(issued);
+                issue(issued, v);
             }
-            // after an abort, the copies in flight land before the shared memory is released
+            // after an abort, the copies in flight land before the shared memory is reused
             if (!ok) {
                 volatile int never = 0;
                 for (int t = max(0, issued - NS); t < issued; ++t)
-                    ta_wait(full_bar(t % NS), (uint32_t)(t / NS) & 1u, &never, a.err);
+                    ta_wait(v ? vfull_bar(t % NS) : kfull_bar(t % NS), (uint32_t)(t / NS) & 1u, &never, a.err);
             }
         }
         __syncwarp();
     } else if (warp == 10) {
         if (lane == 0 && n_tiles > 0) {
-            // ---------------- S issue (one thread): S_t into the S buffer of group t & 1 once
-            // the tile has landed and the group has read S_{t-2}; descriptors advance by
+            // ---------------- S issue (one thread): S of unit u into S buffer u % 2 once its K tiles
+            // have landed and the softmax warps have read unit u - 2; descriptors advance by
             // address >> 4
             const uint64_t dQ = ta_desc_k(sbase + LY::Q);
-            for (int t = 0; t < n_tiles && ok; ++t) {
-                const int st = t % NS, q = t & 1;
-                if (!(ok = ta_wait(full_bar(st), (uint32_t)(t / NS) & 1u, abort_flag, a.err))) break;
-                if (t >= 2 && !(ok = ta_wait(sfree_bar(q), (uint32_t)((t >> 1) - 1) & 1u, abort_flag, a.err))) break;
+            for (int p = 0; p < n_units && ok; ++p) {
+                const int ta = W * p, i = p & 1, nsub = min(W, n_tiles - ta);
+                for (int h = 0; h < nsub && ok; ++h)
+                    ok = ta_wait(kfull_bar((ta + h) % NS), (uint32_t)((ta + h) / NS) & 1u, abort_flag, a.err);
+                if (!ok) break;
+                if (p >= 2 && !(ok = ta_wait(sfree_bar(i), (uint32_t)((p >> 1) - 1) & 1u, abort_flag, a.err))) break;
                 ta_fence_after();
-                const uint64_t dK = ta_desc_k(sbase + (uint32_t)st * 2 * TB);
+                const uint64_t dK = ta_desc_k(sbase + LY::KR + (uint32_t)(ta % NS) * 8192u);
+                const uint32_t id = nsub == 2 ? kIdS2 : kIdS1;
 #pragma unroll
                 for (int kk = 0; kk < HD / 16; ++kk)
-                    ta_mma(tS(q), dQ + (uint64_t)((kk >> 2) * (kTQ * 128 / 16) + (kk & 3) * 2),
-                           dK + (uint64_t)((kk >> 2) * (8192 / 16) + (kk & 3) * 2), kIdS, kk > 0 ? 1u : 0u);
-                ta_commit(sfull_bar(q));
+                    ta_mma(tS(i), dQ + (uint64_t)((kk >> 2) * (kTQ * 128 / 16) + (kk & 3) * 2),
+                           dK + (uint64_t)((kk >> 2) * (NS * 8192 / 16) + (kk & 3) * 2), id, kk > 0 ? 1u : 0u);
+                ta_commit(sfull_bar(i));
+                for (int h = 0; h < nsub; ++h) ta_commit(kempty_bar((ta + h) % NS));
             }
             // every MMA this thread issued has completed before the tensor memory is released
             ta_commit(drain_bar(0));
@@ -969,34 +1002,33 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         __syncwarp();
     } else if (warp == 11) {
         if (lane == 0 && n_tiles > 0) {
-            // ---------------- P V issue (one thread): O_q += P_t V_t once group q = t & 1 has
-            // written P_t (S_t, which read the stage's K, completed before that); the stage is
-            // released when this P V completes
+            // ---------------- P V issue (one thread): O_q += P_t V_t once the V tile has landed and
+            // group q = t & 1 has written P_t; the V slot is released when this P V completes
             const uint64_t dP = ta_desc_k(sbase + LY::P);
             for (int t = 0; t < n_tiles && ok; ++t) {
                 const int st = t % NS, q = t & 1;
+                if (!(ok = ta_wait(vfull_bar(st), (uint32_t)(t / NS) & 1u, abort_flag, a.err))) break;
                 if (!(ok = ta_wait(pready_bar(q), (uint32_t)(t >> 1) & 1u, abort_flag, a.err))) break;
                 ta_fence_after();
-                const uint64_t dV = ta_desc_mn(sbase + (uint32_t)st * 2 * TB + TB);
+                const uint64_t dV = ta_desc_mn(sbase + LY::VR + (uint32_t)st * TB);
                 const uint64_t dPq = dP + (uint64_t)(q * (kTQ * 128 / 16));
 #pragma unroll
                 for (int kk = 0; kk < kKT / 16; ++kk)
                     ta_mma(tO(q), dPq + (uint64_t)(kk * 2), dV + (uint64_t)(kk * 128), kIdO,
                            (t >= 2 || kk > 0) ? 1u : 0u);
                 ta_commit(odone_bar(q));
-                ta_commit(empty_bar(st));
+                ta_commit(vempty_bar(st));
             }
             ta_commit(drain_bar(1));
             volatile int never = 0;
             ta_wait(drain_bar(1), 0, &never, a.err);
         }
         __syncwarp();
-    } else if (warp >= 8) {
-        // warp 9 holds the tensor memory allocation only
     } else {
-        // ---------------- softmax group q (warps 4q .. 4q + 3) takes tiles q, q + 2, ...; thread
-        // = query row tid % 128 = TMEM lane. Every wait is taken by the whole warp and its
-        // outcome made warp-uniform (the tcgen05 loads and stores below are warp-collective).
+        // ---------------- softmax group q (warps 4q .. 4q + 3) takes tiles q, q + 2, ... (at head_dim
+        // 128 the half q of every tile pair); thread = query row tid % 128 = TMEM lane. Every wait is
+        // taken by the whole warp and its outcome made warp-uniform (the tcgen05 loads and stores
+        // below are warp-collective).
         const int q = warp >> 2, row = tid & 127;
         const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
         const bool warp_rows = qt * kTQ + (warp & 3) * 32 < R;   // the warp holds a query row
@@ -1006,16 +1038,18 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         };
         uint8_t* const prow = smem + LY::P + (uint32_t)q * (kTQ * 128) + row * 128;
         for (int t = q; t < n_tiles && ok; t += 2) {
-            if (!(ok = wwait(sfull_bar(q), (uint32_t)(t >> 1) & 1u))) break;
+            const int p = t / W, i = p & 1;
+            const uint32_t col = 64u * (uint32_t)(t - W * p);
+            if (!(ok = wwait(sfull_bar(i), (uint32_t)(p >> 1) & 1u))) break;
             ta_fence_after();
             float sv[64];
             if (warp_rows) {
-                ta_ld32(tS(q) + lane_base, sv);
-                ta_ld32(tS(q) + lane_base + 32, sv + 32);
+                ta_ld32(tS(i) + lane_base + col, sv);
+                ta_ld32(tS(i) + lane_base + col + 32, sv + 32);
             }
             ta_fence_before();
             __syncwarp();
-            if (lane == 0) ta_arrive(sfree_bar(q));
+            if (lane == 0) ta_arrive(sfree_bar(i));
             // keys past the tile's valid count (ragged last tile, block tile) get -inf
             const int valid = t < n_ct ? min(kKT, L - (t0 + t) * kKT) : a.B;
             float mx = -INFINITY;
