@@ -1119,46 +1119,54 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
         const int last = q + ((n_tiles - 1 - q) >> 1) * 2;   // the group's last tile
         if (ok && n_tiles > q) ok = wwait(odone_bar(q), (uint32_t)(last >> 1) & 1u);
         ta_fence_after();
-        // group 1 leaves its (m, l) for group 0 in its own (now unused) P buffer
-        if (q == 1) {
-            float2* xml = reinterpret_cast<float2*>(smem + LY::P + kTQ * 128);
-            xml[row] = make_float2(n_tiles > 1 && ok ? m_used : -INFINITY, n_tiles > 1 && ok ? l : 0.f);
-        }
+        // each group leaves its (m, l) per row in its own (now unused) P buffer for the push
+        float2* xml = reinterpret_cast<float2*>(smem + LY::P + (uint32_t)q * (kTQ * 128));
+        xml[row] = make_float2(n_tiles > q && ok ? m_used : -INFINITY, n_tiles > q && ok ? l : 0.f);
     }
     if (!ok && lane == 0) atomicOr(a.err, DFLARE_DEVERR_TIMEOUT);
     // every CTA of the cluster has finished with its stages (copies landed, MMAs drained) before
     // any partial is pushed into them
     __syncthreads();
     cluster.sync();
-    // Push the partial: group 0 combines both groups' (m, l, O) of query row r and writes it to
-    // CTA r / RP at [s RP + r % RP]. ok is warp-uniform, so the tcgen05 loads stay collective; a
-    // group without tiles (m = -inf) contributes nothing and its O is not read.
+    // Push the partial: both groups' (m, l, O) of query row r are combined and written to CTA
+    // r / RP at [s RP + r % RP]; warpgroup h (warps 4h .. 4h + 3, lane quarter = warp % 4) takes the
+    // head dims [h HD/2, h HD/2 + HD/2). A group without tiles (m = -inf) contributes nothing and
+    // its O is not read; the loads are guarded by warp votes, so they stay collective.
     const int RP = (rows + S - 1) / S;
     __half* rO = reinterpret_cast<__half*>(smem + LY::RO);
     float2* rML = reinterpret_cast<float2*>(smem + LY::RML);
     float* rW = reinterpret_cast<float*>(smem + LY::RW);
-    if (warp < 4 && warp * 32 < rows) {
-        const int r = tid;
+    if (warp < 8 && (warp & 3) * 32 < rows) {
+        const int r = tid & 127, half = warp >> 2;
         const bool row_ok = r < rows;
+        const float2 mlA = reinterpret_cast<const float2*>(smem + LY::P)[r];
         const float2 mlB = reinterpret_cast<const float2*>(smem + LY::P + kTQ * 128)[r];
-        const bool hA = ok && n_tiles > 0, hB = hA && mlB.x != -INFINITY;
-        const float mA = hA ? m_used : -INFINITY;
-        const float M = fmaxf(mA, mlB.x);
-        const float wA = hA ? ex2(mA - M) : 0.f, wB = hB ? ex2(mlB.x - M) : 0.f;
-        const float lt = (hA ? l * wA : 0.f) + (hB ? mlB.y * wB : 0.f);
+        const bool hA = mlA.x != -INFINITY, hB = mlB.x != -INFINITY;
+        const float M = fmaxf(mlA.x, mlB.x);
+        const float wA = hA ? ex2(mlA.x - M) : 0.f, wB = hB ? ex2(mlB.x - M) : 0.f;
+        const float lt = (hA ? mlA.y * wA : 0.f) + (hB ? mlB.y * wB : 0.f);
         const float inv = lt > 0.f ? 1.0f / lt : 0.f;
         const float cA = wA * inv, cB = wB * inv;
         const int dst_cta = row_ok ? r / RP : 0, dst_row = s * RP + (row_ok ? r % RP : 0);
         __half* dst = cluster.map_shared_rank(rO, dst_cta) + (size_t)dst_row * HD;
-        const uint32_t lb = (uint32_t)(warp * 32) << 16;
-        if (hA) {
+        const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+        const bool anyA = __any_sync(0xffffffffu, hA), anyB = __any_sync(0xffffffffu, hB);
+        if (anyA || anyB) {
 #pragma unroll
-            for (int c = 0; c < HD / 32; ++c) {
+            for (int c = half * (HD / 64); c < (half + 1) * (HD / 64); ++c) {
                 float ov[32], ob[32];
-                ta_ld32(tO(0) + lb + c * 32, ov);
-                if (__any_sync(0xffffffffu, hB)) ta_ld32(tO(1) + lb + c * 32, ob);
+                if (anyA) {
+                    ta_ld32(tO(0) + lb + c * 32, ov);
+                } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) ov[i] = hB ? fmaf(ob[i], cB, ov[i] * cA) : ov[i] * cA;
+                    for (int i = 0; i < 32; ++i) ov[i] = 0.f;
+                }
+                if (anyB) ta_ld32(tO(1) + lb + c * 32, ob);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float x = hA ? ov[i] * cA : 0.f;
+                    ov[i] = hB ? fmaf(ob[i], cB, x) : x;
+                }
                 if (row_ok) {
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
@@ -1171,7 +1179,8 @@ __global__ void __launch_bounds__(kTThreads, 1) attn_tc_kernel(const __grid_cons
                 }
             }
         }
-        if (row_ok) *cluster.map_shared_rank(rML + dst_row, dst_cta) = make_float2(hA ? M : -INFINITY, lt);
+        if (row_ok && half == 0)
+            *cluster.map_shared_rank(rML + dst_row, dst_cta) = make_float2(hA || hB ? M : -INFINITY, lt);
     }
     // every partial has arrived; after this barrier no CTA touches another's shared memory
     ta_fence_before();
