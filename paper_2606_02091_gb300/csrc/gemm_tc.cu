@@ -42,11 +42,15 @@ constexpr int kMaxStages = 8;
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 constexpr int kSmemLimit = 227 * 1024;
 constexpr uint32_t kABytes = kBM * kBK * 2;   // one 128 x 64 bf16 weight tile
+constexpr int kMaxTokList = 1024;             // token tiles a compacted launch can list
 
 struct TcArgs {
     CUtensorMap map_a, map_a2, map_b;   // weights, up weights (SwiGLU), activations
     int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks;
     int bn, n_a, stages, n_bufs, tmem_cols;
+    int pair;                  // 1: a unit is two adjacent 128-row tiles of one weight matrix
+                               // (the second accumulator takes rows 128..255 of the pair)
+    int compact;               // EPI_KV_APPEND: skip the token tiles that hold no appended row
     int kbs;                   // 64-wide k-blocks per pipeline stage
     uint32_t b_bytes;          // bytes of one activation sub-tile (bn x 64 bf16)
     int evict_first;           // stream the weights with an L2 evict-first policy
@@ -172,8 +176,9 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
 // The kernel's loop constants, copied out of the parameter block into registers (the block is
 // addressed for the tensor maps, so every asm with a memory clobber would otherwise reload them).
 struct Geom {
-    int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks, n_a, kbs, bn, n_bufs;
+    int n_units, n_tiles, tok_tiles, splits, kb_per_split, k_blocks, n_a, kbs, bn, n_bufs, pair;
     uint32_t b_bytes, stage_bytes, idesc;
+    const int* tok_list;       // token tiles in unit order (compacted launches), else nullptr
 };
 struct Unit {
     int group, n_tile, tok_tile, split, tile_id, kb0, kb1;
@@ -184,6 +189,7 @@ __device__ __forceinline__ Unit decode_unit(const Geom& a, int u) {
     x.tile_id = u / a.splits;
     int t = x.tile_id;
     x.tok_tile = t % a.tok_tiles;
+    if (a.tok_list) x.tok_tile = a.tok_list[x.tok_tile];
     t /= a.tok_tiles;
     x.n_tile = t % a.n_tiles;
     x.group = t / a.n_tiles;
@@ -232,6 +238,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     G.kbs = args.kbs;
     G.bn = args.bn;
     G.n_bufs = args.n_bufs;
+    G.pair = args.pair;
+    G.tok_list = nullptr;
     G.b_bytes = args.b_bytes;
     G.stage_bytes = args.stage_bytes;
     G.idesc = args.idesc;
@@ -271,6 +279,31 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
+    // Compacted launch (a context fill of sequences with different lengths, token row
+    // b * n_max + r): after the dependency wait, warp 0 lists the token tiles that hold at least
+    // one appended row (r < app_cnt[b]); units then run over the listed tiles only.
+    int* const tok_list = reinterpret_cast<int*>(misc + 4);
+    if (args.compact) {
+        pdl_wait();
+        if (tst && threadIdx.x == 0) atomicMin(tst + args.t_slots, (unsigned long long)globaltimer_ns());
+        if (warp == 0) {
+            const int nm = args.ep.n_max;
+            int cnt = 0;
+            for (int base = 0; base < args.tok_tiles; base += 32) {
+                const int tt = base + lane;
+                bool v = false;
+                if (tt < args.tok_tiles) {
+                    const int r0 = tt * G.bn, r1 = min(args.ep.m_tok, r0 + G.bn);
+                    for (int b = r0 / nm; b <= (r1 - 1) / nm && !v; ++b)
+                        v = args.ep.app_cnt[b] > max(0, r0 - b * nm);
+                }
+                const unsigned m = __ballot_sync(0xffffffffu, v);
+                if (v) tok_list[cnt + __popc(m & ((1u << lane) - 1u))] = tt;
+                cnt += __popc(m);
+            }
+            if (lane == 0) misc[3] = (uint32_t)cnt;
+        }
+    }
     if (warp == 5) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(&misc[0])),
@@ -283,6 +316,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     tc_fence_after();
     const uint32_t tmem = misc[0];
     volatile int* abort_flag = reinterpret_cast<volatile int*>(&misc[1]);
+    if (args.compact) {
+        G.n_units = args.n_units / args.tok_tiles * (int)misc[3];
+        G.tok_tiles = (int)misc[3];
+        G.tok_list = tok_list;
+    }
     const int acc_cols = G.n_a * G.bn;
 
     if (warp == 4) {
@@ -300,12 +338,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
             const uint32_t b_base = kABytes * G.n_a * G.kbs;
             const uint32_t tx = kABytes * G.n_a + G.b_bytes;
+            // first weight row of a unit in both maps (a pair's second map starts 128 rows in)
+            const int row_step = kBM << G.pair;
             // Weights do not depend on the previous kernel: the first ring of stages gets its
             // weight tiles before griddepcontrol.wait, the activation tiles after it.
             int pend_kx[kMaxStages], pend_nk[kMaxStages], pend_tok[kMaxStages], pend_grp[kMaxStages];
             uint32_t pend_st[kMaxStages];
             int npend = 0;
-            bool waited = false;
+            bool waited = args.compact != 0;   // a compacted launch waited before the unit list
             auto load_b = [&](uint32_t st, int kx0, int nk, int tok_tile, int group, uint32_t bar) {
                 if constexpr (kAux) {
                     for (int j = 0; j < nk; ++j) {
@@ -334,15 +374,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     for (int j = 0; j < nk; ++j) {
                         const int kx = (kb + j) * kBK;
                         if (evict_first) {
-                            tma_load_3d_hint(st + j * kABytes, mA, kx, x.n_tile * kBM, x.group,
+                            tma_load_3d_hint(st + j * kABytes, mA, kx, x.n_tile * row_step, x.group,
                                              full_bar(stage), policy);
                             if (G.n_a == 2)
-                                tma_load_3d_hint(st + (G.kbs + j) * kABytes, mA2, kx, x.n_tile * kBM,
+                                tma_load_3d_hint(st + (G.kbs + j) * kABytes, mA2, kx, x.n_tile * row_step,
                                                  x.group, full_bar(stage), policy);
                         } else {
-                            tma_load_3d(st + j * kABytes, mA, kx, x.n_tile * kBM, x.group, full_bar(stage));
+                            tma_load_3d(st + j * kABytes, mA, kx, x.n_tile * row_step, x.group, full_bar(stage));
                             if (G.n_a == 2)
-                                tma_load_3d(st + (G.kbs + j) * kABytes, mA2, kx, x.n_tile * kBM, x.group,
+                                tma_load_3d(st + (G.kbs + j) * kABytes, mA2, kx, x.n_tile * row_step, x.group,
                                             full_bar(stage));
                         }
                     }
@@ -608,6 +648,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     epi_bar();
                     if (resid)
                         resid_epilogue(args.ep, epi, x.n_tile, x.tok_tile * bn + c0, t, rr);
+                    else if (G.pair)   // two 128-feature tiles, one per accumulator
+                        for (int a = 0; a < 2; ++a)
+                            apply_epilogue<bf16, kAux>(args.ep, epi + a * kChunk * 128, x.group,
+                                                       2 * x.n_tile + a, x.tok_tile * bn + c0, t);
                     else
                         apply_epilogue<bf16, kAux>(args.ep, epi, x.group, x.n_tile, x.tok_tile * bn + c0, t);
                     epi_bar();
@@ -688,10 +732,21 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     if (g.m_tok <= 0 || g.n <= 0) return cudaSuccess;
     TcArgs a;
     memset(&a, 0, sizeof(a));
-    a.n_a = g.a2 ? 2 : 1;
     a.bn = g.m_tok <= 256 ? ((g.m_tok + 15) / 16) * 16 : 256;
+    // With token tiles of 128 or more rows the GEMM is bound by the tensor pipeline, not by HBM:
+    // two adjacent 128-row weight tiles then share one activation tile (two accumulators, as the
+    // SwiGLU gate and up tiles do), a third fewer shared-memory bytes per FLOP (d 4096, 8 groups,
+    // 2048 tokens alone: 1197 -> 1316 TFLOP/s; batch-16 step 1.965 -> 1.947 ms). Only for the
+    // epilogues that finish a tile through the staged path, and only while the pairs still give
+    // every SM a unit.
+    a.pair = (!g.a2 && a.bn >= 128 && g.n > kBM && g.force_splits <= 0 &&
+              (g.ep.kind == EPI_STORE || g.ep.kind == EPI_F32 || g.ep.kind == EPI_QKV ||
+               g.ep.kind == EPI_KV_APPEND) &&
+              (long long)g.groups * ((g.n + 2 * kBM - 1) / (2 * kBM)) * ((g.m_tok + a.bn - 1) / a.bn) >=
+                  c->num_sms) ? 1 : 0;
+    a.n_a = (g.a2 || a.pair) ? 2 : 1;
     a.tok_tiles = (g.m_tok + a.bn - 1) / a.bn;
-    a.n_tiles = (g.n + kBM - 1) / kBM;
+    a.n_tiles = (g.n + (kBM << a.pair) - 1) / (kBM << a.pair);
     a.k_blocks = (g.k + kBK - 1) / kBK;
     const int tiles = g.groups * a.n_tiles * a.tok_tiles;
     const int sms = c->num_sms;
@@ -713,7 +768,11 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     // (512 contiguous bytes of every weight row; 128-byte rows per request leave DRAM bandwidth
     // unused), fewer when two stages do not fit.
     const int epi_bytes = a.n_a * kChunk * 128 * 4;
-    const int fixed = 1024 + epi_bytes + 8 * (2 * kMaxStages + 5) + 16;
+    // a context fill over several token tiles lists the tiles that hold appended rows (the
+    // sequences of one call can have very different lengths: rows past app_cnt are padding)
+    a.compact = (g.ep.kind == EPI_KV_APPEND && a.tok_tiles > 1 && a.tok_tiles <= kMaxTokList) ? 1 : 0;
+    const int misc_bytes = 16 + (a.compact ? 4 * kMaxTokList : 0);
+    const int fixed = 1024 + epi_bytes + 8 * (2 * kMaxStages + 5) + misc_bytes;
     const int budget = g.max_smem > 0 ? std::min(g.max_smem, kSmemLimit) : kSmemLimit;
     if (g.kbs > 0) {
         a.kbs = g.kbs;
@@ -741,7 +800,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         if (why) *why = "tcgen05 GEMM: tile does not fit in shared memory";
         return cudaErrorInvalidValue;
     }
-    const int smem = 1024 + a.stages * (int)a.stage_bytes + epi_bytes + 8 * (2 * a.stages + 5) + 16;
+    const int smem = 1024 + a.stages * (int)a.stage_bytes + epi_bytes + 8 * (2 * a.stages + 5) + misc_bytes;
     a.n_bufs = (2 * a.n_a * a.bn <= 512) ? 2 : 1;
     int cols = 32;
     while (cols < a.n_bufs * a.n_a * a.bn) cols <<= 1;
@@ -769,8 +828,11 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         if (why) *why = "tcgen05 GEMM: b_kgroup must be a multiple of 64 that divides k, with one group";
         return cudaErrorInvalidValue;
     }
+    // a pair's second tile: the same matrix from row 128 on (rows past its end read as zeros)
+    const void* a2 = g.a2 ? g.a2 : a.pair ? static_cast<const void*>(static_cast<const bf16*>(g.a) + (size_t)kBM * g.k)
+                                          : g.a;
     if (!make_map(&a.map_a, g.a, g.k, g.n, g.groups, a_gr, kBM) ||
-        !make_map(&a.map_a2, g.a2 ? g.a2 : g.a, g.k, g.n, g.groups, a_gr, kBM) ||
+        !make_map(&a.map_a2, a2, g.k, a.pair ? g.n - kBM : g.n, g.groups, a_gr, kBM) ||
         !make_map(&a.map_b, g.b, b_k, g.m_tok, b_groups, b_gr, a.bn)) {
         if (why) *why = "cuTensorMapEncodeTiled failed (alignment or driver entry point)";
         return cudaErrorInvalidValue;

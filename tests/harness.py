@@ -45,6 +45,29 @@ MULTI_TILE = synth.Workload(
 # degenerate and less common shapes: more draft layers than the fusion kernels hold at once
 # (D 10), 128 query rows per KV head (G 8: two 64-row query tiles), a single fused target layer
 # with block 1 (no mask rows: nothing is drafted), and block 2
+# A ragged context fill: one call fills 700, 3 and 40 positions, so 5 of the 9 256-row token
+# tiles of the context K/V projection hold no appended row (skipped); the LM head's 500 rows end
+# inside the first tile of its second 256-row weight pair.
+RAGGED = synth.Workload(
+    "ragged_fill_bf16",
+    synth.Shape(d=384, n_draft_layers=2, n_target_layers=3, n_q_heads=4, n_kv_heads=2,
+                head_dim=64, ffn=512, vocab=500, block=8),
+    (700, 3, 40), 0.8, seed=21)
+# A context fill long enough that the K/V projection pairs adjacent weight tiles over one token
+# tile (2 layers x 4 pairs x 32 token tiles >= the SM count) and skips the 11 token tiles past
+# the shorter sequence.
+LONG_FILL = synth.Workload(
+    "long_fill_bf16",
+    synth.Shape(d=256, n_draft_layers=2, n_target_layers=2, n_q_heads=8, n_kv_heads=4,
+                head_dim=128, ffn=256, vocab=300, block=4),
+    (4000, 1200), 0.8, seed=23)
+# 240 LM-head rows (batch 16 x 15 mask positions) over a vocabulary of 157 weight-tile pairs: the
+# LM head pairs its tiles, and the last pair's second tile lies past the matrix.
+WIDE_VOCAB = synth.Workload(
+    "wide_vocab_bf16_b16",
+    synth.Shape(d=256, n_draft_layers=1, n_target_layers=1, n_q_heads=4, n_kv_heads=2,
+                head_dim=64, ffn=256, vocab=40000, block=16),
+    tuple(5 + (13 * b) % 29 for b in range(16)), 0.8, seed=25)
 D10 = synth.Workload(
     "d10_bf16",
     synth.Shape(d=256, n_draft_layers=10, n_target_layers=2, n_q_heads=4, n_kv_heads=2,

@@ -15,14 +15,14 @@ import pytest
 
 import oracle as O
 import synth
-from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, MULTI_TILE, QT2, SMALL_HD128, SMALL_HD64, TINY,
-                           WIDE_B16,
+from tests.harness import (BLOCK1, BLOCK2, BLOCK32, D10, G8, LONG_FILL, MULTI_TILE, QT2, RAGGED, SMALL_HD128,
+                           SMALL_HD64, TINY, WIDE_B16, WIDE_VOCAB,
                            GpuSide, check_elem, check_kv, check_rows, check_tokens, f64, oracle_for,
                            rel_err, tolerance, verified_steps)
 
 pytestmark = pytest.mark.gpu
 GAP = 1e-2
-WORKLOADS = [TINY, SMALL_HD128, SMALL_HD64, D10, G8, BLOCK1, BLOCK2]
+WORKLOADS = [TINY, SMALL_HD128, SMALL_HD64, D10, G8, BLOCK1, BLOCK2, RAGGED, LONG_FILL]
 
 
 @pytest.fixture(scope="module", params=WORKLOADS, ids=lambda w: w.name)
@@ -179,11 +179,11 @@ def test_attention_kernels_match_oracle(w, kernel):
     assert g.lib.device_error() == 0
 
 
-@pytest.mark.parametrize("w", [WIDE_B16, BLOCK32, MULTI_TILE], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [WIDE_B16, BLOCK32, MULTI_TILE, WIDE_VOCAB], ids=lambda w: w.name)
 def test_wide_token_tiles_match_oracle(w):
-    """256 token rows per projection (batch 16, the widest tcgen05 token tile), block 32, and 288
-    rows (two token tiles, the second ragged): fused context, cached K/V and the draft block
-    against the oracle."""
+    """256 token rows per projection (batch 16, the widest tcgen05 token tile), block 32, 288
+    rows (two token tiles, the second ragged), and a 240-row LM head over paired weight tiles:
+    fused context, cached K/V and the draft block against the oracle."""
     g = GpuSide(w)
     o = oracle_for(w, g.W)
     fused = f64(g.fuse(w.ctx_lens))

@@ -5,14 +5,16 @@ decisions; a decision is compared exactly unless the oracle's float64 evaluation
 the fp32 rounding margin (a top-2 gap of the Gumbel scores, or r q - p for an acceptance, below
 1e-4 relative). The draft logits handed to the oracle's verification are the GPU's own (read back
 through logits_out), the same input the GPU's verification reads; the logits themselves are
-compared with the oracle's by the parity tests. A Monte Carlo test checks the property that
-defines the rule: the first token a step emits follows the target's distribution."""
+compared with the oracle's by the parity tests. test_sampled_step_end_to_end instead lets the oracle
+take every decision of a step from its own logits (with margins for the logit difference between
+the two sides). A Monte Carlo test checks the property that defines the rule: the first token a
+step emits follows the target's distribution."""
 import numpy as np
 import pytest
 
 import oracle as O
 import synth
-from tests.harness import SMALL_HD128, TINY, WIDE_B16, GpuSide
+from tests.harness import SMALL_HD128, TINY, WIDE_B16, GpuSide, oracle_for
 
 pytestmark = pytest.mark.gpu
 MARGIN = 1e-4
@@ -134,6 +136,106 @@ def test_sampled_verification_matches_oracle(w):
                 ok = sc[t_g] + slack[t_g] >= sc[t_o] - slack[t_o]
             assert ok, (rnd, b, int(nxt_h[b]), int(nxt_o))
         assert g.lib.device_error() == 0
+
+
+@pytest.mark.parametrize("w", [TINY, SMALL_HD128], ids=lambda w: w.name)
+def test_sampled_step_end_to_end(w):
+    """One sampled step decided by the oracle alone: it fuses the same target states, computes its
+    own draft logits, draws its own tokens and runs its own acceptance on the same Philox streams,
+    and the GPU's drafts, accept lengths and next tokens must equal those decisions. The target
+    logits are built from the oracle's draft logits. A decision is compared exactly unless the
+    oracle's own margin for it lies within what the logit difference between the two sides can
+    move: 2 max|l_gpu - l_oracle| / T for a draw, the matching relative change of q(d) for an
+    acceptance; such borderline decisions must stay rare."""
+    import torch
+    T, seed, step0 = 1.0, 4321, 11
+    s = w.shape
+    B, V, bsz = s.block, s.vocab, w.batch
+    g, step, toks, logits = _sampled_run(w, T, seed, step0)
+    tok_g = toks.cpu().numpy()
+    lg = logits.cpu().numpy().astype(np.float64)
+    o = oracle_for(w, g.W)
+    for b, n in enumerate(w.ctx_lens):
+        o.fuse_context(b, synth.hidden_states(w, b, 0, n))
+    x_t = synth.initial_tokens(w)
+    rng = np.random.default_rng(5)
+    tl = np.empty((bsz, B, V), np.float32)
+    tok_o = np.zeros((bsz, B - 1), np.int64)
+    dl_o, shift, same = [], [], []
+    decided = borderline = 0
+    for b in range(bsz):
+        _, lo, _ = o.draft_block(b, int(x_t[b]))
+        dl_o.append(lo)
+        delta = float(np.max(np.abs(lg[b] - lo))) / T   # largest score shift between the sides
+        shift.append(delta)
+        agree = True
+        for k in range(B - 1):
+            u = O.uniforms(seed, O.RNG_DRAFT, step0, b * (B - 1) + k, V)
+            sc = _scores(lo[k] / T, u)
+            t = int(np.argmax(sc))
+            tok_o[b, k] = t
+            assert t == O.sample_token(lo[k], T, u)
+            gap = sc[t] - float(np.max(np.delete(sc, t)))
+            if gap > 2.0 * delta + MARGIN * (1.0 + abs(sc[t])):
+                assert int(tok_g[b, k]) == t, (b, k, int(tok_g[b, k]), t, gap, delta)
+                decided += 1
+            else:
+                borderline += 1
+                agree = agree and int(tok_g[b, k]) == t
+        same.append(agree)
+        tl[b, :B - 1] = lo / T * rng.uniform(0.7, 1.3) + 0.3 * rng.standard_normal((B - 1, V))
+        tl[b, B - 1] = 2.0 * rng.standard_normal(V)
+        for k in range(B - 1):
+            if rng.random() < 0.15:
+                tl[b, k] = 2.0 * rng.standard_normal(V)
+    assert decided > 0 and borderline <= max(2, (decided + borderline) // 10), (decided, borderline)
+    acc = torch.zeros(bsz, dtype=torch.int32, device="cuda")
+    nxt = torch.zeros(bsz, dtype=torch.int32, device="cuda")
+    g.lib.verify_sampled(toks, torch.from_numpy(tl).cuda(), T, seed, step, acc, nxt)
+    acc_h, nxt_h = acc.cpu().numpy(), nxt.cpu().numpy()
+    assert int(step.item()) == step0 + 1
+    checked = 0
+    for b in range(bsz):
+        if not same[b]:
+            continue                      # a borderline draw went the other way on the GPU
+        r = O.uniforms(seed, O.RNG_ACCEPT, step0, b, B - 1)
+        u = O.uniforms(seed, O.RNG_RESIDUAL, step0, b, V)
+        rel = np.expm1(2.0 * shift[b])    # bound on the relative change of q(d) between the sides
+        a, clear = 0, True
+        while a < B - 1:
+            p = O.softmax_t(tl[b, a], T)
+            q = O.softmax_t(dl_o[b][a], T)
+            d = int(tok_o[b, a])
+            lhs, rhs = r[a] * q[d], p[d]
+            if abs(lhs - rhs) <= (rel + MARGIN) * max(lhs, rhs):
+                clear = False
+                break
+            if lhs < rhs:
+                a += 1
+            else:
+                break
+        if not clear:
+            continue
+        tau, nxt_o = O.speculative_verify(tok_o[b], tl[b], dl_o[b], T, r, u)
+        assert tau == a + 1
+        assert acc_h[b] == tau, (b, acc_h[b], tau)
+        if a < B - 1:
+            # the replacement draws from max(0, p - q): q moves by at most rel q between the sides
+            p = O.softmax_t(tl[b, a], T)
+            q = O.softmax_t(dl_o[b][a], T)
+            wgt = np.maximum(p - q, 0)
+            slack = (rel + 1e-5) * (p + q) / np.maximum(wgt, 1e-30)
+            with np.errstate(divide="ignore"):
+                sc = _scores(np.log(np.maximum(wgt, 1e-300)), u)
+            t_g, t_o = int(nxt_h[b]), int(nxt_o)
+            assert t_g == t_o or sc[t_g] + slack[t_g] >= sc[t_o] - slack[t_o], (b, t_g, t_o)
+        else:
+            with np.errstate(divide="ignore"):
+                ok, _ = _draw_ok(int(nxt_h[b]), np.log(O.softmax_t(tl[b, B - 1], T)), u)
+            assert ok, (b, int(nxt_h[b]), int(nxt_o))
+        checked += 1
+    assert checked >= 1
+    assert g.lib.device_error() == 0
 
 
 def test_first_emitted_token_follows_the_target():
