@@ -198,18 +198,25 @@ constexpr int kRB = 4;          // target rows per stage
 constexpr int kMaxNS = 16;      // most stages in the ring
 constexpr uint64_t kFillWaitNs = 2000000000ull;
 
+__device__ __forceinline__ bool fill_try(uint32_t bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+// Bounded wait; the timer is read only after 64 unsuccessful polls (a %globaltimer read costs a
+// few hundred ns, and most waits of the ring complete within those polls).
 __device__ __forceinline__ bool fill_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+    for (int i = 0; i < 64; ++i)
+        if (fill_try(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (int it = 0;; ++it) {
-        uint32_t done;
-        asm volatile(
-            "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-            "selp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(done)
-            : "r"(bar), "r"(parity)
-            : "memory");
-        if (done) return true;
+        if (fill_try(bar, parity)) return true;
         if ((it & 63) == 63) {
             if (*abort_flag) return false;
             if (globaltimer_ns() - t0 > kFillWaitNs) {
