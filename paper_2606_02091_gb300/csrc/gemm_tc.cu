@@ -734,16 +734,20 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     memset(&a, 0, sizeof(a));
     a.bn = g.m_tok <= 256 ? ((g.m_tok + 15) / 16) * 16 : 256;
     // With token tiles of 128 or more rows the GEMM is bound by the tensor pipeline, not by HBM:
-    // two adjacent 128-row weight tiles then share one activation tile (two accumulators, as the
-    // SwiGLU gate and up tiles do), a third fewer shared-memory bytes per FLOP (d 4096, 8 groups,
-    // 2048 tokens alone: 1197 -> 1316 TFLOP/s; batch-16 step 1.965 -> 1.947 ms). Only for the
-    // epilogues that finish a tile through the staged path, and only while the pairs still give
-    // every SM a unit.
-    a.pair = (!g.a2 && a.bn >= 128 && g.n > kBM && g.force_splits <= 0 &&
-              (g.ep.kind == EPI_STORE || g.ep.kind == EPI_F32 || g.ep.kind == EPI_QKV ||
-               g.ep.kind == EPI_KV_APPEND) &&
-              (long long)g.groups * ((g.n + 2 * kBM - 1) / (2 * kBM)) * ((g.m_tok + a.bn - 1) / a.bn) >=
-                  c->num_sms) ? 1 : 0;
+    // two adjacent 128-row weight tiles can then share one activation tile (two accumulators, as
+    // the SwiGLU gate and up tiles do), a third fewer shared-memory bytes per FLOP. At 256 token
+    // rows the pair fills all 512 TMEM columns, so a unit's epilogue no longer overlaps the next
+    // unit's MMAs: pairs pay only for the cheap epilogues (fp32 logits, plain stores), and only
+    // when their wave count times ~1.8 single-tile units beats the single tiles' wave count.
+    // Measured: batch-16 step 1.965 -> 1.947 ms (the LM head); the context fill's K/V projection
+    // with its rotary epilogue lost (Qwen3-4B shape 822 -> 640 TFLOP/s).
+    {
+        const long long u1 = (long long)g.groups * ((g.n + kBM - 1) / kBM) * ((g.m_tok + a.bn - 1) / a.bn);
+        const long long u2 = (long long)g.groups * ((g.n + 2 * kBM - 1) / (2 * kBM)) * ((g.m_tok + a.bn - 1) / a.bn);
+        const long long w1 = (u1 + c->num_sms - 1) / c->num_sms, w2 = (u2 + c->num_sms - 1) / c->num_sms;
+        a.pair = (!g.a2 && a.bn >= 128 && g.n > kBM && g.force_splits <= 0 &&
+                  (g.ep.kind == EPI_STORE || g.ep.kind == EPI_F32) && 9 * w2 < 5 * w1) ? 1 : 0;
+    }
     a.n_a = (g.a2 || a.pair) ? 2 : 1;
     a.tok_tiles = (g.m_tok + a.bn - 1) / a.bn;
     a.n_tiles = (g.n + (kBM << a.pair) - 1) / (kBM << a.pair);

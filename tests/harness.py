@@ -53,20 +53,20 @@ RAGGED = synth.Workload(
     synth.Shape(d=384, n_draft_layers=2, n_target_layers=3, n_q_heads=4, n_kv_heads=2,
                 head_dim=64, ffn=512, vocab=500, block=8),
     (700, 3, 40), 0.8, seed=21)
-# A context fill long enough that the K/V projection pairs adjacent weight tiles over one token
-# tile (2 layers x 4 pairs x 32 token tiles >= the SM count) and skips the 11 token tiles past
-# the shorter sequence.
+# A context fill over many token tiles (2 layers x 8 weight tiles x 32 token tiles of 256 rows):
+# the K/V projection skips the 11 token tiles past the shorter sequence.
 LONG_FILL = synth.Workload(
     "long_fill_bf16",
     synth.Shape(d=256, n_draft_layers=2, n_target_layers=2, n_q_heads=8, n_kv_heads=4,
                 head_dim=128, ffn=256, vocab=300, block=4),
     (4000, 1200), 0.8, seed=23)
-# 240 LM-head rows (batch 16 x 15 mask positions) over a vocabulary of 157 weight-tile pairs: the
-# LM head pairs its tiles, and the last pair's second tile lies past the matrix.
+# 240 LM-head rows (batch 16 x 15 mask positions) over a vocabulary of 297 weight tiles: the LM
+# head pairs them (149 pairs run in one wave, the single tiles would take two), and the last
+# pair's second tile lies past the matrix.
 WIDE_VOCAB = synth.Workload(
     "wide_vocab_bf16_b16",
     synth.Shape(d=256, n_draft_layers=1, n_target_layers=1, n_q_heads=4, n_kv_heads=2,
-                head_dim=64, ffn=256, vocab=40000, block=16),
+                head_dim=64, ffn=256, vocab=38000, block=16),
     tuple(5 + (13 * b) % 29 for b in range(16)), 0.8, seed=25)
 D10 = synth.Workload(
     "d10_bf16",
