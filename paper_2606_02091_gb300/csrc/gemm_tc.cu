@@ -7,8 +7,10 @@
 // 128-row UMMA M dimension runs over weight rows (output features) and the small token count is
 // the UMMA N dimension (16..256), so one instruction covers a 128 x bn x 16 piece.
 //
-// Work unit = (group, 128-feature tile, token tile, K split). A persistent grid of one CTA per SM
-// walks the units. Per CTA (192 threads):
+// Work unit = (group, 128-feature tile, token tile, K split); with token tiles of 128+ rows and a
+// cheap epilogue, a pair of adjacent 128-feature tiles (two accumulators over one activation
+// tile); a context fill's units run only over the token tiles that hold appended rows. A
+// persistent grid of one CTA per SM walks the units. Per CTA (192 threads):
 //   warp 4    TMA producer: per stage, kbs consecutive 128x64 bf16 weight tiles (+ the up tiles
 //             for SwiGLU) and the matching bn x 64 activation tiles, 128-byte swizzled; weights
 //             carry an L2 evict-first hint (each byte is read once per step). Weights do not
