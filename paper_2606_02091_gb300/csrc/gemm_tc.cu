@@ -7,9 +7,9 @@
 // 128-row UMMA M dimension runs over weight rows (output features) and the small token count is
 // the UMMA N dimension (16..256), so one instruction covers a 128 x bn x 16 piece.
 //
-// Work unit = (group, 128-feature tile, token tile, K split); with token tiles of 128+ rows and a
-// cheap epilogue, a pair of adjacent 128-feature tiles (two accumulators over one activation
-// tile); a context fill's units run only over the token tiles that hold appended rows. A
+// Work unit = (group, 128-feature tile, token tile, K split); for an LM head over 128+ token rows,
+// a pair of adjacent 128-feature tiles (two accumulators over one activation tile); a context
+// fill's units run only over the token tiles that hold appended rows. A
 // persistent grid of one CTA per SM walks the units. Per CTA (192 threads):
 //   warp 4    TMA producer: per stage, kbs consecutive 128x64 bf16 weight tiles (+ the up tiles
 //             for SwiGLU) and the matching bn x 64 activation tiles, 128-byte swizzled; weights
@@ -739,8 +739,8 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
     // two adjacent 128-row weight tiles can then share one activation tile (two accumulators, as
     // the SwiGLU gate and up tiles do), a third fewer shared-memory bytes per FLOP. At 256 token
     // rows the pair fills all 512 TMEM columns, so a unit's epilogue no longer overlaps the next
-    // unit's MMAs: pairs pay only for the cheap epilogues (fp32 logits, plain stores), and only
-    // when their wave count times ~1.8 single-tile units beats the single tiles' wave count.
+    // unit's MMAs: pairs pay only for the cheap fp32-logit epilogue (the LM head), and only when
+    // their wave count times ~1.8 single-tile units beats the single tiles' wave count.
     // Measured: batch-16 step 1.965 -> 1.947 ms (the LM head); the context fill's K/V projection
     // with its rotary epilogue lost (Qwen3-4B shape 822 -> 640 TFLOP/s).
     {
@@ -748,7 +748,7 @@ cudaError_t launch_gemm_tc(dflare_ctx* c, const GemmDesc& g, cudaStream_t s, std
         const long long u2 = (long long)g.groups * ((g.n + 2 * kBM - 1) / (2 * kBM)) * ((g.m_tok + a.bn - 1) / a.bn);
         const long long w1 = (u1 + c->num_sms - 1) / c->num_sms, w2 = (u2 + c->num_sms - 1) / c->num_sms;
         a.pair = (!g.a2 && a.bn >= 128 && g.n > kBM && g.force_splits <= 0 &&
-                  (g.ep.kind == EPI_STORE || g.ep.kind == EPI_F32) && 9 * w2 < 5 * w1) ? 1 : 0;
+                  g.ep.kind == EPI_F32 && 9 * w2 < 5 * w1) ? 1 : 0;
     }
     a.n_a = (g.a2 || a.pair) ? 2 : 1;
     a.tok_tiles = (g.m_tok + a.bn - 1) / a.bn;
